@@ -1,0 +1,205 @@
+/*
+ * semshare_oracle.c -- CPU oracle for SemShareKV's fuzzy token-matching path.
+ *
+ * TEST INFRASTRUCTURE ONLY.  The tests, the smoke check and the bench's CPU-baseline leg
+ * are the only callers.  The product path (the CUDA library) never calls, links or loads
+ * this file, and this file shares no code, header, table or helper with it.
+ *
+ * It is a plain, slow restatement of what the path computes, in fp64, one step at a time,
+ * in the paper's order (SemShareKV, arXiv 2509.24832):
+ *
+ *   1. rope    Rotary position encoding of every embedding row (Sec. 3.3.1: RoPE is applied
+ *              to the E cache of both the reference and the target prompt; formula Eq. 1,
+ *              App. A.1).  Pair (x[2k], x[2k+1]) of the row at position m is rotated by the
+ *              angle m * theta_k, theta_k = base^(-2k/d), d = the embedding dimension.
+ *   2. hash    Random-hyperplane LSH (Sec. 3.3 "we use LSH", App. A.2, App. D "LSH from
+ *              FAISS"): p_j = <r_j, y> for each of nbits hyperplanes r_j, code bit j = [p_j > 0],
+ *              packed LSB-first into 32-bit words (bit j -> word j/32, bit j%32).
+ *              Operand contract: y is rounded to bf16 (nearest, ties to even) before the
+ *              products, the hyperplanes are bf16; the dot product is accumulated in fp64.
+ *   3. match   For each target token the reference token with the smallest Hamming distance
+ *              between codes (Sec. 3.3: "for each token in the target prompt, the most similar
+ *              token in the reference prompt"); an exhaustive scan in ascending reference
+ *              order that keeps the first minimum, so ties go to the lowest index.
+ *   4. gather  The reordered cache has the target's length and every row comes from the
+ *              reference cache (Sec. 3.3): out[b][l][h][t] = ref[l][h][idx[b][t]] for every
+ *              layer l and KV head h, copied bit for bit (Sec. 3.3.2: KV is stored after RoPE,
+ *              so nothing is re-encoded).
+ *
+ * Build: gcc -O2 -fopenmp -ffp-contract=off -shared -fPIC (no fused multiply-add, so x86 and
+ * Arm hosts produce the same bits).
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+int oracle_num_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+/* ---- bf16 <-> fp64 --------------------------------------------------------------------- */
+
+/* Value of a bf16 bit pattern (exact). */
+double oracle_bf16_value(uint16_t h) {
+    uint32_t u = (uint32_t)h << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+/* Nearest bf16 to v, ties to even, rounded once from the fp64 value.
+ * (float)v is rounded first; that second rounding can only differ from the direct one when
+ * (float)v lands exactly on a bf16 midpoint while v itself does not, and then the side v
+ * lies on decides. */
+uint16_t oracle_bf16_round(double v) {
+    if (v != v) return (uint16_t)0x7FC0u;
+    float f = (float)v;
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    if ((u & 0xFFFFu) == 0x8000u && (double)f != v && !isinf(f))
+        return (uint16_t)((u >> 16) + (fabs(v) > fabs((double)f) ? 1u : 0u));
+    u += 0x7FFFu + ((u >> 16) & 1u);
+    return (uint16_t)(u >> 16);
+}
+
+/* ---- step 1: rotary position encoding (Eq. 1) ----------------------------------------- */
+
+/* theta_k = base^(-2k/d), the rotation frequency of pair k (Eq. 1, App. A.1). */
+double oracle_theta(int32_t k, int32_t d, double base) {
+    return pow(base, -2.0 * (double)k / (double)d);
+}
+
+static void rope_row(const double* x, int32_t d, double m, const double* theta, double* y) {
+    for (int32_t k = 0; k < d / 2; ++k) {
+        const double a = m * theta[k];
+        const double c = cos(a), s = sin(a);
+        const double x0 = x[2 * k], x1 = x[2 * k + 1];
+        y[2 * k] = x0 * c - x1 * s;
+        y[2 * k + 1] = x0 * s + x1 * c;
+    }
+}
+
+/* y[i] = RoPE(x[i], pos[i]) for n rows of width d (row-major, fp64). */
+void oracle_rope(const double* x, int64_t n, int32_t d, const int32_t* pos, double base, double* y) {
+    double* theta = (double*)malloc(sizeof(double) * (size_t)(d / 2));
+    for (int32_t k = 0; k < d / 2; ++k) theta[k] = oracle_theta(k, d, base);
+#pragma omp parallel for schedule(static)
+    for (int64_t i = 0; i < n; ++i)
+        rope_row(x + i * d, d, (double)pos[i], theta, y + i * d);
+    free(theta);
+}
+
+/* ---- step 2: random-hyperplane LSH codes ----------------------------------------------- */
+
+/* emb: n rows of d values, row i starting at element i*row_stride; emb_f32 = 1 for float32
+ * rows, 0 for bf16 bit patterns.  positions: n token positions (NULL -> 0..n-1).
+ * hyperplanes: [nbits][d] bf16 bit patterns.  codes: [n][nbits/32] words.
+ * proj (nullable): [n][nbits] float projections (the fp64 sum rounded to float).
+ * round_operand = 1 applies the bf16 operand contract to y; 0 keeps y in fp64 (diagnostic). */
+void oracle_hash(const void* emb, int32_t emb_f32, int64_t n, int32_t d, int64_t row_stride,
+                 const int32_t* positions, double base, const uint16_t* hyperplanes, int32_t nbits,
+                 uint32_t* codes, float* proj, int32_t round_operand) {
+    const int32_t w = nbits / 32;
+    double* theta = (double*)malloc(sizeof(double) * (size_t)(d / 2));
+    double* r = (double*)malloc(sizeof(double) * (size_t)nbits * (size_t)d);
+    for (int32_t k = 0; k < d / 2; ++k) theta[k] = oracle_theta(k, d, base);
+    for (int64_t e = 0; e < (int64_t)nbits * d; ++e) r[e] = oracle_bf16_value(hyperplanes[e]);
+
+#pragma omp parallel
+    {
+        double* x = (double*)malloc(sizeof(double) * (size_t)d);
+        double* y = (double*)malloc(sizeof(double) * (size_t)d);
+#pragma omp for schedule(dynamic, 16)
+        for (int64_t i = 0; i < n; ++i) {
+            for (int32_t c = 0; c < d; ++c)
+                x[c] = emb_f32 ? (double)((const float*)emb)[i * row_stride + c]
+                               : oracle_bf16_value(((const uint16_t*)emb)[i * row_stride + c]);
+            const double m = positions ? (double)positions[i] : (double)i;
+            rope_row(x, d, m, theta, y);
+            if (round_operand)
+                for (int32_t c = 0; c < d; ++c) y[c] = oracle_bf16_value(oracle_bf16_round(y[c]));
+            for (int32_t q = 0; q < w; ++q) codes[i * w + q] = 0u;
+            for (int32_t j = 0; j < nbits; ++j) {
+                double p = 0.0;
+                for (int32_t c = 0; c < d; ++c) p += r[(int64_t)j * d + c] * y[c];
+                if (p > 0.0) codes[i * w + j / 32] |= 1u << (j % 32);
+                if (proj) proj[i * nbits + j] = (float)p;
+            }
+        }
+        free(x);
+        free(y);
+    }
+    free(theta);
+    free(r);
+}
+
+/* ---- step 3: Hamming nearest neighbour ------------------------------------------------- */
+
+/* Hamming distance between two packed codes of w words. */
+int32_t oracle_hamming(const uint32_t* a, const uint32_t* b, int32_t w) {
+    int32_t s = 0;
+    for (int32_t q = 0; q < w; ++q) s += __builtin_popcount(a[q] ^ b[q]);
+    return s;
+}
+
+/* idx[t] = the lowest j minimising hamming(tgt[t], ref[j]); dist[t] = that minimum. */
+void oracle_match(const uint32_t* tgt, int64_t n_tgt, const uint32_t* ref, int64_t n_ref, int32_t nbits,
+                  int32_t* idx, int32_t* dist) {
+    const int32_t w = nbits / 32;
+#pragma omp parallel for schedule(dynamic, 64)
+    for (int64_t t = 0; t < n_tgt; ++t) {
+        int32_t best = nbits + 1;
+        int64_t best_j = -1;
+        for (int64_t j = 0; j < n_ref; ++j) {
+            const int32_t h = oracle_hamming(tgt + t * w, ref + j * w, w);
+            if (h < best) {
+                best = h;
+                best_j = j;
+            }
+        }
+        idx[t] = (int32_t)best_j;
+        dist[t] = best;
+    }
+}
+
+/* ---- step 4: KV rearrangement ---------------------------------------------------------- */
+
+/* Reference cache: n_seg segments (one per reference prompt); segment s holds the global rows
+ * seg_offsets[s] <= r < seg_offsets[s+1] as its local rows r - seg_offsets[s], laid out
+ * [L][H][n_s][row_bytes] with n_s = seg_offsets[s+1] - seg_offsets[s].
+ * idx: [n_batch][n_tgt] global rows.  out_k/out_v: [n_batch][L][H][n_tgt][row_bytes].
+ * A row whose idx is outside [0, seg_offsets[n_seg]) is left untouched and counted.
+ * Returns the number of such rows (per batch and target token). */
+int64_t oracle_gather_kv(const uint8_t* const* seg_k, const uint8_t* const* seg_v, const int64_t* seg_offsets,
+                         int32_t n_seg, int32_t L, int32_t H, int64_t row_bytes, const int32_t* idx, int64_t n_tgt,
+                         int32_t n_batch, uint8_t* out_k, uint8_t* out_v) {
+    const int64_t total = seg_offsets[n_seg];
+    int64_t bad = 0;
+    for (int64_t e = 0; e < (int64_t)n_batch * n_tgt; ++e)
+        if (idx[e] < 0 || idx[e] >= total) ++bad;
+#pragma omp parallel for collapse(2) schedule(static)
+    for (int32_t b = 0; b < n_batch; ++b)
+        for (int32_t l = 0; l < L; ++l)
+            for (int32_t h = 0; h < H; ++h)
+                for (int64_t t = 0; t < n_tgt; ++t) {
+                    const int64_t r = idx[(int64_t)b * n_tgt + t];
+                    if (r < 0 || r >= total) continue;
+                    int32_t s = 0;
+                    while (!(seg_offsets[s] <= r && r < seg_offsets[s + 1])) ++s;
+                    const int64_t n_s = seg_offsets[s + 1] - seg_offsets[s];
+                    const int64_t src_row = ((int64_t)l * H + h) * n_s + (r - seg_offsets[s]);
+                    const int64_t dst_row = (((int64_t)b * L + l) * H + h) * n_tgt + t;
+                    memcpy(out_k + dst_row * row_bytes, seg_k[s] + src_row * row_bytes, (size_t)row_bytes);
+                    memcpy(out_v + dst_row * row_bytes, seg_v[s] + src_row * row_bytes, (size_t)row_bytes);
+                }
+    return bad;
+}
