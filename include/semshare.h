@@ -1,0 +1,189 @@
+/*
+ * semshare.h -- C ABI of the GB300 (sm_103a) fuzzy token-matching library.
+ *
+ * SemShareKV (arXiv 2509.24832) lets a target prompt reuse the KV cache of a semantically
+ * similar reference prompt.  Its matching path (Sec. 3.2, Sec. 3.3) has four steps:
+ * rotary position encoding of both prompts' embedding rows (Sec. 3.3.1, Eq. 1), locality
+ * sensitive hashing of the rotated rows (Sec. 3.3, App. A.2), a per-token nearest-neighbour
+ * match of every target token to a reference token (Sec. 3.3), and a rearrangement of the
+ * reference K/V cache to the target's token order (Sec. 3.3, Sec. 3.3.2).  This library
+ * exposes them as three calls, semshare_hash (steps 1-2), semshare_match (step 3) and
+ * semshare_gather_kv (step 4), plus semshare_rope_table, which precomputes the per-pair
+ * rotation frequencies that semshare_hash consumes.
+ *
+ * Conventions shared by every call:
+ *   - Buffers are owned by the caller.  Pointers marked "device" point to memory of the
+ *     current CUDA device; "host" marks host memory read during the call only.  No call
+ *     allocates or frees memory, and the library keeps no state between calls.
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream).  Work is enqueued on it
+ *     and runs asynchronously; a call returns once the work is enqueued.
+ *   - Argument errors are detected on the host before anything is enqueued and returned as
+ *     SEMSHARE_EINVAL / SEMSHARE_EUNSUPPORTED; nothing is launched in that case.  A failed
+ *     launch returns SEMSHARE_ECUDA.
+ *   - Errors found by a kernel while it runs are OR-ed into an optional device word
+ *     `err_flag` (SEMSHARE_FLAG_*); the caller reads it after synchronising and may turn it
+ *     into a status with semshare_flag_status().  Kernels never trap.
+ *   - Results are deterministic: the same inputs give the same bits on every run.
+ */
+#ifndef SEMSHARE_H
+#define SEMSHARE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SEMSHARE_ABI_VERSION 1
+
+typedef enum {
+    SEMSHARE_OK = 0,
+    SEMSHARE_EINVAL = 1,        /* null / misaligned pointer, bad size or stride */
+    SEMSHARE_EUNSUPPORTED = 2,  /* valid request outside what the kernels implement */
+    SEMSHARE_ECUDA = 3,         /* a CUDA runtime or driver call failed */
+    SEMSHARE_EINDEX = 4,        /* a kernel met an index outside its table (from err_flag) */
+    SEMSHARE_ETIMEOUT = 5       /* a kernel pipeline wait hit its time limit (from err_flag) */
+} semshare_status;
+
+typedef enum { SEMSHARE_BF16 = 0, SEMSHARE_F32 = 1 } semshare_dtype;
+
+/* Bits a kernel ORs into `err_flag`. */
+#define SEMSHARE_FLAG_INDEX 1u
+#define SEMSHARE_FLAG_TIMEOUT 2u
+
+/* Human-readable name of a status. */
+const char* semshare_status_string(semshare_status s);
+
+/* Maps the err_flag bits read back by the caller to a status (TIMEOUT wins over INDEX). */
+semshare_status semshare_flag_status(uint32_t flags);
+
+/* SEMSHARE_ABI_VERSION of the loaded library. */
+int32_t semshare_abi_version(void);
+
+/*
+ * semshare_rope_table -- rotation frequencies of Eq. 1 (App. A.1) in fixed point.
+ *
+ * Pair k of a d-wide embedding row turns by theta_k = rope_base^(-2k/d) radians per position
+ * (Eq. 1; the angle at position m is m * theta_k, Sec. 3.3.1).  table[k] receives
+ * frac(theta_k / (2*pi)) * 2^64 rounded: the turns per position modulo one turn as an
+ * unsigned 0.64 fixed-point fraction, so a kernel gets the angle of position m modulo a full
+ * turn from the low 64 bits of m * table[k] with integer arithmetic.  Computed on the device
+ * in double precision.
+ *
+ *   d          embedding dimension, even, 2 <= d <= 65536
+ *   rope_base  the RoPE base (10000 in Eq. 1), finite and > 0
+ *   table      device, d/2 uint64 words, 8-byte aligned; written
+ * Returns EINVAL for a bad d, base or pointer.  The table depends only on (d, rope_base):
+ * compute it once and reuse it for every semshare_hash call.
+ */
+semshare_status semshare_rope_table(int32_t d, double rope_base, uint64_t* table, void* stream);
+
+/*
+ * semshare_hash -- steps 1-2: rotary encoding + random-hyperplane LSH codes.
+ *
+ * For each row i (Sec. 3.3.1: RoPE is applied to the E cache of both prompts, then LSH):
+ *   y = RoPE(emb[i], positions[i])       Eq. 1, pairs (2k, 2k+1), angle positions[i]*theta_k
+ *   p_j = <hyperplanes[j], bf16(y)>      fp32 accumulation on the tensor cores
+ *   bit j of codes[i] = [p_j > 0]         sign random projection (App. A.2, App. D: LSH)
+ * y is computed in fp32 and rounded to bf16 (nearest even) before the products.
+ *
+ *   emb         device, n rows of d elements of `dtype`, row i at element offset i*row_stride;
+ *               16-byte aligned base, row_stride*element_size a multiple of 16 bytes
+ *   dtype       SEMSHARE_BF16 or SEMSHARE_F32
+ *   n           rows (0 is allowed: nothing is launched); n < 2^31
+ *   d           embedding dimension, a multiple of 64, 64 <= d <= 65536
+ *   row_stride  elements between consecutive rows, >= d
+ *   positions   device, n int32 token positions >= 0, or NULL for positions 0..n-1.  Each
+ *               prompt uses its own 0-based positions; rows of several prompts may be hashed
+ *               in one call by passing each row's position.
+ *   rope_table  device, d/2 words from semshare_rope_table(d, base, ...)
+ *   hyperplanes device, [nbits][d] bf16 bit patterns, row-major, 16-byte aligned
+ *   nbits       code length: 32, 64, ..., 256
+ *   codes       device, [n][nbits/32] uint32, bit j of row i in word j/32 at bit j%32; written
+ *   proj_out    device or NULL; if given, [n][nbits] float32 projections p_j are written too
+ *   err_flag    device or NULL; SEMSHARE_FLAG_TIMEOUT is OR-ed in if a pipeline wait of the
+ *               kernel exceeds its limit (the kernel then stops and leaves codes incomplete)
+ * Returns EINVAL / EUNSUPPORTED for bad arguments, ECUDA if the launch fails.
+ */
+semshare_status semshare_hash(const void* emb, semshare_dtype dtype, int64_t n, int32_t d, int64_t row_stride,
+                              const int32_t* positions, const uint64_t* rope_table, const uint16_t* hyperplanes,
+                              int32_t nbits, uint32_t* codes, float* proj_out, uint32_t* err_flag, void* stream);
+
+/*
+ * semshare_match -- step 3: Hamming nearest reference token of every target token.
+ *
+ * Sec. 3.3: "for each token in the target prompt, the most similar token in the reference
+ * prompt".  idx[t] = the lowest j minimising popcount(tgt_codes[t] XOR ref_codes[j]) over
+ * 0 <= j < n_ref; dist[t] = that minimum.  Ties go to the lowest reference index, so the
+ * result does not depend on how the search is split across the GPU.  A pool of reference
+ * prompts is searched by concatenating their codes; idx is then the global pool row.
+ *
+ *   tgt_codes  device, [n_tgt][nbits/32] uint32, 16-byte aligned
+ *   n_tgt      target rows, 0 <= n_tgt < 2^31 (0: nothing is launched)
+ *   ref_codes  device, [n_ref][nbits/32] uint32, 16-byte aligned
+ *   n_ref      reference rows, 1 <= n_ref < 2^31
+ *   nbits      32, 64, ..., 256
+ *   idx        device, [n_tgt] int32; written
+ *   dist       device, [n_tgt] int32, or NULL; written
+ *   workspace  device scratch of at least semshare_match_workspace_size(n_tgt) bytes,
+ *              8-byte aligned; its contents on entry do not matter and are overwritten
+ * Returns EINVAL / EUNSUPPORTED for bad arguments, ECUDA if a launch fails.
+ */
+size_t semshare_match_workspace_size(int64_t n_tgt);
+semshare_status semshare_match(const uint32_t* tgt_codes, int64_t n_tgt, const uint32_t* ref_codes, int64_t n_ref,
+                               int32_t nbits, int32_t* idx, int32_t* dist, void* workspace, size_t workspace_bytes,
+                               void* stream);
+
+/*
+ * Layout of a K or V cache: element (b, l, h, t, e) of a cache with this layout lives at
+ * element offset b*stride_batch + l*stride_layer + h*stride_head + t*stride_token + e.
+ * A row (fixed b, l, h, t) holds head_dim contiguous elements of elem_bytes bytes.
+ */
+typedef struct {
+    int32_t n_layers;     /* L */
+    int32_t n_heads;      /* KV heads H */
+    int32_t head_dim;     /* elements per row */
+    int32_t elem_bytes;   /* 2 for bf16/fp16, 4 for fp32 */
+    int64_t stride_batch; /* elements; ignored for the reference cache */
+    int64_t stride_layer;
+    int64_t stride_head;
+    int64_t stride_token;
+} semshare_kv_layout;
+
+/*
+ * semshare_gather_kv -- step 4: rearrange the reference K/V cache to the target's order.
+ *
+ * Sec. 3.3: the reordered cache matches the target prompt's length and its key-value pairs
+ * all come from the reference cache; Sec. 3.3.2: K/V are stored after RoPE, so rows are
+ * copied bit for bit with no re-encoding.  For every target prompt b < n_batch, layer l,
+ * KV head h and target token t < n_tgt:
+ *     out_k[b][l][h][t][:] = ref_k[l][h][idx[b*n_tgt + t]][:]      (same for V)
+ *
+ *   ref_k, ref_v   host arrays of n_seg device base pointers, one reference prompt each.
+ *                  Global reference row r belongs to the segment s with
+ *                  seg_offsets[s] <= r < seg_offsets[s+1] and is its local row
+ *                  r - seg_offsets[s].  Every segment uses the strides of `src`.
+ *   seg_offsets    host, n_seg+1 ascending int64 values, seg_offsets[0] = 0
+ *   n_seg          1 <= n_seg <= 64
+ *   src            layout of every reference segment (stride_batch ignored)
+ *   idx            device, [n_batch][n_tgt] int32 global reference rows (from semshare_match)
+ *   n_tgt, n_batch target tokens per prompt and prompts; 0 of either launches nothing
+ *   out_k, out_v   device destination caches with layout `dst`
+ *   dst            layout of the destination (same n_layers, n_heads, head_dim, elem_bytes)
+ *   err_flag       device or NULL; a row whose idx lies outside [0, seg_offsets[n_seg]) is
+ *                  not written and SEMSHARE_FLAG_INDEX is OR-ed in
+ * Every base pointer and every stride (in bytes) must be a multiple of 16, and
+ * head_dim*elem_bytes a multiple of 16: rows move as 16-byte vectors.
+ * Returns EINVAL for bad arguments, ECUDA if the launch fails.
+ */
+semshare_status semshare_gather_kv(const void* const* ref_k, const void* const* ref_v, const int64_t* seg_offsets,
+                                   int32_t n_seg, semshare_kv_layout src, const int32_t* idx, int64_t n_tgt,
+                                   int32_t n_batch, void* out_k, void* out_v, semshare_kv_layout dst,
+                                   uint32_t* err_flag, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SEMSHARE_H */

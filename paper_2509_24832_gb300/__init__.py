@@ -1,0 +1,28 @@
+"""GB300-native (sm_103a) fuzzy token matching for SemShareKV (arXiv 2509.24832).
+
+The path: rotary position encoding of the embedding rows of a target and a reference prompt
+(Sec. 3.3.1, Eq. 1), random-hyperplane LSH sign codes (Sec. 3.3, App. A.2), the Hamming
+nearest reference token of every target token (Sec. 3.3), and the rearrangement of the
+reference K/V cache into the target's order (Sec. 3.3, Sec. 3.3.2).
+
+The compute lives in libsemshare.so (C ABI: include/semshare.h); this package is its thin
+ctypes binding with the same names.  Build the library with `paper_2509_24832_gb300.build`."""
+from ._native import (  # noqa: F401
+    FLAG_INDEX,
+    FLAG_TIMEOUT,
+    KVLayout,
+    LIB_PATH,
+    SemshareError,
+    check_flag,
+    flag_status,
+    kv_layout,
+    load,
+    new_err_flag,
+    semshare_abi_version,
+    semshare_gather_kv,
+    semshare_hash,
+    semshare_match,
+    semshare_match_workspace_size,
+    semshare_rope_table,
+    status_string,
+)

@@ -1,0 +1,249 @@
+"""ctypes binding of libsemshare.so (the C ABI declared in include/semshare.h).
+
+Argument marshalling only: every step of the path runs in the library's CUDA kernels.
+PyTorch supplies device memory and the current stream.  There is no fallback: if the
+library is missing the call raises."""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "_lib", "libsemshare.so")
+
+OK, EINVAL, EUNSUPPORTED, ECUDA, EINDEX, ETIMEOUT = range(6)
+FLAG_INDEX, FLAG_TIMEOUT = 1, 2
+BF16, F32 = 0, 1
+
+_lock = threading.Lock()
+_lib = None
+
+
+class SemshareError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} (status {status})")
+
+
+class KVLayout(ctypes.Structure):
+    """semshare_kv_layout: element (b, l, h, t, e) at b*stride_batch + l*stride_layer +
+    h*stride_head + t*stride_token + e (strides in elements)."""
+    _fields_ = [("n_layers", ctypes.c_int32), ("n_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("elem_bytes", ctypes.c_int32), ("stride_batch", ctypes.c_int64), ("stride_layer", ctypes.c_int64),
+                ("stride_head", ctypes.c_int64), ("stride_token", ctypes.c_int64)]
+
+
+def load():
+    """Loads libsemshare.so (built in-tree by paper_2509_24832_gb300.build)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it first (python -c 'import __graft_entry__ as g; g.build()')")
+        lib = ctypes.CDLL(LIB_PATH)
+        P, i32, i64, u32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32
+        lib.semshare_status_string.argtypes = [ctypes.c_int]
+        lib.semshare_status_string.restype = ctypes.c_char_p
+        lib.semshare_flag_status.argtypes = [u32]
+        lib.semshare_flag_status.restype = ctypes.c_int
+        lib.semshare_abi_version.restype = i32
+        lib.semshare_rope_table.argtypes = [i32, ctypes.c_double, P, P]
+        lib.semshare_rope_table.restype = ctypes.c_int
+        lib.semshare_hash.argtypes = [P, ctypes.c_int, i64, i32, i64, P, P, P, i32, P, P, P, P]
+        lib.semshare_hash.restype = ctypes.c_int
+        lib.semshare_match_workspace_size.argtypes = [i64]
+        lib.semshare_match_workspace_size.restype = ctypes.c_size_t
+        lib.semshare_match.argtypes = [P, i64, P, i64, i32, P, P, P, ctypes.c_size_t, P]
+        lib.semshare_match.restype = ctypes.c_int
+        lib.semshare_gather_kv.argtypes = [P, P, P, i32, KVLayout, P, i64, i32, P, P, KVLayout, P, P]
+        lib.semshare_gather_kv.restype = ctypes.c_int
+        _lib = lib
+        return lib
+
+
+def status_string(status: int) -> str:
+    try:
+        return load().semshare_status_string(int(status)).decode()
+    except RuntimeError:
+        return f"status {status}"
+
+
+def _check(status: int, where: str):
+    if status != OK:
+        raise SemshareError(status, where)
+
+
+def _ptr(t: torch.Tensor | None):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _need_cuda(t: torch.Tensor, name: str):
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+
+
+def new_err_flag(device=None) -> torch.Tensor:
+    """A zeroed device word for the kernels' error bits."""
+    return torch.zeros(1, dtype=torch.int32, device=device or "cuda")
+
+
+def flag_status(err_flag: torch.Tensor) -> int:
+    """Reads an error word back (synchronising on it) and maps its bits to a status."""
+    return int(load().semshare_flag_status(int(err_flag.item()) & 0xFFFFFFFF))
+
+
+def check_flag(err_flag: torch.Tensor, where: str = "kernel"):
+    _check(flag_status(err_flag), where)
+
+
+def semshare_abi_version() -> int:
+    return int(load().semshare_abi_version())
+
+
+def semshare_rope_table(d: int, rope_base: float = 10000.0, out: torch.Tensor | None = None, device=None,
+                        stream=None) -> torch.Tensor:
+    """Fixed-point rotation frequencies for semshare_hash: [d/2] uint64 words (int64 storage)."""
+    if out is None:
+        out = torch.empty(d // 2, dtype=torch.int64, device=device or "cuda")
+    _need_cuda(out, "out")
+    _check(load().semshare_rope_table(int(d), float(rope_base), _ptr(out), _stream(stream)), "semshare_rope_table")
+    return out
+
+
+def semshare_hash(emb: torch.Tensor, rope_table: torch.Tensor, hyperplanes: torch.Tensor,
+                  positions: torch.Tensor | None = None, codes: torch.Tensor | None = None,
+                  proj_out: torch.Tensor | None = None, err_flag: torch.Tensor | None = None,
+                  stream=None) -> torch.Tensor:
+    """LSH codes of RoPE-encoded rows.  emb [n][d] bf16/fp32 (rows may be strided),
+    hyperplanes [nbits][d] bf16, positions [n] int32 (None: 0..n-1).
+    Returns codes [n][nbits/32] int32 (uint32 bit patterns)."""
+    _need_cuda(emb, "emb")
+    _need_cuda(hyperplanes, "hyperplanes")
+    if emb.dim() != 2 or emb.stride(1) != 1:
+        raise ValueError("emb must be [n][d] with unit stride along d")
+    if emb.dtype == torch.bfloat16:
+        dt = BF16
+    elif emb.dtype == torch.float32:
+        dt = F32
+    else:
+        raise ValueError("emb must be bfloat16 or float32")
+    if hyperplanes.dtype != torch.bfloat16 or not hyperplanes.is_contiguous():
+        raise ValueError("hyperplanes must be contiguous bfloat16 [nbits][d]")
+    n, d = emb.shape
+    nbits = hyperplanes.shape[0]
+    if hyperplanes.shape[1] != d:
+        raise ValueError("hyperplanes width differs from emb")
+    if positions is not None:
+        if positions.dtype != torch.int32 or positions.numel() != n or not positions.is_contiguous():
+            raise ValueError("positions must be contiguous int32 [n]")
+    if codes is None:
+        codes = torch.empty((n, nbits // 32), dtype=torch.int32, device=emb.device)
+    st = load().semshare_hash(_ptr(emb), dt, n, d, emb.stride(0), _ptr(positions), _ptr(rope_table),
+                              _ptr(hyperplanes), nbits, _ptr(codes), _ptr(proj_out), _ptr(err_flag), _stream(stream))
+    _check(st, "semshare_hash")
+    return codes
+
+
+def semshare_match_workspace_size(n_tgt: int) -> int:
+    return int(load().semshare_match_workspace_size(int(n_tgt)))
+
+
+def semshare_match(tgt_codes: torch.Tensor, ref_codes: torch.Tensor, idx: torch.Tensor | None = None,
+                   dist: torch.Tensor | None = None, workspace: torch.Tensor | None = None, nbits: int | None = None,
+                   stream=None):
+    """Hamming nearest reference row per target row (ties to the lowest index).
+    Returns (idx int32 [n_tgt], dist int32 [n_tgt])."""
+    _need_cuda(tgt_codes, "tgt_codes")
+    _need_cuda(ref_codes, "ref_codes")
+    if not tgt_codes.is_contiguous() or not ref_codes.is_contiguous():
+        raise ValueError("codes must be contiguous")
+    n_tgt, w = tgt_codes.shape
+    n_ref = ref_codes.shape[0]
+    if ref_codes.shape[1] != w:
+        raise ValueError("code widths differ")
+    nbits = 32 * w if nbits is None else nbits
+    dev = tgt_codes.device
+    if idx is None:
+        idx = torch.empty(n_tgt, dtype=torch.int32, device=dev)
+    if dist is None:
+        dist = torch.empty(n_tgt, dtype=torch.int32, device=dev)
+    ws_bytes = semshare_match_workspace_size(n_tgt)
+    if workspace is None:
+        workspace = torch.empty(max(ws_bytes, 8), dtype=torch.uint8, device=dev)
+    st = load().semshare_match(_ptr(tgt_codes), n_tgt, _ptr(ref_codes), n_ref, nbits, _ptr(idx), _ptr(dist),
+                               _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream))
+    _check(st, "semshare_match")
+    return idx, dist
+
+
+def kv_layout(t: torch.Tensor, batched: bool) -> KVLayout:
+    """Layout of a [B][L][H][T][hd] (batched) or [L][H][T][hd] cache tensor."""
+    if t.stride(-1) != 1:
+        raise ValueError("head_dim must be contiguous")
+    if batched:
+        if t.dim() != 5:
+            raise ValueError("expected [n_batch][L][H][T][head_dim]")
+        sb, sl, sh, st = t.stride(0), t.stride(1), t.stride(2), t.stride(3)
+        L, H, hd = t.shape[1], t.shape[2], t.shape[4]
+    else:
+        if t.dim() != 4:
+            raise ValueError("expected [L][H][T][head_dim]")
+        sb, (sl, sh, st) = 0, t.stride()[:3]
+        L, H, hd = t.shape[0], t.shape[1], t.shape[3]
+    return KVLayout(L, H, hd, t.element_size(), sb, sl, sh, st)
+
+
+def semshare_gather_kv(ref_k, ref_v, idx: torch.Tensor, out_k: torch.Tensor | None = None,
+                       out_v: torch.Tensor | None = None, err_flag: torch.Tensor | None = None, stream=None):
+    """Reordered K/V cache: out[b][l][h][t] = ref[l][h][idx[b][t]].
+
+    ref_k/ref_v: a [L][H][N][hd] CUDA tensor, or a list of them (a pool of reference prompts
+    with identical strides; global row r = running offset of its segment + local row).
+    idx: [n_batch][n_tgt] or [n_tgt] int32.  Returns (out_k, out_v), [n_batch][L][H][n_tgt][hd]."""
+    seg_k = list(ref_k) if isinstance(ref_k, (list, tuple)) else [ref_k]
+    seg_v = list(ref_v) if isinstance(ref_v, (list, tuple)) else [ref_v]
+    if len(seg_k) != len(seg_v) or not seg_k:
+        raise ValueError("ref_k and ref_v must have the same number of segments")
+    for t in seg_k + seg_v:
+        _need_cuda(t, "ref")
+    src = kv_layout(seg_k[0], batched=False)
+    for t in seg_k[1:] + seg_v:
+        o = kv_layout(t, batched=False)
+        if (o.stride_layer, o.stride_head, o.stride_token, o.head_dim, o.elem_bytes) != \
+                (src.stride_layer, src.stride_head, src.stride_token, src.head_dim, src.elem_bytes):
+            raise ValueError("all segments must share one layout")
+    _need_cuda(idx, "idx")
+    idx2 = idx if idx.dim() == 2 else idx.view(1, -1)
+    if idx2.dtype != torch.int32 or not idx2.is_contiguous():
+        raise ValueError("idx must be contiguous int32")
+    n_batch, n_tgt = idx2.shape
+    L, H, hd = src.n_layers, src.n_heads, src.head_dim
+    if out_k is None:
+        out_k = torch.empty((n_batch, L, H, n_tgt, hd), dtype=seg_k[0].dtype, device=seg_k[0].device)
+    if out_v is None:
+        out_v = torch.empty((n_batch, L, H, n_tgt, hd), dtype=seg_v[0].dtype, device=seg_v[0].device)
+    dst = kv_layout(out_k, batched=True)
+    dv = kv_layout(out_v, batched=True)
+    if (dst.stride_batch, dst.stride_layer, dst.stride_head, dst.stride_token) != \
+            (dv.stride_batch, dv.stride_layer, dv.stride_head, dv.stride_token):
+        raise ValueError("out_k and out_v must share one layout")
+    n_seg = len(seg_k)
+    offs = [0]
+    for t in seg_k:
+        offs.append(offs[-1] + t.shape[2])
+    pk = (ctypes.c_void_p * n_seg)(*[t.data_ptr() for t in seg_k])
+    pv = (ctypes.c_void_p * n_seg)(*[t.data_ptr() for t in seg_v])
+    po = (ctypes.c_int64 * (n_seg + 1))(*offs)
+    st = load().semshare_gather_kv(pk, pv, po, n_seg, src, _ptr(idx2), n_tgt, n_batch, _ptr(out_k), _ptr(out_v), dst,
+                                   _ptr(err_flag), _stream(stream))
+    _check(st, "semshare_gather_kv")
+    return out_k, out_v

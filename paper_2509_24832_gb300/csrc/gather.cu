@@ -1,0 +1,234 @@
+// gather.cu -- semshare_gather_kv: rearrange the reference K/V cache into the target's token
+// order with 16-byte vector copies.
+//
+// What it computes (SemShareKV, arXiv 2509.24832): Sec. 3.3 reorders the reference prompt's
+// KV cache token by token so that it has the target's length and every pair comes from the
+// reference cache; Sec. 3.3.2 stores K/V after RoPE, so rows move bit for bit.  For prompt b,
+// layer l, KV head h, token t:  out[b][l][h][t] = ref[l][h][idx[b][t]]  (K and V alike).
+//
+// Kernel design.  Pure streaming copy, bound by HBM bandwidth.  A CTA owns 64 target tokens
+// of one (b, l, h) plane and moves their 64 K rows and 64 V rows: it resolves the 64 indices
+// once (segment and local row, bounds-checked) into shared memory, then every thread issues
+// all of its 16-byte loads (read-only path, no L1 allocation) before any of its stores, so
+// each thread keeps 2*64*row_bytes/(16*256) requests in flight.  Consecutive threads touch
+// consecutive 16-byte chunks of a row and consecutive rows of the destination.
+#include "common.cuh"
+
+namespace semshare {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kTokens = 64;  // target tokens per CTA
+constexpr int kMaxSeg = 64;
+
+struct GatherArgs {
+    const uint8_t* src_k[kMaxSeg];
+    const uint8_t* src_v[kMaxSeg];
+    int64_t seg_off[kMaxSeg + 1];
+    int32_t n_seg;
+    int32_t n_layers;
+    int32_t n_heads;
+    int32_t n_batch;
+    int64_t n_tgt;
+    int64_t s_layer, s_head, s_token;           // source strides, bytes
+    int64_t d_batch, d_layer, d_head, d_token;  // destination strides, bytes
+    const int32_t* idx;
+    uint8_t* dst_k;
+    uint8_t* dst_v;
+    uint32_t* err_flag;
+};
+
+__device__ __forceinline__ uint4 load_stream(const void* p) {
+    uint4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
+}
+
+__device__ __forceinline__ void store_vec(void* p, const uint4& v) {
+    asm volatile("st.global.v4.u32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+
+// C = 16-byte chunks per row (row_bytes / 16).
+template <int C>
+__global__ void __launch_bounds__(kThreads) kv_gather_kernel(const __grid_constant__ GatherArgs a) {
+    constexpr int kRowsPerPass = kThreads / C;
+    constexpr int kPasses = 2 * kTokens / kRowsPerPass;  // K rows then V rows
+    static_assert(kThreads % C == 0 && (2 * kTokens) % kRowsPerPass == 0, "row split");
+
+    __shared__ int64_t s_src_off[kTokens];  // byte offset of the source row inside its segment
+    __shared__ int32_t s_seg[kTokens];      // segment, -1 = skip (tail or bad index)
+
+    const int64_t plane = blockIdx.y + static_cast<int64_t>(gridDim.y) * blockIdx.z;  // (b, l, h)
+    const int h = static_cast<int>(plane % a.n_heads);
+    const int l = static_cast<int>((plane / a.n_heads) % a.n_layers);
+    const int64_t b = plane / (static_cast<int64_t>(a.n_heads) * a.n_layers);
+    const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kTokens;
+
+    if (threadIdx.x < kTokens) {
+        const int64_t t = t0 + threadIdx.x;
+        int32_t seg = -1;
+        int64_t off = 0;
+        if (t < a.n_tgt) {
+            const int64_t r = __ldg(a.idx + b * a.n_tgt + t);
+            if (r >= 0 && r < a.seg_off[a.n_seg]) {
+                seg = 0;
+                while (r >= a.seg_off[seg + 1]) ++seg;
+                off = l * a.s_layer + h * a.s_head + (r - a.seg_off[seg]) * a.s_token;
+            } else if (a.err_flag) {
+                atomicOr(a.err_flag, SEMSHARE_FLAG_INDEX);
+            }
+        }
+        s_seg[threadIdx.x] = seg;
+        s_src_off[threadIdx.x] = off;
+    }
+    __syncthreads();
+
+    const int c = threadIdx.x % C;
+    const int rr = threadIdx.x / C;
+    const int64_t dst_plane = b * a.d_batch + l * a.d_layer + h * a.d_head;
+    uint4 v[kPasses];
+#pragma unroll
+    for (int p = 0; p < kPasses; ++p) {
+        const int row = rr + p * kRowsPerPass;  // 0..2*kTokens-1: K rows, then V rows
+        const int tt = row % kTokens;
+        const int seg = s_seg[tt];
+        if (seg >= 0) {
+            const uint8_t* base = (row < kTokens) ? a.src_k[seg] : a.src_v[seg];
+            v[p] = load_stream(base + s_src_off[tt] + c * 16);
+        }
+    }
+#pragma unroll
+    for (int p = 0; p < kPasses; ++p) {
+        const int row = rr + p * kRowsPerPass;
+        const int tt = row % kTokens;
+        if (s_seg[tt] >= 0) {
+            uint8_t* base = (row < kTokens) ? a.dst_k : a.dst_v;
+            store_vec(base + dst_plane + (t0 + tt) * a.d_token + c * 16, v[p]);
+        }
+    }
+}
+
+// Rows whose size is not a power-of-two number of 16-byte chunks: one chunk per thread per
+// step over the CTA's rows.
+__global__ void __launch_bounds__(kThreads) kv_gather_generic_kernel(const __grid_constant__ GatherArgs a, int chunks) {
+    __shared__ int64_t s_src_off[kTokens];
+    __shared__ int32_t s_seg[kTokens];
+    const int64_t plane = blockIdx.y + static_cast<int64_t>(gridDim.y) * blockIdx.z;
+    const int h = static_cast<int>(plane % a.n_heads);
+    const int l = static_cast<int>((plane / a.n_heads) % a.n_layers);
+    const int64_t b = plane / (static_cast<int64_t>(a.n_heads) * a.n_layers);
+    const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kTokens;
+    if (threadIdx.x < kTokens) {
+        const int64_t t = t0 + threadIdx.x;
+        int32_t seg = -1;
+        int64_t off = 0;
+        if (t < a.n_tgt) {
+            const int64_t r = __ldg(a.idx + b * a.n_tgt + t);
+            if (r >= 0 && r < a.seg_off[a.n_seg]) {
+                seg = 0;
+                while (r >= a.seg_off[seg + 1]) ++seg;
+                off = l * a.s_layer + h * a.s_head + (r - a.seg_off[seg]) * a.s_token;
+            } else if (a.err_flag) {
+                atomicOr(a.err_flag, SEMSHARE_FLAG_INDEX);
+            }
+        }
+        s_seg[threadIdx.x] = seg;
+        s_src_off[threadIdx.x] = off;
+    }
+    __syncthreads();
+    const int64_t dst_plane = b * a.d_batch + l * a.d_layer + h * a.d_head;
+    const int total = 2 * kTokens * chunks;
+    for (int e = threadIdx.x; e < total; e += kThreads) {
+        const int row = e / chunks, c = e - row * chunks;
+        const int tt = row % kTokens;
+        const int seg = s_seg[tt];
+        if (seg < 0) continue;
+        const uint8_t* src = ((row < kTokens) ? a.src_k[seg] : a.src_v[seg]) + s_src_off[tt] + c * 16;
+        uint8_t* dst = ((row < kTokens) ? a.dst_k : a.dst_v) + dst_plane + (t0 + tt) * a.d_token + c * 16;
+        store_vec(dst, load_stream(src));
+    }
+}
+
+bool stride_ok(int64_t s, int64_t elem) { return s >= 0 && ((s * elem) % 16) == 0; }
+
+}  // namespace
+}  // namespace semshare
+
+extern "C" semshare_status semshare_gather_kv(const void* const* ref_k, const void* const* ref_v,
+                                              const int64_t* seg_offsets, int32_t n_seg, semshare_kv_layout src,
+                                              const int32_t* idx, int64_t n_tgt, int32_t n_batch, void* out_k,
+                                              void* out_v, semshare_kv_layout dst, uint32_t* err_flag,
+                                              void* stream) {
+    using namespace semshare;
+    if (n_seg < 1 || n_seg > kMaxSeg || !ref_k || !ref_v || !seg_offsets) return SEMSHARE_EINVAL;
+    if (n_tgt < 0 || n_batch < 0) return SEMSHARE_EINVAL;
+    if (src.n_layers < 1 || src.n_heads < 1 || src.head_dim < 1) return SEMSHARE_EINVAL;
+    if (src.elem_bytes != 1 && src.elem_bytes != 2 && src.elem_bytes != 4 && src.elem_bytes != 8)
+        return SEMSHARE_EINVAL;
+    if (dst.n_layers != src.n_layers || dst.n_heads != src.n_heads || dst.head_dim != src.head_dim ||
+        dst.elem_bytes != src.elem_bytes)
+        return SEMSHARE_EINVAL;
+    const int64_t eb = src.elem_bytes;
+    const int64_t row_bytes = static_cast<int64_t>(src.head_dim) * eb;
+    if (row_bytes % 16 != 0) return SEMSHARE_EINVAL;
+    if (!stride_ok(src.stride_layer, eb) || !stride_ok(src.stride_head, eb) || !stride_ok(src.stride_token, eb) ||
+        !stride_ok(dst.stride_batch, eb) || !stride_ok(dst.stride_layer, eb) || !stride_ok(dst.stride_head, eb) ||
+        !stride_ok(dst.stride_token, eb))
+        return SEMSHARE_EINVAL;
+    if (seg_offsets[0] != 0) return SEMSHARE_EINVAL;
+    for (int s = 0; s < n_seg; ++s) {
+        if (seg_offsets[s + 1] < seg_offsets[s]) return SEMSHARE_EINVAL;
+        if (seg_offsets[s + 1] > seg_offsets[s] && (!ref_k[s] || !ref_v[s] || !aligned(ref_k[s], 16) || !aligned(ref_v[s], 16)))
+            return SEMSHARE_EINVAL;
+    }
+    if (seg_offsets[n_seg] >= (int64_t(1) << 31)) return SEMSHARE_EUNSUPPORTED;
+    if (n_tgt == 0 || n_batch == 0) return SEMSHARE_OK;
+    if (!idx || !out_k || !out_v || !aligned(idx, 4) || !aligned(out_k, 16) || !aligned(out_v, 16) ||
+        (err_flag && !aligned(err_flag, 4)))
+        return SEMSHARE_EINVAL;
+
+    GatherArgs a{};
+    for (int s = 0; s < n_seg; ++s) {
+        a.src_k[s] = static_cast<const uint8_t*>(ref_k[s]);
+        a.src_v[s] = static_cast<const uint8_t*>(ref_v[s]);
+    }
+    for (int s = 0; s <= n_seg; ++s) a.seg_off[s] = seg_offsets[s];
+    a.n_seg = n_seg;
+    a.n_layers = src.n_layers;
+    a.n_heads = src.n_heads;
+    a.n_batch = n_batch;
+    a.n_tgt = n_tgt;
+    a.s_layer = src.stride_layer * eb;
+    a.s_head = src.stride_head * eb;
+    a.s_token = src.stride_token * eb;
+    a.d_batch = dst.stride_batch * eb;
+    a.d_layer = dst.stride_layer * eb;
+    a.d_head = dst.stride_head * eb;
+    a.d_token = dst.stride_token * eb;
+    a.idx = idx;
+    a.dst_k = static_cast<uint8_t*>(out_k);
+    a.dst_v = static_cast<uint8_t*>(out_v);
+    a.err_flag = err_flag;
+
+    const int64_t planes = static_cast<int64_t>(n_batch) * src.n_layers * src.n_heads;
+    const int64_t tblocks = (n_tgt + kTokens - 1) / kTokens;
+    if (tblocks > 0x7FFFFFFF) return SEMSHARE_EUNSUPPORTED;
+    // planes tile the (y, z) grid exactly: y = the largest divisor of planes within 65535
+    int64_t gy = planes < 65535 ? planes : 65535;
+    while (planes % gy != 0) --gy;
+    if (planes / gy > 65535) return SEMSHARE_EUNSUPPORTED;
+    const dim3 grid(static_cast<unsigned>(tblocks), static_cast<unsigned>(gy), static_cast<unsigned>(planes / gy));
+    const int chunks = static_cast<int>(row_bytes / 16);
+    cudaStream_t s = as_stream(stream);
+    switch (chunks) {
+        case 4: kv_gather_kernel<4><<<grid, kThreads, 0, s>>>(a); break;
+        case 8: kv_gather_kernel<8><<<grid, kThreads, 0, s>>>(a); break;
+        case 16: kv_gather_kernel<16><<<grid, kThreads, 0, s>>>(a); break;
+        case 32: kv_gather_kernel<32><<<grid, kThreads, 0, s>>>(a); break;
+        default: kv_gather_generic_kernel<<<grid, kThreads, 0, s>>>(a, chunks); break;
+    }
+    return launch_status();
+}

@@ -1,0 +1,116 @@
+"""The C-ABI library loads, exports every declared entry point and rejects bad arguments on the
+host, before touching the GPU (these tests run without one)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2509_24832_gb300 import build
+
+    build.build()
+    import paper_2509_24832_gb300 as ss
+
+    return ss.load()
+
+
+def _declared():
+    names = set()
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", fn)).read()
+            text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+            names |= set(re.findall(r"\b(semshare_\w+)\s*\(", text))
+    return sorted(names)
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = _declared()
+    assert {"semshare_hash", "semshare_match", "semshare_gather_kv", "semshare_rope_table"} <= set(names)
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_status_helpers(lib):
+    assert lib.semshare_abi_version() == 1
+    assert lib.semshare_status_string(0) == b"ok"
+    assert lib.semshare_flag_status(0) == 0
+    assert lib.semshare_flag_status(1) == 4
+    assert lib.semshare_flag_status(3) == 5
+    assert lib.semshare_match_workspace_size(1000) == 8000
+
+
+FAKE = ctypes.c_void_p(1 << 20)  # aligned, never dereferenced: every case below fails validation first
+
+
+def _hash(lib, **kw):
+    a = dict(emb=FAKE, dtype=0, n=10, d=128, row_stride=128, positions=None, table=FAKE, hyp=FAKE, nbits=64,
+             codes=FAKE, proj=None, flag=None, stream=None)
+    a.update(kw)
+    return lib.semshare_hash(a["emb"], a["dtype"], a["n"], a["d"], a["row_stride"], a["positions"], a["table"],
+                             a["hyp"], a["nbits"], a["codes"], a["proj"], a["flag"], a["stream"])
+
+
+def test_hash_argument_errors(lib):
+    assert _hash(lib, dtype=7) == 1
+    assert _hash(lib, n=-1) == 1
+    assert _hash(lib, d=127, row_stride=127) == 1
+    assert _hash(lib, d=96, row_stride=96) == 2          # d not a multiple of 64
+    assert _hash(lib, nbits=48) == 2
+    assert _hash(lib, nbits=288) == 2
+    assert _hash(lib, row_stride=100) == 1               # shorter than d
+    assert _hash(lib, row_stride=132) == 1               # 264-byte rows: not 16-byte multiple
+    assert _hash(lib, emb=None) == 1
+    assert _hash(lib, emb=ctypes.c_void_p((1 << 20) + 4)) == 1  # misaligned
+    assert _hash(lib, codes=None) == 1
+    assert _hash(lib, n=1 << 31) == 2
+    assert _hash(lib, n=0, emb=None, codes=None) == 0    # empty: nothing to do
+
+
+def test_match_argument_errors(lib):
+    m = lib.semshare_match
+    assert m(FAKE, 10, FAKE, 0, 64, FAKE, None, FAKE, 80, None) == 1   # n_ref = 0
+    assert m(FAKE, 10, FAKE, 5, 40, FAKE, None, FAKE, 80, None) == 2   # nbits
+    assert m(FAKE, 10, FAKE, 5, 64, FAKE, None, FAKE, 79, None) == 1   # workspace too small
+    assert m(FAKE, 10, FAKE, 5, 64, None, None, FAKE, 80, None) == 1
+    assert m(None, 0, FAKE, 5, 64, None, None, None, 0, None) == 0     # empty target
+
+
+def test_gather_argument_errors(lib):
+    import paper_2509_24832_gb300 as ss
+
+    lay = ss.KVLayout(2, 4, 64, 2, 0, 4 * 100 * 64, 100 * 64, 64)
+    out = ss.KVLayout(2, 4, 64, 2, 2 * 4 * 10 * 64, 4 * 10 * 64, 10 * 64, 64)
+    pk = (ctypes.c_void_p * 1)(1 << 20)
+    offs = (ctypes.c_int64 * 2)(0, 100)
+    g = lib.semshare_gather_kv
+    assert g(pk, pk, offs, 0, lay, FAKE, 10, 1, FAKE, FAKE, out, None, None) == 1       # n_seg
+    bad = ss.KVLayout(2, 4, 60, 2, 0, 4 * 100 * 60, 100 * 60, 60)                        # 120-byte rows
+    assert g(pk, pk, offs, 1, bad, FAKE, 10, 1, FAKE, FAKE, bad, None, None) == 1
+    other = ss.KVLayout(2, 8, 64, 2, 0, 8 * 100 * 64, 100 * 64, 64)
+    assert g(pk, pk, offs, 1, lay, FAKE, 10, 1, FAKE, FAKE, other, None, None) == 1     # head mismatch
+    offs_bad = (ctypes.c_int64 * 2)(5, 100)
+    assert g(pk, pk, offs_bad, 1, lay, FAKE, 10, 1, FAKE, FAKE, out, None, None) == 1
+    assert g(pk, pk, offs, 1, lay, None, 0, 1, None, None, out, None, None) == 0        # empty
+
+
+def test_rope_table_argument_errors(lib):
+    t = lib.semshare_rope_table
+    assert t(7, 10000.0, FAKE, None) == 1
+    assert t(64, 0.0, FAKE, None) == 1
+    assert t(64, float('nan'), FAKE, None) == 1
+    assert t(64, 10000.0, None, None) == 1
+
+
+def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
+    import paper_2509_24832_gb300._native as nat
+
+    monkeypatch.setattr(nat, "LIB_PATH", str(tmp_path / "missing.so"))
+    monkeypatch.setattr(nat, "_lib", None)
+    with pytest.raises(RuntimeError):
+        nat.load()

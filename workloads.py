@@ -206,3 +206,33 @@ def kv_cache(wl: Workload, seed: int | None = None, segment: int | None = None):
 def random_codes(n: int, nbits: int, seed: int, stream: int = 0) -> np.ndarray:
     """Uniform random packed codes [n][nbits/32] (uint32) for search-only tests."""
     return rng(seed, 100 + stream).integers(0, 1 << 32, size=(n, nbits // 32), dtype=np.uint64).astype(np.uint32)
+
+
+def kv_cache_device(wl: Workload, device, seed: int | None = None, segment: int = 0):
+    """One reference prompt's K and V caches drawn on the device: bf16 N(0,1), each
+    [L][H][seg_len][hd].  For the multi-GB caches of the batched and pool workloads, where
+    drawing on the host would dominate; seeded through a device generator."""
+    import torch
+
+    seed = wl.base_seed if seed is None else seed
+    L, H, hd = wl.kv
+    g = torch.Generator(device=device).manual_seed((seed * 1000003 + 7919 * (segment + 1)) & 0x7FFFFFFFFFFFFFFF)
+    k = torch.randn((L, H, wl.seg_len, hd), generator=g, device=device).to(torch.bfloat16)
+    v = torch.randn((L, H, wl.seg_len, hd), generator=g, device=device).to(torch.bfloat16)
+    return k, v
+
+
+def prompt_rows(wl: Workload, seed: int | None = None, batches=None):
+    """Host rows of one matching problem, reference rows first:
+    (emb [n_ref + B*n_tgt][d], positions, source rows [B][n_tgt]) for target prompts `batches`
+    (default: all n_batch of them)."""
+    seed = wl.base_seed if seed is None else seed
+    batches = range(wl.n_batch) if batches is None else list(batches)
+    ref = reference_embeddings(wl, seed)
+    rows, pos, src = [ref], [reference_positions(wl)], []
+    for b in batches:
+        x, p, s = target_prompt(wl, b=b, ref=ref, seed=seed)
+        rows.append(x)
+        pos.append(p)
+        src.append(s)
+    return np.concatenate(rows), np.concatenate(pos).astype(np.int32), np.stack(src)
