@@ -43,7 +43,8 @@ typedef enum {
     SEMSHARE_EUNSUPPORTED = 2,  /* valid request outside what the kernels implement */
     SEMSHARE_ECUDA = 3,         /* a CUDA runtime or driver call failed */
     SEMSHARE_EINDEX = 4,        /* a kernel met an index outside its table (from err_flag) */
-    SEMSHARE_ETIMEOUT = 5       /* a kernel pipeline wait hit its time limit (from err_flag) */
+    SEMSHARE_ETIMEOUT = 5,      /* a kernel pipeline wait hit its time limit (from err_flag) */
+    SEMSHARE_ETOOLARGE = 6      /* a size exceeds semshare_match_static's fixed scratch capacity */
 } semshare_status;
 
 typedef enum { SEMSHARE_BF16 = 0, SEMSHARE_F32 = 1 } semshare_dtype;
@@ -134,6 +135,31 @@ size_t semshare_match_workspace_size(int64_t n_tgt);
 semshare_status semshare_match(const uint32_t* tgt_codes, int64_t n_tgt, const uint32_t* ref_codes, int64_t n_ref,
                                int32_t nbits, int32_t* idx, int32_t* dist, void* workspace, size_t workspace_bytes,
                                void* stream);
+
+/*
+ * semshare_match_static -- semshare_match without a caller-provided workspace.
+ *
+ * The paper has no counterpart: this entry point exists for callers that cannot allocate
+ * device memory (for example code embedded in a host framework that owns the whole device
+ * memory pool and forbids allocations, or a serving loop that must not allocate on its hot
+ * path).  It computes exactly what semshare_match computes, with the same arguments minus the
+ * workspace, and allocates nothing: its scratch (one 64-bit key per target) is a fixed array
+ * inside the library, SEMSHARE_MATCH_STATIC_MAX_TARGETS keys (2 MiB), which every device that
+ * loads the library holds until the process exits.
+ *
+ *   n_tgt      0 <= n_tgt <= SEMSHARE_MATCH_STATIC_MAX_TARGETS; larger requests return
+ *              SEMSHARE_ETOOLARGE before anything is enqueued
+ *   other arguments as for semshare_match
+ * The first call on a device looks up that device's address of the array (once per device,
+ * with the device current); make that first call before any stream capture.  All calls on a
+ * device share the one array and it keeps the previous call's contents; each call resets the
+ * keys it uses before its search.  Calls whose work overlaps on the GPU (other streams, other
+ * host threads on the same device) race on the array and give wrong results: serialise them.
+ * Unlike the other entry points this one keeps state: the array and the per-device address.
+ */
+#define SEMSHARE_MATCH_STATIC_MAX_TARGETS 262144
+semshare_status semshare_match_static(const uint32_t* tgt_codes, int64_t n_tgt, const uint32_t* ref_codes,
+                                      int64_t n_ref, int32_t nbits, int32_t* idx, int32_t* dist, void* stream);
 
 /*
  * Layout of a K or V cache: element (b, l, h, t, e) of a cache with this layout lives at

@@ -12,6 +12,7 @@ from ._native import (  # noqa: F401
     FLAG_TIMEOUT,
     KVLayout,
     LIB_PATH,
+    MATCH_STATIC_MAX_TARGETS,
     SemshareError,
     check_flag,
     flag_status,
@@ -22,6 +23,7 @@ from ._native import (  # noqa: F401
     semshare_gather_kv,
     semshare_hash,
     semshare_match,
+    semshare_match_static,
     semshare_match_workspace_size,
     semshare_rope_table,
     status_string,

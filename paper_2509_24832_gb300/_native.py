@@ -14,7 +14,8 @@ import torch
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "_lib", "libsemshare.so")
 
-OK, EINVAL, EUNSUPPORTED, ECUDA, EINDEX, ETIMEOUT = range(6)
+OK, EINVAL, EUNSUPPORTED, ECUDA, EINDEX, ETIMEOUT, ETOOLARGE = range(7)
+MATCH_STATIC_MAX_TARGETS = 262144
 FLAG_INDEX, FLAG_TIMEOUT = 1, 2
 BF16, F32 = 0, 1
 
@@ -59,6 +60,8 @@ def load():
         lib.semshare_match_workspace_size.restype = ctypes.c_size_t
         lib.semshare_match.argtypes = [P, i64, P, i64, i32, P, P, P, ctypes.c_size_t, P]
         lib.semshare_match.restype = ctypes.c_int
+        lib.semshare_match_static.argtypes = [P, i64, P, i64, i32, P, P, P]
+        lib.semshare_match_static.restype = ctypes.c_int
         lib.semshare_gather_kv.argtypes = [P, P, P, i32, KVLayout, P, i64, i32, P, P, KVLayout, P, P]
         lib.semshare_gather_kv.restype = ctypes.c_int
         _lib = lib
@@ -182,6 +185,30 @@ def semshare_match(tgt_codes: torch.Tensor, ref_codes: torch.Tensor, idx: torch.
     st = load().semshare_match(_ptr(tgt_codes), n_tgt, _ptr(ref_codes), n_ref, nbits, _ptr(idx), _ptr(dist),
                                _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream))
     _check(st, "semshare_match")
+    return idx, dist
+
+
+def semshare_match_static(tgt_codes: torch.Tensor, ref_codes: torch.Tensor, idx: torch.Tensor | None = None,
+                          dist: torch.Tensor | None = None, nbits: int | None = None, stream=None):
+    """semshare_match for callers that cannot allocate device memory: no workspace argument,
+    the library's own fixed scratch (at most MATCH_STATIC_MAX_TARGETS targets) is used.
+    Pass preallocated idx/dist to keep the call itself free of allocations.
+    Returns (idx int32 [n_tgt], dist int32 [n_tgt])."""
+    _need_cuda(tgt_codes, "tgt_codes")
+    _need_cuda(ref_codes, "ref_codes")
+    if not tgt_codes.is_contiguous() or not ref_codes.is_contiguous():
+        raise ValueError("codes must be contiguous")
+    n_tgt, w = tgt_codes.shape
+    if ref_codes.shape[1] != w:
+        raise ValueError("code widths differ")
+    nbits = 32 * w if nbits is None else nbits
+    if idx is None:
+        idx = torch.empty(n_tgt, dtype=torch.int32, device=tgt_codes.device)
+    if dist is None:
+        dist = torch.empty(n_tgt, dtype=torch.int32, device=tgt_codes.device)
+    st = load().semshare_match_static(_ptr(tgt_codes), n_tgt, _ptr(ref_codes), ref_codes.shape[0], nbits, _ptr(idx),
+                                      _ptr(dist), _stream(stream))
+    _check(st, "semshare_match_static")
     return idx, dist
 
 

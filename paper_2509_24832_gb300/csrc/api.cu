@@ -29,6 +29,7 @@ extern "C" const char* semshare_status_string(semshare_status s) {
         case SEMSHARE_ECUDA: return "CUDA error";
         case SEMSHARE_EINDEX: return "index out of range";
         case SEMSHARE_ETIMEOUT: return "kernel wait timed out";
+        case SEMSHARE_ETOOLARGE: return "size exceeds the fixed scratch capacity";
     }
     return "unknown status";
 }

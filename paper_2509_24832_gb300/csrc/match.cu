@@ -14,6 +14,8 @@
 // block, each target's best (distance << 32 | global index) goes to a 64-bit atomicMin in the
 // workspace.  atomicMin of that key is exactly "smallest distance, then lowest index", so the
 // result does not depend on the partition.  A final pass splits the keys into idx and dist.
+#include <mutex>
+
 #include "common.cuh"
 
 namespace semshare {
@@ -189,6 +191,83 @@ extern "C" semshare_status semshare_match(const uint32_t* tgt_codes, int64_t n_t
     keys_init_kernel<<<small_grid, 256, 0, s>>>(keys, n_tgt);
     if (launch_status() != SEMSHARE_OK) return SEMSHARE_ECUDA;
     semshare_status st = SEMSHARE_EUNSUPPORTED;
+    switch (nbits / 32) {
+        case 1: st = launch_search<1>(tgt_codes, n_tgt, ref_codes, n_ref, keys, sms, s); break;
+        case 2: st = launch_search<2>(tgt_codes, n_tgt, ref_codes, n_ref, keys, sms, s); break;
+        case 3: st = launch_search<3>(tgt_codes, n_tgt, ref_codes, n_ref, keys, sms, s); break;
+        case 4: st = launch_search<4>(tgt_codes, n_tgt, ref_codes, n_ref, keys, sms, s); break;
+        case 5: st = launch_search<5>(tgt_codes, n_tgt, ref_codes, n_ref, keys, sms, s); break;
+        case 6: st = launch_search<6>(tgt_codes, n_tgt, ref_codes, n_ref, keys, sms, s); break;
+        case 7: st = launch_search<7>(tgt_codes, n_tgt, ref_codes, n_ref, keys, sms, s); break;
+        case 8: st = launch_search<8>(tgt_codes, n_tgt, ref_codes, n_ref, keys, sms, s); break;
+    }
+    if (st != SEMSHARE_OK) return st;
+    keys_split_kernel<<<small_grid, 256, 0, s>>>(keys, n_tgt, idx, dist);
+    return launch_status();
+}
+
+// ---- semshare_match_static: the same search with library-owned scratch ------------------------
+//
+// For callers that cannot allocate device memory themselves (for example code embedded in a
+// host framework that owns the whole device memory pool and forbids allocations, or a serving
+// loop that must not allocate on its hot path).  The per-target keys live in one file-scope
+// device array instead of a caller workspace; every device that loads this library holds it
+// (SEMSHARE_MATCH_STATIC_MAX_TARGETS x 8 bytes = 2 MiB) until the process exits.
+
+static __device__ __align__(256) unsigned long long g_static_match_keys[SEMSHARE_MATCH_STATIC_MAX_TARGETS];
+
+namespace semshare {
+namespace {
+
+constexpr int kStaticMaxDevices = 64;
+std::mutex g_static_keys_mutex;
+unsigned long long* g_static_keys_addr[kStaticMaxDevices] = {};
+
+// Device address of g_static_match_keys on the current device.  In host code the array's name
+// is only a host-side stand-in, so the address is looked up once per device (with that device
+// current) and cached.
+semshare_status static_keys_on_current_device(unsigned long long** keys) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return SEMSHARE_ECUDA;
+    if (dev < 0 || dev >= kStaticMaxDevices) return SEMSHARE_EUNSUPPORTED;
+    std::lock_guard<std::mutex> lock(g_static_keys_mutex);
+    if (g_static_keys_addr[dev] == nullptr) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_static_match_keys) != cudaSuccess || p == nullptr) return SEMSHARE_ECUDA;
+        g_static_keys_addr[dev] = static_cast<unsigned long long*>(p);
+    }
+    *keys = g_static_keys_addr[dev];
+    return SEMSHARE_OK;
+}
+
+}  // namespace
+}  // namespace semshare
+
+extern "C" semshare_status semshare_match_static(const uint32_t* tgt_codes, int64_t n_tgt, const uint32_t* ref_codes,
+                                                 int64_t n_ref, int32_t nbits, int32_t* idx, int32_t* dist,
+                                                 void* stream) {
+    using namespace semshare;
+    if (n_tgt < 0 || n_ref < 1) return SEMSHARE_EINVAL;
+    if (nbits < 32 || nbits > 256 || nbits % 32 != 0) return SEMSHARE_EUNSUPPORTED;
+    if (n_ref >= (int64_t(1) << 31)) return SEMSHARE_EUNSUPPORTED;
+    if (n_tgt > SEMSHARE_MATCH_STATIC_MAX_TARGETS) return SEMSHARE_ETOOLARGE;
+    if (n_tgt == 0) return SEMSHARE_OK;
+    if (!tgt_codes || !ref_codes || !idx) return SEMSHARE_EINVAL;
+    if (!aligned(tgt_codes, 16) || !aligned(ref_codes, 16) || !aligned(idx, 4) || (dist && !aligned(dist, 4)))
+        return SEMSHARE_EINVAL;
+
+    unsigned long long* keys = nullptr;
+    semshare_status st = static_keys_on_current_device(&keys);
+    if (st != SEMSHARE_OK) return st;
+    int sms = 0;
+    if (current_sm_count(&sms, nullptr) != SEMSHARE_OK) return SEMSHARE_ECUDA;
+    cudaStream_t s = as_stream(stream);
+    const int small_grid = static_cast<int>((n_tgt + 255) / 256 < sms * 4 ? (n_tgt + 255) / 256 : sms * 4);
+
+    // the array keeps the previous call's keys: reset the ones this call uses
+    keys_init_kernel<<<small_grid, 256, 0, s>>>(keys, n_tgt);
+    if (launch_status() != SEMSHARE_OK) return SEMSHARE_ECUDA;
+    st = SEMSHARE_EUNSUPPORTED;
     switch (nbits / 32) {
         case 1: st = launch_search<1>(tgt_codes, n_tgt, ref_codes, n_ref, keys, sms, s); break;
         case 2: st = launch_search<2>(tgt_codes, n_tgt, ref_codes, n_ref, keys, sms, s); break;
