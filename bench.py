@@ -214,6 +214,8 @@ class Problem:
         self.idx = torch.empty(n_t, dtype=torch.int32, device=device)
         self.dist = torch.empty(n_t, dtype=torch.int32, device=device)
         self.ws = torch.empty(ss.semshare_match_workspace_size(n_t), dtype=torch.uint8, device=device)
+        self.hash_ws = torch.zeros(max(256, ss.semshare_hash_workspace_size(rows, wl.d, wl.nbits)), dtype=torch.uint8,
+                                   device=device)
         segs = [workloads.kv_cache_device(wl, device, seed=seed, segment=s) for s in range(wl.n_seg)]
         self.ref_k = [s[0] for s in segs]
         self.ref_v = [s[1] for s in segs]
@@ -223,7 +225,8 @@ class Problem:
         self.flag = ss.new_err_flag(device)
 
     def hash(self):
-        self.ss.semshare_hash(self.emb, self.table, self.hyp, self.pos, codes=self.codes, err_flag=self.flag)
+        self.ss.semshare_hash(self.emb, self.table, self.hyp, self.pos, codes=self.codes, err_flag=self.flag,
+                              workspace=self.hash_ws)
 
     def match(self):
         n_ref = self.wl.n_ref

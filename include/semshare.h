@@ -14,7 +14,9 @@
  * Conventions shared by every call:
  *   - Buffers are owned by the caller.  Pointers marked "device" point to memory of the
  *     current CUDA device; "host" marks host memory read during the call only.  No call
- *     allocates or frees memory, and the library keeps no state between calls.
+ *     allocates or frees memory.  Scratch memory is passed in by the caller (the
+ *     workspace arguments); apart from semshare_match_static the library keeps no state
+ *     between calls.
  *   - `stream` is a cudaStream_t (NULL = the legacy default stream).  Work is enqueued on it
  *     and runs asynchronously; a call returns once the work is enqueued.
  *   - Argument errors are detected on the host before anything is enqueued and returned as
@@ -66,15 +68,16 @@ int32_t semshare_abi_version(void);
  * semshare_rope_table -- rotation frequencies of Eq. 1 (App. A.1) in fixed point.
  *
  * Pair k of a d-wide embedding row turns by theta_k = rope_base^(-2k/d) radians per position
- * (Eq. 1; the angle at position m is m * theta_k, Sec. 3.3.1).  table[k] receives
+ * (Eq. 1; the angle at position m is m * theta_k, Sec. 3.3.1).  For k < d/2, table[k] receives
  * frac(theta_k / (2*pi)) * 2^64 rounded: the turns per position modulo one turn as an
  * unsigned 0.64 fixed-point fraction, so a kernel gets the angle of position m modulo a full
- * turn from the low 64 bits of m * table[k] with integer arithmetic.  Computed on the device
- * in double precision.
+ * turn from the low 64 bits of m * table[k] with integer arithmetic; table[d/2 + k] receives
+ * cos(32*theta_k) (low 32 bits) and sin(32*theta_k) (high 32 bits) as floats, the rotation
+ * between two positions 32 apart.  Computed on the device in double precision.
  *
  *   d          embedding dimension, even, 2 <= d <= 65536
  *   rope_base  the RoPE base (10000 in Eq. 1), finite and > 0
- *   table      device, d/2 uint64 words, 8-byte aligned; written
+ *   table      device, d uint64 words, 16-byte aligned; written
  * Returns EINVAL for a bad d, base or pointer.  The table depends only on (d, rope_base):
  * compute it once and reuse it for every semshare_hash call.
  */
@@ -87,7 +90,9 @@ semshare_status semshare_rope_table(int32_t d, double rope_base, uint64_t* table
  *   y = RoPE(emb[i], positions[i])       Eq. 1, pairs (2k, 2k+1), angle positions[i]*theta_k
  *   p_j = <hyperplanes[j], bf16(y)>      fp32 accumulation on the tensor cores
  *   bit j of codes[i] = [p_j > 0]         sign random projection (App. A.2, App. D: LSH)
- * y is computed in fp32 and rounded to bf16 (nearest even) before the products.
+ * y is computed in fp32 and rounded to bf16 (nearest even) before the products.  The K range
+ * of a 128-row tile may be split across SMs; the partial sums are then added in K order, so
+ * the codes are the same on every run on a given device.
  *
  *   emb         device, n rows of d elements of `dtype`, row i at element offset i*row_stride;
  *               16-byte aligned base, row_stride*element_size a multiple of 16 bytes
@@ -98,18 +103,28 @@ semshare_status semshare_rope_table(int32_t d, double rope_base, uint64_t* table
  *   positions   device, n int32 token positions >= 0, or NULL for positions 0..n-1.  Each
  *               prompt uses its own 0-based positions; rows of several prompts may be hashed
  *               in one call by passing each row's position.
- *   rope_table  device, d/2 words from semshare_rope_table(d, base, ...)
+ *   rope_table  device, the d words written by semshare_rope_table(d, base, ...)
  *   hyperplanes device, [nbits][d] bf16 bit patterns, row-major, 16-byte aligned
  *   nbits       code length: 32, 64, ..., 256
  *   codes       device, [n][nbits/32] uint32, bit j of row i in word j/32 at bit j%32; written
  *   proj_out    device or NULL; if given, [n][nbits] float32 projections p_j are written too
+ *   workspace   device scratch of at least semshare_hash_workspace_size(n, d, nbits) bytes,
+ *               256-byte aligned.  It must be zero-filled before its first use; every call
+ *               that completes without an error flag leaves it zero-filled again, so one
+ *               workspace serves any number of calls made one after another.  Calls that may
+ *               run concurrently need separate workspaces.
  *   err_flag    device or NULL; SEMSHARE_FLAG_TIMEOUT is OR-ed in if a pipeline wait of the
- *               kernel exceeds its limit (the kernel then stops and leaves codes incomplete)
- * Returns EINVAL / EUNSUPPORTED for bad arguments, ECUDA if the launch fails.
+ *               kernel exceeds its limit (the kernel then stops, leaves codes incomplete and
+ *               the workspace in an unknown state: zero it before the next call)
+ * Returns EINVAL / EUNSUPPORTED for bad arguments (EINVAL for a short workspace), ECUDA if the
+ * launch fails.  semshare_hash_workspace_size returns 0 for arguments semshare_hash rejects;
+ * it depends on the current device (its SM count).
  */
+size_t semshare_hash_workspace_size(int64_t n, int32_t d, int32_t nbits);
 semshare_status semshare_hash(const void* emb, semshare_dtype dtype, int64_t n, int32_t d, int64_t row_stride,
                               const int32_t* positions, const uint64_t* rope_table, const uint16_t* hyperplanes,
-                              int32_t nbits, uint32_t* codes, float* proj_out, uint32_t* err_flag, void* stream);
+                              int32_t nbits, uint32_t* codes, float* proj_out, void* workspace,
+                              size_t workspace_bytes, uint32_t* err_flag, void* stream);
 
 /*
  * semshare_match -- step 3: Hamming nearest reference token of every target token.

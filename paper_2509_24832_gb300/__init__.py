@@ -16,12 +16,14 @@ from ._native import (  # noqa: F401
     SemshareError,
     check_flag,
     flag_status,
+    hash_workspace,
     kv_layout,
     load,
     new_err_flag,
     semshare_abi_version,
     semshare_gather_kv,
     semshare_hash,
+    semshare_hash_workspace_size,
     semshare_match,
     semshare_match_static,
     semshare_match_workspace_size,

@@ -54,7 +54,9 @@ def load():
         lib.semshare_abi_version.restype = i32
         lib.semshare_rope_table.argtypes = [i32, ctypes.c_double, P, P]
         lib.semshare_rope_table.restype = ctypes.c_int
-        lib.semshare_hash.argtypes = [P, ctypes.c_int, i64, i32, i64, P, P, P, i32, P, P, P, P]
+        lib.semshare_hash_workspace_size.argtypes = [i64, i32, i32]
+        lib.semshare_hash_workspace_size.restype = ctypes.c_size_t
+        lib.semshare_hash.argtypes = [P, ctypes.c_int, i64, i32, i64, P, P, P, i32, P, P, P, ctypes.c_size_t, P, P]
         lib.semshare_hash.restype = ctypes.c_int
         lib.semshare_match_workspace_size.argtypes = [i64]
         lib.semshare_match_workspace_size.restype = ctypes.c_size_t
@@ -114,20 +116,44 @@ def semshare_abi_version() -> int:
 
 def semshare_rope_table(d: int, rope_base: float = 10000.0, out: torch.Tensor | None = None, device=None,
                         stream=None) -> torch.Tensor:
-    """Fixed-point rotation frequencies for semshare_hash: [d/2] uint64 words (int64 storage)."""
+    """Rotation table for semshare_hash: [d] uint64 words (int64 storage): d/2 fixed-point turn
+    fractions, then d/2 (cos, sin) pairs of the 32-position rotation."""
     if out is None:
-        out = torch.empty(d // 2, dtype=torch.int64, device=device or "cuda")
+        out = torch.empty(d, dtype=torch.int64, device=device or "cuda")
     _need_cuda(out, "out")
     _check(load().semshare_rope_table(int(d), float(rope_base), _ptr(out), _stream(stream)), "semshare_rope_table")
     return out
 
 
+_hash_ws = {}
+
+
+def semshare_hash_workspace_size(n: int, d: int, nbits: int) -> int:
+    return int(load().semshare_hash_workspace_size(int(n), int(d), int(nbits)))
+
+
+def hash_workspace(n: int, d: int, nbits: int, device=None) -> torch.Tensor:
+    """A zero-filled hash workspace large enough for (n, d, nbits), kept per device and grown on
+    demand.  The library leaves it zero-filled after every successful call, so calls issued one
+    after another (on one stream) can share it; concurrent calls need their own."""
+    dev = torch.device(device or "cuda")
+    if dev.index is None:
+        dev = torch.device("cuda", torch.cuda.current_device())
+    need = max(256, semshare_hash_workspace_size(n, d, nbits))
+    ws = _hash_ws.get(dev)
+    if ws is None or ws.numel() < need:
+        ws = torch.zeros(need, dtype=torch.uint8, device=dev)
+        _hash_ws[dev] = ws
+    return ws
+
+
 def semshare_hash(emb: torch.Tensor, rope_table: torch.Tensor, hyperplanes: torch.Tensor,
                   positions: torch.Tensor | None = None, codes: torch.Tensor | None = None,
                   proj_out: torch.Tensor | None = None, err_flag: torch.Tensor | None = None,
-                  stream=None) -> torch.Tensor:
+                  workspace: torch.Tensor | None = None, stream=None) -> torch.Tensor:
     """LSH codes of RoPE-encoded rows.  emb [n][d] bf16/fp32 (rows may be strided),
-    hyperplanes [nbits][d] bf16, positions [n] int32 (None: 0..n-1).
+    hyperplanes [nbits][d] bf16, positions [n] int32 (None: 0..n-1).  workspace: a zero-filled
+    uint8 device buffer (default: the per-device one of hash_workspace()).
     Returns codes [n][nbits/32] int32 (uint32 bit patterns)."""
     _need_cuda(emb, "emb")
     _need_cuda(hyperplanes, "hyperplanes")
@@ -150,8 +176,12 @@ def semshare_hash(emb: torch.Tensor, rope_table: torch.Tensor, hyperplanes: torc
             raise ValueError("positions must be contiguous int32 [n]")
     if codes is None:
         codes = torch.empty((n, nbits // 32), dtype=torch.int32, device=emb.device)
+    if workspace is None:
+        workspace = hash_workspace(n, d, nbits, emb.device)
+    ws_bytes = workspace.numel() * workspace.element_size()
     st = load().semshare_hash(_ptr(emb), dt, n, d, emb.stride(0), _ptr(positions), _ptr(rope_table),
-                              _ptr(hyperplanes), nbits, _ptr(codes), _ptr(proj_out), _ptr(err_flag), _stream(stream))
+                              _ptr(hyperplanes), nbits, _ptr(codes), _ptr(proj_out), _ptr(workspace), ws_bytes,
+                              _ptr(err_flag), _stream(stream))
     _check(st, "semshare_hash")
     return codes
 

@@ -5,9 +5,11 @@
 namespace semshare {
 namespace {
 
-// table[k] = frac(theta_k / (2*pi)) * 2^64 rounded, theta_k = base^(-2k/d)  (Eq. 1, App. A.1):
-// the turns per position modulo one full turn, as an unsigned 0.64 fixed-point fraction.
-// Whole turns do not change the rotation, so only the fraction is kept; scaling by 2^64 is exact.
+// Rotation table of Eq. 1 (App. A.1), theta_k = base^(-2k/d), k < d/2:
+//   table[k]           frac(theta_k / (2*pi)) * 2^64 rounded: the turns per position modulo one
+//                      full turn, an unsigned 0.64 fixed-point fraction (scaling by 2^64 is exact)
+//   table[d/2 + k]     cos(32*theta_k) and sin(32*theta_k) as two floats (low word: cos): the
+//                      rotation between positions 32 apart, for stepping from one row to another
 __global__ void rope_table_kernel(int32_t d, double base, uint64_t* __restrict__ table) {
     const int32_t k = blockIdx.x * blockDim.x + threadIdx.x;
     if (k >= d / 2) return;
@@ -16,6 +18,9 @@ __global__ void rope_table_kernel(int32_t d, double base, uint64_t* __restrict__
     turns -= floor(turns);
     const double q = ldexp(turns, 64);
     table[k] = q >= 18446744073709551616.0 ? 0ull : __double2ull_rn(q);
+    const double a32 = 6.283185307179586476925286766559 * (32.0 * turns - floor(32.0 * turns));
+    const float c = static_cast<float>(cos(a32)), s = static_cast<float>(sin(a32));
+    table[d / 2 + k] = static_cast<uint64_t>(__float_as_uint(c)) | (static_cast<uint64_t>(__float_as_uint(s)) << 32);
 }
 
 }  // namespace
@@ -46,7 +51,7 @@ extern "C" semshare_status semshare_rope_table(int32_t d, double rope_base, uint
     using namespace semshare;
     if (d < 2 || d > 65536 || (d & 1)) return SEMSHARE_EINVAL;
     if (!(rope_base > 0.0) || !(rope_base < 1e300)) return SEMSHARE_EINVAL;
-    if (table == nullptr || !aligned(table, 8)) return SEMSHARE_EINVAL;
+    if (table == nullptr || !aligned(table, 16)) return SEMSHARE_EINVAL;
     const int32_t pairs = d / 2;
     rope_table_kernel<<<(pairs + 255) / 256, 256, 0, as_stream(stream)>>>(d, rope_base, table);
     return launch_status();

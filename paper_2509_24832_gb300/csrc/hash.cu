@@ -6,15 +6,30 @@
 // For row i at position m: y = RoPE(x_i, m) (pair (2k, 2k+1) turned by m * theta_k),
 // p = R * bf16(y) with fp32 accumulation, code bit j = [p_j > 0].
 //
-// Kernel design (one persistent CTA per SM, 128-row tiles, 512 threads):
-//   warp 0        TMA producer: the tile's 128 x 64 embedding block (bf16 in place, or fp32
-//                 into a staging buffer) and the nbits x 64 hyperplane block, 128-byte swizzle
+// Work split (stream-K).  The n_tiles x n_kblocks (128-row tile, 64-wide K block) iterations
+// are cut into one equal contiguous range per CTA, one persistent CTA per SM, so every SM does
+// the same amount of rotation and MMA work even when there are fewer tiles than SMs.  A tile
+// covered by one CTA is finished in place.  A tile shared by several CTAs is finished by the
+// last of them to arrive: each writes its fp32 partial accumulator to its workspace slot,
+// fences, and bumps the tile's counter; the CTA that sees the count complete adds the partials
+// in K order (so the sum, and the codes, do not depend on arrival order), packs the signs and
+// puts the counter back to zero.  Nobody waits for another CTA.  The hand-off of a CTA's last
+// segment and every fix-up run after its main loop, shared by all 512 threads (the final
+// partial is staged through the then idle pipeline buffers).
+//
+// Roles inside a CTA (512 threads):
+//   warp 0        TMA producer: the 128 x 64 embedding block (bf16 in place, fp32 into a
+//                 staging buffer) and the nbits x 64 hyperplane block, 128-byte swizzle; the
+//                 embedding blocks are also prefetched into L2 two pipeline depths ahead
 //   warp 1        TMEM allocator and MMA issuer: 4 x tcgen05.mma (M=128, N=nbits, K=16) per
 //                 stage into one of two fp32 TMEM accumulators
-//   warps 4-11    RoPE: rotate each staged pair in shared memory, round to bf16 in the
-//                 operand tile, then hand the stage to the MMA warp
+//   warps 4-11    RoPE: rotate each staged pair in shared memory, round to bf16 in the operand
+//                 tile, hand the stage to the MMA warp; the next stage's rotation table entries
+//                 are fetched while the current one is processed.  A thread owns 4 pairs of 4
+//                 rows 32 apart: when their positions are 32 apart too, only the first row's
+//                 angles go through sincos and the others step by the 32-position rotation
 //   warps 12-15   epilogue: tcgen05.ld of the accumulator (lane = row), sign bits packed into
-//                 32-bit words per 32 columns, coalesced stores of codes (and projections)
+//                 32-bit words, or the partial-sum hand-off of a shared tile
 // Every pipeline wait is bounded; on timeout the CTA raises SEMSHARE_FLAG_TIMEOUT, lets its
 // copies and MMAs in flight finish, frees TMEM and returns.
 #include <cuda.h>
@@ -37,9 +52,12 @@ constexpr int kEpiWarp0 = 12;                  // 12 % 4 == 0: epilogue warp w r
 constexpr int kEpiWarps = 4;
 constexpr uint32_t kABytes = kBM * kBK * 2;    // bf16 operand tile, 16 KB
 constexpr uint32_t kF32Bytes = kBM * kBK * 4;  // fp32 staging: two 128-byte-wide boxes, 32 KB
+constexpr int kEpiBarrier = 1;                 // named barrier of the epilogue warps
+constexpr size_t kFixedSmem = 1024 + 512;      // alignment slack + barriers + TMEM slot + flags
 
 struct HashArgs {
     int64_t n;
+    int64_t total_iters;  // n_tiles * n_kblocks
     int32_t nbits;
     int32_t n_kblocks;
     int32_t n_tiles;
@@ -54,11 +72,24 @@ struct HashArgs {
     uint32_t* codes;
     float* proj;
     uint32_t* err_flag;
+    uint32_t* tile_count;  // workspace: [n_tiles] arrivals of shared tiles, zero between calls
+    float4* partials;      // workspace: [2 * gridDim.x][nbits/32][8][128] partial accumulators
     uint64_t wait_limit_ns;
 };
 
-// cos and sin of the rotation angle m * theta_k (Eq. 1).  turns_q64 = theta_k/(2*pi) as a
-// 0.64 fixed-point fraction, so bits 32..63 of m * turns_q64 (mod 2^64) are the angle's
+// First iteration of CTA b's range (b = gridDim.x gives the end).
+__device__ __forceinline__ int64_t range_begin(int64_t b, int64_t total, int64_t G) { return (b * total) / G; }
+
+// The CTA whose range holds iteration i.
+__device__ __forceinline__ int64_t range_owner(int64_t i, int64_t total, int64_t G) {
+    int64_t b = (i * G) / total;
+    while (b + 1 < G && range_begin(b + 1, total, G) <= i) ++b;
+    while (b > 0 && range_begin(b, total, G) > i) --b;
+    return b;
+}
+
+// cos and sin of the rotation angle m * theta_k (Eq. 1).  turns_q64 = frac(theta_k/(2*pi)) as
+// a 0.64 fixed-point fraction, so bits 32..63 of m * turns_q64 (mod 2^64) are the angle's
 // fraction of a full turn: the reduction modulo 2*pi is exact integer arithmetic for every
 // int32 position.  The fraction, centred on [-1/2, 1/2) and rounded to 23 bits, becomes a
 // float through the mantissa (a wrap from +1/2 to -1/2 is the same angle).
@@ -87,6 +118,69 @@ __device__ __forceinline__ bool drain_wait(uint32_t bar, uint32_t parity, uint64
     return true;
 }
 
+__device__ __forceinline__ void epilogue_sync() {
+    asm volatile("bar.sync %0, %1;" ::"n"(kEpiBarrier), "n"(kEpiWarps * 32) : "memory");
+}
+
+// AND of v over the epilogue warps (also a barrier among them): they continue or stop together,
+// so none can be left waiting at the hand-off barrier.
+__device__ __forceinline__ bool epilogue_all(bool v) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "bar.red.and.pred q, %2, %3, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}\n"
+        : "=r"(r)
+        : "r"(static_cast<uint32_t>(v)), "n"(kEpiBarrier), "n"(kEpiWarps * 32)
+        : "memory");
+    return r != 0;
+}
+
+// Table entries of the 4 pairs (kb*32 + 4c .. +3): turn fractions, and the rotation between
+// positions 32 apart (cos in the low word, sin in the high word).
+struct Pairs4 {
+    uint64_t turns[4];
+    uint64_t cis32[4];
+};
+
+__device__ __forceinline__ void load_pairs4(const uint64_t* table, int half, int kb, int c, Pairs4& t) {
+    const ulonglong2* tp = reinterpret_cast<const ulonglong2*>(table + kb * (kBK / 2) + c * 4);
+    const ulonglong2* cp = reinterpret_cast<const ulonglong2*>(table + half + kb * (kBK / 2) + c * 4);
+    const ulonglong2 t01 = __ldg(tp), t23 = __ldg(tp + 1), c01 = __ldg(cp), c23 = __ldg(cp + 1);
+    t.turns[0] = t01.x; t.turns[1] = t01.y; t.turns[2] = t23.x; t.turns[3] = t23.y;
+    t.cis32[0] = c01.x; t.cis32[1] = c01.y; t.cis32[2] = c23.x; t.cis32[3] = c23.y;
+}
+
+// Sign bits of 32 fp32 values given as bit patterns: bit j = [v_j > 0].
+__device__ __forceinline__ uint32_t sign_word(const uint32_t (&v)[32]) {
+    uint32_t bits = 0u;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) bits |= (static_cast<int32_t>(v[j]) > 0 ? 1u : 0u) << j;
+    return bits;
+}
+
+__device__ __forceinline__ void store_proj(float* proj, int64_t row, int nbits, int q, const uint32_t (&v)[32]) {
+    float4* pp = reinterpret_cast<float4*>(proj + row * nbits + q * 32);
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+        pp[j] = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]), __uint_as_float(v[4 * j + 2]),
+                            __uint_as_float(v[4 * j + 3]));
+}
+
+__device__ __forceinline__ void store_codes(uint32_t* codes, int64_t row, int W, const uint32_t (&words)[8]) {
+    uint32_t* cp = codes + row * W;
+    if ((W & 3) == 0) {
+#pragma unroll
+        for (int q = 0; q < 8; q += 4)
+            if (q < W) *reinterpret_cast<uint4*>(cp + q) = make_uint4(words[q], words[q + 1], words[q + 2], words[q + 3]);
+    } else {
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+            if (q < W) cp[q] = words[q];
+    }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     lsh_hash_kernel(const __grid_constant__ CUtensorMap tmap_emb, const __grid_constant__ CUtensorMap tmap_hyp,
                     const HashArgs a) {
@@ -105,9 +199,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem_slot = bar_mma_done + 8u;
     volatile uint32_t* const tmem_slot_ptr = reinterpret_cast<volatile uint32_t*>(gbase + (tmem_slot - sbase));
     volatile int* const abort_flag = reinterpret_cast<volatile int*>(gbase + (tmem_slot + 4u - sbase));
+    volatile uint32_t* const arrival = reinterpret_cast<volatile uint32_t*>(gbase + (tmem_slot + 8u - sbase));
+    // hand-off bookkeeping shared with the end phase: [0] final partial staged (0/1), [1] its tile,
+    // [2] its slot, [3] b_lo, [4] b_hi, [5] fix-ups pending, [6 + 3f ..] tile, b_lo, b_hi of fix-up f
+    volatile int64_t* const ctl = reinterpret_cast<volatile int64_t*>(gbase + (tmem_slot + 16u - sbase));
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
+    const int64_t G = gridDim.x;
+    const int64_t i0 = range_begin(blockIdx.x, a.total_iters, G);
+    const int64_t i1 = range_begin(static_cast<int64_t>(blockIdx.x) + 1, a.total_iters, G);
+    const int nkb = a.n_kblocks;
 
     if (threadIdx.x == 0) {
         for (uint32_t s = 0; s < S; ++s) {
@@ -121,6 +223,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         mbar_init(bar_mma_done, 1);
         *abort_flag = 0;
+        ctl[0] = 0;
+        ctl[5] = 0;
         fence_barrier_init();
     }
     if (warp == 0 && lane == 0) {
@@ -139,33 +243,50 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 0) {
         // ---------------- TMA producer ----------------
         if (lane == 0) {
-            uint32_t it = 0;
+            uint32_t q = 0;
             bool ok = true;
-            for (int tile = blockIdx.x; ok && tile < a.n_tiles; tile += gridDim.x) {
-                const int32_t row0 = tile * kBM;
-                for (int kb = 0; kb < a.n_kblocks; ++kb, ++it) {
-                    const uint32_t s = it % S, ph = (it / S) & 1u;
-                    if (!mbar_wait_bounded(bar_empty + 8u * s, ph ^ 1u, abort_flag, a.err_flag, SEMSHARE_FLAG_TIMEOUT,
-                                           a.wait_limit_ns)) {
-                        ok = false;
-                        break;
-                    }
-                    const uint32_t st = sbase + s * a.stage_bytes;
-                    const uint32_t full = bar_full + 8u * s;
-                    mbar_arrive_expect_tx(full, a.tx_bytes);
-                    if (a.is_f32) {
-                        const uint32_t stg = st + kABytes + a.b_bytes;
-                        tma_load_2d(stg, &tmap_emb, full, kb * kBK, row0);
-                        tma_load_2d(stg + kF32Bytes / 2, &tmap_emb, full, kb * kBK + 32, row0);
-                    } else {
-                        tma_load_2d(st, &tmap_emb, full, kb * kBK, row0);
-                    }
-                    tma_load_2d(st + kABytes, &tmap_hyp, full, kb * kBK, 0);
+            int tile = static_cast<int>(i0 / nkb), kb = static_cast<int>(i0 % nkb);
+            // L2 prefetch of the embedding blocks, 2*S iterations ahead of the loads
+            int pf_tile = tile, pf_kb = kb;
+            int64_t pf_it = i0;
+            auto prefetch_next = [&]() {
+                if (pf_it >= i1) return;
+                tma_prefetch_l2_2d(&tmap_emb, pf_kb * kBK, pf_tile * kBM);
+                if (a.is_f32) tma_prefetch_l2_2d(&tmap_emb, pf_kb * kBK + 32, pf_tile * kBM);
+                ++pf_it;
+                if (++pf_kb == nkb) {
+                    pf_kb = 0;
+                    ++pf_tile;
+                }
+            };
+            for (uint32_t i = 0; i < 2 * S; ++i) prefetch_next();
+            for (int64_t it = i0; it < i1; ++it, ++q) {
+                const uint32_t s = q % S, ph = (q / S) & 1u;
+                if (!mbar_wait_bounded(bar_empty + 8u * s, ph ^ 1u, abort_flag, a.err_flag, SEMSHARE_FLAG_TIMEOUT,
+                                       a.wait_limit_ns)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t st = sbase + s * a.stage_bytes;
+                const uint32_t full = bar_full + 8u * s;
+                mbar_arrive_expect_tx(full, a.tx_bytes);
+                if (a.is_f32) {
+                    const uint32_t stg = st + kABytes + a.b_bytes;
+                    tma_load_2d(stg, &tmap_emb, full, kb * kBK, tile * kBM);
+                    tma_load_2d(stg + kF32Bytes / 2, &tmap_emb, full, kb * kBK + 32, tile * kBM);
+                } else {
+                    tma_load_2d(st, &tmap_emb, full, kb * kBK, tile * kBM);
+                }
+                tma_load_2d(st + kABytes, &tmap_hyp, full, kb * kBK, 0);
+                prefetch_next();
+                if (++kb == nkb) {
+                    kb = 0;
+                    ++tile;
                 }
             }
             if (!ok) {
                 // the last issue of every stage may still be landing: wait for it before exit
-                for (uint32_t i = (it > S ? it - S : 0); i < it; ++i)
+                for (uint32_t i = (q > S ? q - S : 0); i < q; ++i)
                     drain_wait(bar_full + 8u * (i % S), (i / S) & 1u, kWaitLimitNs);
             }
         }
@@ -174,35 +295,38 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---------------- MMA issuer ----------------
         if (lane == 0) {
             const uint32_t idesc = umma_idesc_bf16_f32(kBM, a.nbits);
-            uint32_t it = 0, acc = 0;
-            bool ok = true;
-            for (int tile = blockIdx.x; ok && tile < a.n_tiles; tile += gridDim.x, ++acc) {
-                const uint32_t buf = acc & 1u, aph = (acc >> 1) & 1u;
-                if (!mbar_wait_bounded(bar_accempty + 8u * buf, aph ^ 1u, abort_flag, a.err_flag,
-                                       SEMSHARE_FLAG_TIMEOUT, a.wait_limit_ns)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after_sync();
-                const uint32_t d_tmem = tmem_base + buf * (a.tmem_cols >> 1);
-                for (int kb = 0; kb < a.n_kblocks; ++kb, ++it) {
-                    const uint32_t s = it % S, ph = (it / S) & 1u;
-                    if (!mbar_wait_bounded(bar_ready + 8u * s, ph, abort_flag, a.err_flag, SEMSHARE_FLAG_TIMEOUT,
-                                           a.wait_limit_ns)) {
-                        ok = false;
+            uint32_t q = 0, acc = 0, d_tmem = 0;
+            bool seg_first = true;
+            int kb = static_cast<int>(i0 % nkb);
+            for (int64_t it = i0; it < i1; ++it, ++q) {
+                if (seg_first) {
+                    const uint32_t buf = acc & 1u, aph = (acc >> 1) & 1u;
+                    if (!mbar_wait_bounded(bar_accempty + 8u * buf, aph ^ 1u, abort_flag, a.err_flag,
+                                           SEMSHARE_FLAG_TIMEOUT, a.wait_limit_ns))
                         break;
-                    }
                     tc_fence_after_sync();
-                    const uint32_t st = sbase + s * a.stage_bytes;
-#pragma unroll
-                    for (int k = 0; k < kBK / kUmmaK; ++k) {
-                        const uint64_t adesc = sw128_kmajor_desc(st + k * kUmmaK * 2);
-                        const uint64_t bdesc = sw128_kmajor_desc(st + kABytes + k * kUmmaK * 2);
-                        umma_bf16_ss(d_tmem, adesc, bdesc, idesc, (kb | k) != 0 ? 1u : 0u);
-                    }
-                    umma_commit(bar_empty + 8u * s);
+                    d_tmem = tmem_base + buf * (a.tmem_cols >> 1);
                 }
-                if (ok) umma_commit(bar_accfull + 8u * buf);
+                const uint32_t s = q % S, ph = (q / S) & 1u;
+                if (!mbar_wait_bounded(bar_ready + 8u * s, ph, abort_flag, a.err_flag, SEMSHARE_FLAG_TIMEOUT,
+                                       a.wait_limit_ns))
+                    break;
+                tc_fence_after_sync();
+                const uint32_t st = sbase + s * a.stage_bytes;
+#pragma unroll
+                for (int k = 0; k < kBK / kUmmaK; ++k) {
+                    const uint64_t adesc = sw128_kmajor_desc(st + k * kUmmaK * 2);
+                    const uint64_t bdesc = sw128_kmajor_desc(st + kABytes + k * kUmmaK * 2);
+                    umma_bf16_ss(d_tmem, adesc, bdesc, idesc, (seg_first && k == 0) ? 0u : 1u);
+                }
+                umma_commit(bar_empty + 8u * s);
+                const bool seg_last = (kb == nkb - 1) || (it == i1 - 1);
+                if (seg_last) {
+                    umma_commit(bar_accfull + 8u * (acc & 1u));
+                    ++acc;
+                }
+                seg_first = seg_last;
+                if (++kb == nkb) kb = 0;
             }
             // every MMA issued above has finished once this arrives: TMEM may then be freed
             umma_commit(bar_mma_done);
@@ -215,119 +339,280 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int c = rt & 7;                          // 16-byte chunk of the 128-byte row: pairs 4c..4c+3
         const int rg = rt >> 3;                        // rows rg + 32*i, i < 4 (all with row & 7 == rg & 7)
         const uint32_t swz = static_cast<uint32_t>(rg & 7);
-        uint32_t it = 0;
-        bool ok = true;
-        for (int tile = blockIdx.x; ok && tile < a.n_tiles; tile += gridDim.x) {
-            const int64_t row0 = static_cast<int64_t>(tile) * kBM;
-            uint32_t m[4];
+        const uint32_t chunk_off = (static_cast<uint32_t>(c) ^ swz) << 4;
+        uint32_t q = 0;
+        int tile = static_cast<int>(i0 / nkb), kb = static_cast<int>(i0 % nkb), cur_tile = -1;
+        const int half = nkb * (kBK / 2);  // d/2: start of the 32-position rotations in the table
+        uint32_t m[4] = {0u, 0u, 0u, 0u};
+        bool steps32 = false;
+        Pairs4 tn;
+        load_pairs4(a.rope_table, half, kb, c, tn);
+        for (int64_t it = i0; it < i1; ++it, ++q) {
+            if (tile != cur_tile) {
+                cur_tile = tile;
+                const int64_t row0 = static_cast<int64_t>(tile) * kBM;
+                const int64_t r0 = row0 + rg;
+                m[0] = r0 < a.n ? (a.positions ? static_cast<uint32_t>(__ldg(a.positions + r0)) : static_cast<uint32_t>(r0))
+                                : 0u;
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int64_t row = row0 + rg + 32 * i;
-                m[i] = row < a.n ? (a.positions ? static_cast<uint32_t>(__ldg(a.positions + row))
-                                                : static_cast<uint32_t>(row))
-                                 : 0u;
-            }
-            for (int kb = 0; kb < a.n_kblocks; ++kb, ++it) {
-                const uint32_t s = it % S, ph = (it / S) & 1u;
-                const bool got = mbar_wait_bounded(bar_full + 8u * s, ph, abort_flag, a.err_flag,
-                                                   SEMSHARE_FLAG_TIMEOUT, a.wait_limit_ns);
-                if (!__all_sync(0xFFFFFFFFu, got)) {
-                    ok = false;
-                    break;
+                for (int i = 1; i < 4; ++i) {
+                    // rows past n are zero-filled by TMA: any angle will do, keep the 32-step pattern
+                    const int64_t row = r0 + 32 * i;
+                    m[i] = row < a.n ? (a.positions ? static_cast<uint32_t>(__ldg(a.positions + row))
+                                                    : static_cast<uint32_t>(row))
+                                     : m[0] + 32u * i;
                 }
-                const ulonglong2* tp = reinterpret_cast<const ulonglong2*>(a.rope_table + kb * (kBK / 2) + c * 4);
-                const ulonglong2 t01 = __ldg(tp), t23 = __ldg(tp + 1);
-                const uint64_t T[4] = {t01.x, t01.y, t23.x, t23.y};
-                uint8_t* const st = gbase + s * a.stage_bytes;
+                steps32 = m[1] == m[0] + 32u && m[2] == m[0] + 64u && m[3] == m[0] + 96u;
+            }
+            const Pairs4 tc = tn;
+            const int kb_next = kb + 1 == nkb ? 0 : kb + 1;
+            if (it + 1 < i1) load_pairs4(a.rope_table, half, kb_next, c, tn);  // next stage's table entries
+
+            const uint32_t s = q % S, ph = (q / S) & 1u;
+            const bool got = mbar_wait_bounded(bar_full + 8u * s, ph, abort_flag, a.err_flag, SEMSHARE_FLAG_TIMEOUT,
+                                               a.wait_limit_ns);
+            if (!__all_sync(0xFFFFFFFFu, got)) break;
+            uint8_t* const st = gbase + s * a.stage_bytes;
+            float x[4][8];
+            if (a.is_f32) {
+                const uint32_t c0 = static_cast<uint32_t>((c & 3) * 2);
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
-                    const int r = rg + 32 * i;
-                    uint4* const dst = reinterpret_cast<uint4*>(st + r * 128 + ((static_cast<uint32_t>(c) ^ swz) << 4));
-                    float x[8];
-                    if (a.is_f32) {
-                        const uint8_t* stg = st + kABytes + a.b_bytes + (c >> 2) * (kF32Bytes / 2) + r * 128;
-                        const uint32_t c0 = static_cast<uint32_t>((c & 3) * 2);
-                        const float4 f0 = *reinterpret_cast<const float4*>(stg + ((c0 ^ swz) << 4));
-                        const float4 f1 = *reinterpret_cast<const float4*>(stg + (((c0 + 1u) ^ swz) << 4));
-                        x[0] = f0.x; x[1] = f0.y; x[2] = f0.z; x[3] = f0.w;
-                        x[4] = f1.x; x[5] = f1.y; x[6] = f1.z; x[7] = f1.w;
-                    } else {
-                        const uint4 v = *dst;
-                        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+                    const uint8_t* stg = st + kABytes + a.b_bytes + (c >> 2) * (kF32Bytes / 2) + (rg + 32 * i) * 128;
+                    const float4 f0 = *reinterpret_cast<const float4*>(stg + ((c0 ^ swz) << 4));
+                    const float4 f1 = *reinterpret_cast<const float4*>(stg + (((c0 + 1u) ^ swz) << 4));
+                    x[i][0] = f0.x; x[i][1] = f0.y; x[i][2] = f0.z; x[i][3] = f0.w;
+                    x[i][4] = f1.x; x[i][5] = f1.y; x[i][6] = f1.z; x[i][7] = f1.w;
+                }
+            } else {
 #pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            x[2 * q] = __uint_as_float(w[q] << 16);
-                            x[2 * q + 1] = __uint_as_float(w[q] & 0xFFFF0000u);
+                for (int i = 0; i < 4; ++i) {
+                    const uint4 v = *reinterpret_cast<const uint4*>(st + (rg + 32 * i) * 128 + chunk_off);
+                    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                    for (int p = 0; p < 4; ++p) {
+                        x[i][2 * p] = __uint_as_float(w[p] << 16);
+                        x[i][2 * p + 1] = __uint_as_float(w[p] & 0xFFFF0000u);
+                    }
+                }
+            }
+            uint32_t y[4][4];
+            if (steps32) {
+                // row i+1 sits 32 positions after row i: turn the angle on by the 32-step rotation
+                float cs[4], sn[4];
+#pragma unroll
+                for (int p = 0; p < 4; ++p) rotation(m[0], tc.turns[p], cs[p], sn[p]);
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int p = 0; p < 4; ++p) {
+                        y[i][p] = rotate_to_bf16(x[i][2 * p], x[i][2 * p + 1], cs[p], sn[p]);
+                        if (i < 3) {
+                            const float c32 = __uint_as_float(static_cast<uint32_t>(tc.cis32[p]));
+                            const float s32 = __uint_as_float(static_cast<uint32_t>(tc.cis32[p] >> 32));
+                            const float nc = fmaf(cs[p], c32, -sn[p] * s32);
+                            sn[p] = fmaf(cs[p], s32, sn[p] * c32);
+                            cs[p] = nc;
                         }
                     }
-                    uint32_t y[4];
+            } else {
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int p = 0; p < 4; ++p) {
                         float cs, sn;
-                        rotation(m[i], T[q], cs, sn);
-                        y[q] = rotate_to_bf16(x[2 * q], x[2 * q + 1], cs, sn);
+                        rotation(m[i], tc.turns[p], cs, sn);
+                        y[i][p] = rotate_to_bf16(x[i][2 * p], x[i][2 * p + 1], cs, sn);
                     }
-                    *dst = make_uint4(y[0], y[1], y[2], y[3]);
-                }
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(bar_ready + 8u * s);
             }
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                *reinterpret_cast<uint4*>(st + (rg + 32 * i) * 128 + chunk_off) =
+                    make_uint4(y[i][0], y[i][1], y[i][2], y[i][3]);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_ready + 8u * s);
+            kb = kb_next;
+            if (kb == 0) ++tile;
         }
     } else if (warp >= kEpiWarp0) {
-        // ---------------- epilogue: signs -> packed codes ----------------
+        // ---------------- epilogue: signs -> packed codes, or partial hand-off ----------------
         const int ew = warp - kEpiWarp0;
+        const int r = ew * 32 + lane;  // row within the tile == TMEM lane
         const int W = a.nbits >> 5;
         uint32_t acc = 0;
-        for (int tile = blockIdx.x; tile < a.n_tiles; tile += gridDim.x, ++acc) {
+        for (int64_t it = i0; it < i1; ++acc) {
+            const int tile = static_cast<int>(it / nkb);
+            const int kb_begin = static_cast<int>(it - static_cast<int64_t>(tile) * nkb);
+            const int64_t seg_len = (i1 - it) < (nkb - kb_begin) ? (i1 - it) : (nkb - kb_begin);
+            const bool whole = kb_begin == 0 && seg_len == nkb;
+            const bool last_seg = it + seg_len == i1;
+            const int64_t tile_it0 = static_cast<int64_t>(tile) * nkb;
+            int64_t b_lo = 0, b_hi = 0;
+            if (!whole) {  // contributors of this tile, worked out while its MMAs run
+                b_lo = range_owner(tile_it0, a.total_iters, G);
+                b_hi = range_owner(tile_it0 + nkb - 1, a.total_iters, G);
+            }
             const uint32_t buf = acc & 1u, aph = (acc >> 1) & 1u;
             const bool got = mbar_wait_bounded(bar_accfull + 8u * buf, aph, abort_flag, a.err_flag,
                                                SEMSHARE_FLAG_TIMEOUT, a.wait_limit_ns);
-            if (!__all_sync(0xFFFFFFFFu, got)) break;
+            if (!epilogue_all(got)) break;
             tc_fence_after_sync();
-            const int64_t row = static_cast<int64_t>(tile) * kBM + ew * 32 + lane;
-            const uint32_t taddr =
-                tmem_base + (static_cast<uint32_t>(ew * 32) << 16) + buf * (a.tmem_cols >> 1);
-            uint32_t words[8];
+            const int64_t row = static_cast<int64_t>(tile) * kBM + r;
+            const uint32_t taddr = tmem_base + (static_cast<uint32_t>(ew * 32) << 16) + buf * (a.tmem_cols >> 1);
+            if (whole) {
+                uint32_t words[8];
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                words[q] = 0u;
-                if (q < W) {
-                    uint32_t v[32];
-                    tmem_load_32cols(taddr + q * 32, v);
-                    tmem_load_wait();
-                    uint32_t bits = 0u;
+                for (int qq = 0; qq < 8; ++qq) {
+                    words[qq] = 0u;
+                    if (qq < W) {
+                        uint32_t v[32];
+                        tmem_load_32cols(taddr + qq * 32, v);
+                        tmem_load_wait();
+                        words[qq] = sign_word(v);
+                        if (a.proj != nullptr && row < a.n) store_proj(a.proj, row, a.nbits, qq, v);
+                    }
+                }
+                tc_fence_before_sync();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar_accempty + 8u * buf);
+                if (row < a.n) store_codes(a.codes, row, W, words);
+            } else {
+                // shared tile: this CTA's partial sum goes to its workspace slot.  The last segment's
+                // is staged in the idle pipeline buffers and published by the whole CTA at the end.
+                const int64_t slot = 2 * static_cast<int64_t>(blockIdx.x) + (i0 >= tile_it0 ? 0 : 1);
+                float4* dst = last_seg ? reinterpret_cast<float4*>(gbase) : a.partials + slot * W * 8 * kBM;
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) bits |= (static_cast<int32_t>(v[j]) > 0 ? 1u : 0u) << j;
-                    words[q] = bits;
-                    if (a.proj != nullptr && row < a.n) {
-                        float4* pp = reinterpret_cast<float4*>(a.proj + row * a.nbits + q * 32);
+                for (int qq = 0; qq < 8; ++qq) {
+                    if (qq < W) {
+                        uint32_t v[32];
+                        tmem_load_32cols(taddr + qq * 32, v);
+                        tmem_load_wait();
 #pragma unroll
                         for (int j = 0; j < 8; ++j)
-                            pp[j] = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
-                                                __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+                            dst[(qq * 8 + j) * kBM + r] =
+                                make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                                            __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+                    }
+                }
+                tc_fence_before_sync();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar_accempty + 8u * buf);
+                if (last_seg) {
+                    if (threadIdx.x == kEpiWarp0 * 32) {
+                        ctl[1] = tile;
+                        ctl[2] = slot;
+                        ctl[3] = b_lo;
+                        ctl[4] = b_hi;
+                        ctl[0] = 1;
+                    }
+                } else {
+                    __threadfence();
+                    epilogue_sync();
+                    if (threadIdx.x == kEpiWarp0 * 32) {
+                        if (atomicAdd(a.tile_count + tile, 1u) == static_cast<uint32_t>(b_hi - b_lo)) {
+                            const int64_t f = ctl[5];
+                            ctl[6 + 3 * f] = tile;
+                            ctl[7 + 3 * f] = b_lo;
+                            ctl[8 + 3 * f] = b_hi;
+                            ctl[5] = f + 1;
+                        }
                     }
                 }
             }
-            tc_fence_before_sync();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar_accempty + 8u * buf);
-            if (row < a.n) {
-                uint32_t* cp = a.codes + row * W;
-                if ((W & 3) == 0) {
-#pragma unroll
-                    for (int q = 0; q < 8; q += 4)
-                        if (q < W) *reinterpret_cast<uint4*>(cp + q) = make_uint4(words[q], words[q + 1], words[q + 2], words[q + 3]);
-                } else {
-#pragma unroll
-                    for (int q = 0; q < 8; ++q)
-                        if (q < W) cp[q] = words[q];
-                }
-            }
+            it += seg_len;
         }
     }
 
     tc_fence_before_sync();
+    __syncthreads();
+
+    // ---------------- end phase: publish the final partial, finish the tiles this CTA closes ----
+    if (*abort_flag == 0) {
+        const int W = a.nbits >> 5;
+        const int items = W * 8 * kBM;  // float4 per partial slot
+        if (ctl[0]) {
+            const float4* stage = reinterpret_cast<const float4*>(gbase);
+            float4* dst = a.partials + ctl[2] * items;
+            for (int e = threadIdx.x; e < items; e += kThreads) dst[e] = stage[e];
+            __threadfence();
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                const int64_t tile = ctl[1];
+                if (atomicAdd(a.tile_count + tile, 1u) == static_cast<uint32_t>(ctl[4] - ctl[3])) {
+                    const int64_t f = ctl[5];
+                    ctl[6 + 3 * f] = tile;
+                    ctl[7 + 3 * f] = ctl[3];
+                    ctl[8 + 3 * f] = ctl[4];
+                    ctl[5] = f + 1;
+                }
+            }
+            __syncthreads();
+        }
+        const int n_fix = static_cast<int>(ctl[5]);
+        for (int f = 0; f < n_fix; ++f) {
+            // every partial of the tile is in place: add them in K order (contributor order)
+            __threadfence();
+            const int tile = static_cast<int>(ctl[6 + 3 * f]);
+            const int64_t b_lo = ctl[7 + 3 * f], b_hi = ctl[8 + 3 * f];
+            const int64_t tile_it0 = static_cast<int64_t>(tile) * nkb;
+            for (int e = threadIdx.x; e < W * kBM; e += kThreads) {
+                const int qq = e / kBM, rr = e % kBM;
+                float sum[32];
+#pragma unroll
+                for (int j = 0; j < 32; ++j) sum[j] = 0.0f;
+                int64_t bb = b_lo;
+                for (; bb + 1 <= b_hi; bb += 2) {  // two contributors' loads in flight at once
+                    const int64_t s0 = 2 * bb + (range_begin(bb, a.total_iters, G) >= tile_it0 ? 0 : 1);
+                    const int64_t s1 = 2 * (bb + 1) + (range_begin(bb + 1, a.total_iters, G) >= tile_it0 ? 0 : 1);
+                    const float4* p0 = a.partials + s0 * items + qq * 8 * kBM + rr;
+                    const float4* p1 = a.partials + s1 * items + qq * 8 * kBM + rr;
+                    float4 f0[8], f1[8];
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        f0[j] = __ldcg(p0 + j * kBM);
+                        f1[j] = __ldcg(p1 + j * kBM);
+                    }
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        sum[4 * j] += f0[j].x;
+                        sum[4 * j + 1] += f0[j].y;
+                        sum[4 * j + 2] += f0[j].z;
+                        sum[4 * j + 3] += f0[j].w;
+                    }
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        sum[4 * j] += f1[j].x;
+                        sum[4 * j + 1] += f1[j].y;
+                        sum[4 * j + 2] += f1[j].z;
+                        sum[4 * j + 3] += f1[j].w;
+                    }
+                }
+                if (bb <= b_hi) {
+                    const int64_t s0 = 2 * bb + (range_begin(bb, a.total_iters, G) >= tile_it0 ? 0 : 1);
+                    const float4* p0 = a.partials + s0 * items + qq * 8 * kBM + rr;
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        const float4 f0 = __ldcg(p0 + j * kBM);
+                        sum[4 * j] += f0.x;
+                        sum[4 * j + 1] += f0.y;
+                        sum[4 * j + 2] += f0.z;
+                        sum[4 * j + 3] += f0.w;
+                    }
+                }
+                uint32_t v[32];
+#pragma unroll
+                for (int j = 0; j < 32; ++j) v[j] = __float_as_uint(sum[j]);
+                const int64_t row = static_cast<int64_t>(tile) * kBM + rr;
+                if (row < a.n) {
+                    a.codes[row * W + qq] = sign_word(v);
+                    if (a.proj != nullptr) store_proj(a.proj, row, a.nbits, qq, v);
+                }
+            }
+            if (threadIdx.x == 0) a.tile_count[tile] = 0u;  // leave the workspace zeroed
+        }
+    }
+
     __syncthreads();
     if (warp == 1) {
         tc_fence_after_sync();
@@ -361,13 +646,43 @@ bool encode_2d(CUtensorMap* map, CUtensorMapDataType type, const void* base, uin
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Grid and workspace of one call: one CTA per SM (fewer if there are fewer iterations), a
+// 256-byte-aligned array of per-tile counters, then two partial-accumulator slots per CTA.
+struct HashPlan {
+    int64_t n_tiles;
+    int64_t total_iters;
+    int grid;
+    size_t count_bytes;
+    size_t partial_bytes;
+};
+
+semshare_status plan_hash(int64_t n, int32_t d, int32_t nbits, HashPlan* p) {
+    int sms = 0;
+    if (current_sm_count(&sms, nullptr) != SEMSHARE_OK) return SEMSHARE_ECUDA;
+    p->n_tiles = (n + kBM - 1) / kBM;
+    p->total_iters = p->n_tiles * (d / kBK);
+    p->grid = static_cast<int>(p->total_iters < sms ? p->total_iters : sms);
+    p->count_bytes = ((static_cast<size_t>(p->n_tiles) * 4 + 255) / 256) * 256;
+    p->partial_bytes = static_cast<size_t>(2) * p->grid * kBM * static_cast<size_t>(nbits) * 4;
+    return SEMSHARE_OK;
+}
+
 }  // namespace
 }  // namespace semshare
+
+extern "C" size_t semshare_hash_workspace_size(int64_t n, int32_t d, int32_t nbits) {
+    using namespace semshare;
+    if (n <= 0 || d < kBK || d % kBK != 0 || nbits < 32 || nbits > 256 || nbits % 32 != 0) return 0;
+    HashPlan p;
+    if (plan_hash(n, d, nbits, &p) != SEMSHARE_OK) return 0;
+    return p.count_bytes + p.partial_bytes;
+}
 
 extern "C" semshare_status semshare_hash(const void* emb, semshare_dtype dtype, int64_t n, int32_t d,
                                          int64_t row_stride, const int32_t* positions, const uint64_t* rope_table,
                                          const uint16_t* hyperplanes, int32_t nbits, uint32_t* codes,
-                                         float* proj_out, uint32_t* err_flag, void* stream) {
+                                         float* proj_out, void* workspace, size_t workspace_bytes,
+                                         uint32_t* err_flag, void* stream) {
     using namespace semshare;
     if (dtype != SEMSHARE_BF16 && dtype != SEMSHARE_F32) return SEMSHARE_EINVAL;
     if (n < 0 || d <= 0 || (d & 1) || row_stride < d) return SEMSHARE_EINVAL;
@@ -377,24 +692,28 @@ extern "C" semshare_status semshare_hash(const void* emb, semshare_dtype dtype, 
     const int64_t esize = dtype == SEMSHARE_BF16 ? 2 : 4;
     if ((row_stride * esize) % 16 != 0) return SEMSHARE_EINVAL;
     if (n == 0) return SEMSHARE_OK;
-    if (!emb || !rope_table || !hyperplanes || !codes) return SEMSHARE_EINVAL;
-    if (!aligned(emb, 16) || !aligned(rope_table, 16) || !aligned(hyperplanes, 16) || !aligned(codes, 16))
+    if (!emb || !rope_table || !hyperplanes || !codes || !workspace) return SEMSHARE_EINVAL;
+    if (!aligned(emb, 16) || !aligned(rope_table, 16) || !aligned(hyperplanes, 16) || !aligned(codes, 16) ||
+        !aligned(workspace, 256))
         return SEMSHARE_EINVAL;
     if ((proj_out && !aligned(proj_out, 16)) || (positions && !aligned(positions, 4)) ||
         (err_flag && !aligned(err_flag, 4)))
         return SEMSHARE_EINVAL;
 
-    int sms = 0, dev = 0;
-    if (current_sm_count(&sms, &dev) != SEMSHARE_OK) return SEMSHARE_ECUDA;
-    int smem_optin = 0;
-    if (cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+    HashPlan plan;
+    if (plan_hash(n, d, nbits, &plan) != SEMSHARE_OK) return SEMSHARE_ECUDA;
+    if (workspace_bytes < plan.count_bytes + plan.partial_bytes) return SEMSHARE_EINVAL;
+    int dev = 0, smem_optin = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
         return SEMSHARE_ECUDA;
 
     HashArgs a{};
     a.n = n;
+    a.total_iters = plan.total_iters;
     a.nbits = nbits;
     a.n_kblocks = d / kBK;
-    a.n_tiles = static_cast<int32_t>((n + kBM - 1) / kBM);
+    a.n_tiles = static_cast<int32_t>(plan.n_tiles);
     a.is_f32 = dtype == SEMSHARE_F32;
     a.b_bytes = static_cast<uint32_t>(nbits) * kBK * 2;
     a.stage_bytes = kABytes + a.b_bytes + (a.is_f32 ? kF32Bytes : 0u);
@@ -402,16 +721,20 @@ extern "C" semshare_status semshare_hash(const void* emb, semshare_dtype dtype, 
     uint32_t cols = 32;
     while (cols < 2u * static_cast<uint32_t>(nbits)) cols <<= 1;
     a.tmem_cols = cols;
-    const size_t fixed = 1024 + 256;  // alignment slack + barriers + TMEM slot + abort flag
+    const size_t fixed = kFixedSmem;
     int stages = static_cast<int>((static_cast<size_t>(smem_optin) - fixed) / a.stage_bytes);
     if (stages > 6) stages = 6;
     if (stages < 2) return SEMSHARE_EUNSUPPORTED;
+    // the last segment's partial accumulator (128 x nbits fp32) is staged in the stage buffers
+    if (static_cast<size_t>(stages) * a.stage_bytes < static_cast<size_t>(kBM) * nbits * 4) return SEMSHARE_EUNSUPPORTED;
     a.stages = stages;
     a.positions = positions;
     a.rope_table = rope_table;
     a.codes = codes;
     a.proj = proj_out;
     a.err_flag = err_flag;
+    a.tile_count = static_cast<uint32_t*>(workspace);
+    a.partials = reinterpret_cast<float4*>(static_cast<uint8_t*>(workspace) + plan.count_bytes);
     a.wait_limit_ns = kWaitLimitNs;
     const size_t smem = fixed + static_cast<size_t>(stages) * a.stage_bytes;
 
@@ -427,7 +750,6 @@ extern "C" semshare_status semshare_hash(const void* emb, semshare_dtype dtype, 
     if (cudaFuncSetAttribute(lsh_hash_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
         cudaSuccess)
         return SEMSHARE_ECUDA;
-    const int grid = a.n_tiles < sms ? a.n_tiles : sms;
-    lsh_hash_kernel<<<grid, kThreads, smem, as_stream(stream)>>>(tm_emb, tm_hyp, a);
+    lsh_hash_kernel<<<plan.grid, kThreads, smem, as_stream(stream)>>>(tm_emb, tm_hyp, a);
     return launch_status();
 }

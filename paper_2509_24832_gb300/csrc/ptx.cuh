@@ -83,6 +83,13 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const void* desc, uint
         : "memory");
 }
 
+// Brings the box at (x, y) into L2 ahead of its load (no shared memory, no completion).
+__device__ __forceinline__ void tma_prefetch_l2_2d(const void* desc, int32_t x, int32_t y) {
+    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global [%0, {%1, %2}];" ::"l"(reinterpret_cast<uint64_t>(desc)),
+                 "r"(x), "r"(y)
+                 : "memory");
+}
+
 // Orders this thread's generic-proxy shared-memory writes before later async-proxy reads
 // (tcgen05.mma operands) of the same bytes.
 __device__ __forceinline__ void fence_proxy_async_smem() {

@@ -50,10 +50,11 @@ FAKE = ctypes.c_void_p(1 << 20)  # aligned, never dereferenced: every case below
 
 def _hash(lib, **kw):
     a = dict(emb=FAKE, dtype=0, n=10, d=128, row_stride=128, positions=None, table=FAKE, hyp=FAKE, nbits=64,
-             codes=FAKE, proj=None, flag=None, stream=None)
+             codes=FAKE, proj=None, ws=FAKE, ws_bytes=1 << 30, flag=None, stream=None)
     a.update(kw)
     return lib.semshare_hash(a["emb"], a["dtype"], a["n"], a["d"], a["row_stride"], a["positions"], a["table"],
-                             a["hyp"], a["nbits"], a["codes"], a["proj"], a["flag"], a["stream"])
+                             a["hyp"], a["nbits"], a["codes"], a["proj"], a["ws"], a["ws_bytes"], a["flag"],
+                             a["stream"])
 
 
 def test_hash_argument_errors(lib):
@@ -69,6 +70,8 @@ def test_hash_argument_errors(lib):
     assert _hash(lib, emb=ctypes.c_void_p((1 << 20) + 4)) == 1  # misaligned
     assert _hash(lib, codes=None) == 1
     assert _hash(lib, n=1 << 31) == 2
+    assert _hash(lib, ws=None) == 1
+    assert _hash(lib, ws=ctypes.c_void_p((1 << 20) + 16)) == 1  # workspace not 256-byte aligned
     assert _hash(lib, n=0, emb=None, codes=None) == 0    # empty: nothing to do
 
 

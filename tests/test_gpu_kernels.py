@@ -132,6 +132,18 @@ def test_hash_empty_and_repeatable(ss):
     a = ss.semshare_hash(x, table, R)
     b = ss.semshare_hash(x, table, R)
     assert torch.equal(a, b)
+    # the shared-tile counters are back at zero after every call
+    ws = ss.hash_workspace(300, 128, 64)
+    torch.cuda.synchronize()
+    assert int(ws[: 256].count_nonzero()) == 0
+
+
+def test_hash_stream_k_split_tiles_are_deterministic(ss, orc):
+    # 3 tiles x 64 K blocks over all SMs: every tile is shared by many CTAs
+    gc1, gp1, oc, op, emb, pos, R = _hash_case(ss, orc, 300, 4096, 256, "bf16", "own", seed=5)
+    gc2, gp2, _, _, _, _, _ = _hash_case(ss, orc, 300, 4096, 256, "bf16", "own", seed=5)
+    assert np.array_equal(gc1, gc2) and np.array_equal(gp1, gp2)
+    check_hash(gc1, gp1, oc, op)
 
 
 # ---- match ----------------------------------------------------------------------------------
