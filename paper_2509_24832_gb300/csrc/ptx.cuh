@@ -47,6 +47,21 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     return done != 0;
 }
 
+// Like mbar_try_wait, but lets the hardware suspend the thread for up to `hint_ns` while the
+// phase is incomplete (it resumes as soon as the phase completes), so a waiting warp does
+// not take issue slots from the warps that are working.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity, uint32_t hint_ns) {
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}\n"
+        : "=r"(done)
+        : "r"(bar), "r"(parity), "r"(hint_ns)
+        : "memory");
+    return done != 0;
+}
+
 // Waits for the phase of `bar` with parity `parity` to complete.  Gives up, returning false,
 // when another thread of the CTA has raised *abort or when `limit_ns` nanoseconds pass; in
 // the second case it raises *abort itself and ORs `timeout_bit` into *err (if non-null).
@@ -55,8 +70,8 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = global_timer_ns();
     for (uint32_t i = 1;; ++i) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if ((i & 31u) == 0u) {
+        if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+        if ((i & 3u) == 0u) {
             if (*abort_flag) return false;
             if (global_timer_ns() - t0 > limit_ns) {
                 *abort_flag = 1;
