@@ -38,7 +38,7 @@ METRIC = "target tokens matched+gathered/sec at 5k tokens"
 DEFAULT_WORKLOAD = "llama8b-5k"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 L2_FLUSH_BYTES = 256 << 20
-LAUNCHES_PER_STEP = 5  # hash 1, match 3 (key init, search, split), gather 1
+LAUNCHES_PER_STEP = 5  # hash 1, match 3 (tc: expand + key reset, search, split; popc: key init, search, split), gather 1
 
 # DRAM bytes per launch from ncu captures (dram__bytes_read.sum + dram__bytes_write.sum),
 # valid only while the kernel source has the recorded sha256 prefix.
@@ -56,6 +56,8 @@ def parse_args(argv=None):
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads.WORKLOADS))
     p.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    p.add_argument("--matcher", default="tc", choices=["tc", "popc"],
+                   help="Hamming search: tensor-core GEMM (semshare_match_tc) or xor/popc (semshare_match)")
     p.add_argument("--e2e-steps", type=int, default=20)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-clocks", action="store_true")
@@ -191,12 +193,12 @@ class ClockSampler:
 class Problem:
     """Device buffers of one matching problem and the three library calls of a step."""
 
-    def __init__(self, wl: workloads.Workload, device, seed: int):
+    def __init__(self, wl: workloads.Workload, device, seed: int, matcher: str = "tc"):
         import torch
 
         import paper_2509_24832_gb300 as ss
 
-        self.ss, self.wl, self.dev = ss, wl, device
+        self.ss, self.wl, self.dev, self.matcher = ss, wl, device, matcher
         emb, pos, _ = workloads.prompt_rows(wl, seed=seed)
         self.host_emb, self.host_pos = emb, pos
         if wl.emb_dtype == "f32":
@@ -214,6 +216,8 @@ class Problem:
         self.idx = torch.empty(n_t, dtype=torch.int32, device=device)
         self.dist = torch.empty(n_t, dtype=torch.int32, device=device)
         self.ws = torch.empty(ss.semshare_match_workspace_size(n_t), dtype=torch.uint8, device=device)
+        self.tc_ws = torch.empty(max(256, ss.semshare_match_tc_workspace_size(n_t, wl.n_ref, wl.nbits)),
+                                 dtype=torch.uint8, device=device)
         self.hash_ws = torch.zeros(max(256, ss.semshare_hash_workspace_size(rows, wl.d, wl.nbits)), dtype=torch.uint8,
                                    device=device)
         segs = [workloads.kv_cache_device(wl, device, seed=seed, segment=s) for s in range(wl.n_seg)]
@@ -230,8 +234,12 @@ class Problem:
 
     def match(self):
         n_ref = self.wl.n_ref
-        self.ss.semshare_match(self.codes[n_ref:], self.codes[:n_ref], idx=self.idx, dist=self.dist,
-                               workspace=self.ws)
+        if self.matcher == "tc":
+            self.ss.semshare_match_tc(self.codes[n_ref:], self.codes[:n_ref], idx=self.idx, dist=self.dist,
+                                      workspace=self.tc_ws, err_flag=self.flag)
+        else:
+            self.ss.semshare_match(self.codes[n_ref:], self.codes[:n_ref], idx=self.idx, dist=self.dist,
+                                   workspace=self.ws)
 
     def gather(self):
         self.ss.semshare_gather_kv(self.ref_k, self.ref_v, self.idx.view(self.wl.n_batch, self.wl.n_tgt),
@@ -261,7 +269,7 @@ def run_gpu_arm(args, rank, world, local_rank):
     torch.cuda.set_device(device)
     wl = workloads.WORKLOADS[args.workload]
     seed = wl.base_seed + 7919 * rank
-    prob = Problem(wl, device, seed)
+    prob = Problem(wl, device, seed, args.matcher)
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
 
     for _ in range(max(args.warmup, 3)):
@@ -312,7 +320,15 @@ def run_gpu_arm(args, rank, world, local_rank):
     stages["hash"]["frac_tensor"] = stages["hash"]["tflops"] / peaks["bf16_tflops"]
     stages["hash"]["frac_hbm"] = stages["hash"]["gbs"] / peaks["hbm_gbs"]
     popc_peak = popc_peak_wordops(sm_mhz, props.multi_processor_count)
-    stages["match"]["frac_popc"] = stages["match"]["gwordops"] * 1e9 / popc_peak
+    stages["match"]["matcher"] = args.matcher
+    if args.matcher == "popc":
+        stages["match"]["frac_popc"] = stages["match"]["gwordops"] * 1e9 / popc_peak
+    else:
+        # the GEMM over padded code bits: 2 * n_t * n_ref * kpad fp8 flops; fp8 peak = 2 x bf16 (nominal ratio)
+        kpad = ((wl.nbits + 127) // 128) * 128
+        fl = 2.0 * W["targets"] * wl.n_ref * kpad
+        stages["match"]["tflops_fp8"] = fl / (stage_ms["match"] * 1e-3) / 1e12
+        stages["match"]["frac_fp8_tensor"] = stages["match"]["tflops_fp8"] / (2.0 * peaks["bf16_tflops"])
     stages["gather"]["frac_hbm"] = stages["gather"]["gbs"] / peaks["hbm_gbs"]
 
     dominant = max(stage_ms, key=stage_ms.get)
@@ -324,10 +340,14 @@ def run_gpu_arm(args, rank, world, local_rank):
         roof = {"kernel": "lsh_hash_kernel", "bound": "tensor", "achieved": stages["hash"]["tflops"],
                 "peak": peaks["bf16_tflops"], "unit": "TFLOP/s"}
         tr = NCU_TRAFFIC.get("hash")
-    else:
+    elif args.matcher == "popc":
         roof = {"kernel": "hamming_nn_kernel", "bound": "alu", "achieved": stages["match"]["gwordops"],
                 "peak": popc_peak / 1e9, "unit": "Gwordop/s"}
         tr = NCU_TRAFFIC.get("match")
+    else:
+        roof = {"kernel": "hamming_tc_kernel", "bound": "tensor", "achieved": stages["match"]["tflops_fp8"],
+                "peak": 2.0 * peaks["bf16_tflops"], "unit": "TFLOP/s"}
+        tr = None
     roof["frac"] = roof["achieved"] / roof["peak"]
     roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"
     if tr and tr.get("sha") == kernel_sha(tr["file"]):
@@ -348,7 +368,8 @@ def run_gpu_arm(args, rank, world, local_rank):
         "data": "synthetic (seeded; see workloads.py)",
         "config": {"workload": wl.name, "n_ref": wl.n_ref, "n_tgt": wl.n_tgt, "n_batch": wl.n_batch,
                    "n_seg": wl.n_seg, "d": wl.d, "nbits": wl.nbits, "kv": list(wl.kv),
-                   "parallelism": f"replicas x{world}", "l2": "flushed before every step (256 MB write)"},
+                   "parallelism": f"replicas x{world}", "l2": "flushed before every step (256 MB write)",
+                   "matcher": args.matcher},
         "roofline": roof, "stages": stages, "e2e": e2e, "cpu_baseline": cpu,
         "gpu_launches": LAUNCHES_PER_STEP * K, "clocks": clocks, "wall_s_timed": reduce_max(t_wall, device),
         "impl": "gb300",

@@ -152,6 +152,27 @@ semshare_status semshare_match(const uint32_t* tgt_codes, int64_t n_tgt, const u
                                void* stream);
 
 /*
+ * semshare_match_tc -- step 3 on the tensor cores: exactly semshare_match's result.
+ *
+ * Same problem and tie rule as semshare_match (Sec. 3.3: the most similar reference token of
+ * each target token).  With s = 2*bit - 1, popcount(a XOR b) = (nbits - <s_a, s_b>) / 2, so
+ * the all-pairs distances are one dense contraction: the codes are expanded to fp8 +-1 rows
+ * and multiplied on the tcgen05 tensor cores (fp32 accumulation, exact for these integers),
+ * and each row of the product is reduced to its best reference on the fly.
+ *
+ *   arguments as for semshare_match, plus
+ *   workspace  device scratch of at least semshare_match_tc_workspace_size(n_tgt, n_ref, nbits)
+ *              bytes, 256-byte aligned; contents on entry do not matter, overwritten
+ *   err_flag   device or NULL; SEMSHARE_FLAG_TIMEOUT is OR-ed in if a pipeline wait of the
+ *              kernel exceeds its limit (idx/dist are then incomplete)
+ * tgt_codes and ref_codes need only 4-byte alignment here.  Returns as semshare_match.
+ */
+size_t semshare_match_tc_workspace_size(int64_t n_tgt, int64_t n_ref, int32_t nbits);
+semshare_status semshare_match_tc(const uint32_t* tgt_codes, int64_t n_tgt, const uint32_t* ref_codes, int64_t n_ref,
+                                  int32_t nbits, int32_t* idx, int32_t* dist, void* workspace, size_t workspace_bytes,
+                                  uint32_t* err_flag, void* stream);
+
+/*
  * semshare_match_static -- semshare_match without a caller-provided workspace.
  *
  * The paper has no counterpart: this entry point exists for callers that cannot allocate

@@ -26,6 +26,8 @@ from ._native import (  # noqa: F401
     semshare_hash_workspace_size,
     semshare_match,
     semshare_match_static,
+    semshare_match_tc,
+    semshare_match_tc_workspace_size,
     semshare_match_workspace_size,
     semshare_rope_table,
     status_string,

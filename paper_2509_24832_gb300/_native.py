@@ -62,6 +62,10 @@ def load():
         lib.semshare_match_workspace_size.restype = ctypes.c_size_t
         lib.semshare_match.argtypes = [P, i64, P, i64, i32, P, P, P, ctypes.c_size_t, P]
         lib.semshare_match.restype = ctypes.c_int
+        lib.semshare_match_tc_workspace_size.argtypes = [i64, i64, i32]
+        lib.semshare_match_tc_workspace_size.restype = ctypes.c_size_t
+        lib.semshare_match_tc.argtypes = [P, i64, P, i64, i32, P, P, P, ctypes.c_size_t, P, P]
+        lib.semshare_match_tc.restype = ctypes.c_int
         lib.semshare_match_static.argtypes = [P, i64, P, i64, i32, P, P, P]
         lib.semshare_match_static.restype = ctypes.c_int
         lib.semshare_gather_kv.argtypes = [P, P, P, i32, KVLayout, P, i64, i32, P, P, KVLayout, P, P]
@@ -215,6 +219,38 @@ def semshare_match(tgt_codes: torch.Tensor, ref_codes: torch.Tensor, idx: torch.
     st = load().semshare_match(_ptr(tgt_codes), n_tgt, _ptr(ref_codes), n_ref, nbits, _ptr(idx), _ptr(dist),
                                _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream))
     _check(st, "semshare_match")
+    return idx, dist
+
+
+def semshare_match_tc_workspace_size(n_tgt: int, n_ref: int, nbits: int) -> int:
+    return int(load().semshare_match_tc_workspace_size(int(n_tgt), int(n_ref), int(nbits)))
+
+
+def semshare_match_tc(tgt_codes: torch.Tensor, ref_codes: torch.Tensor, idx: torch.Tensor | None = None,
+                      dist: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
+                      err_flag: torch.Tensor | None = None, nbits: int | None = None, stream=None):
+    """semshare_match computed on the tensor cores (same result).  Returns (idx, dist)."""
+    _need_cuda(tgt_codes, "tgt_codes")
+    _need_cuda(ref_codes, "ref_codes")
+    if not tgt_codes.is_contiguous() or not ref_codes.is_contiguous():
+        raise ValueError("codes must be contiguous")
+    n_tgt, w = tgt_codes.shape
+    n_ref = ref_codes.shape[0]
+    if ref_codes.shape[1] != w:
+        raise ValueError("code widths differ")
+    nbits = 32 * w if nbits is None else nbits
+    dev = tgt_codes.device
+    if idx is None:
+        idx = torch.empty(n_tgt, dtype=torch.int32, device=dev)
+    if dist is None:
+        dist = torch.empty(n_tgt, dtype=torch.int32, device=dev)
+    if workspace is None:
+        workspace = torch.empty(max(256, semshare_match_tc_workspace_size(n_tgt, n_ref, nbits)), dtype=torch.uint8,
+                                device=dev)
+    st = load().semshare_match_tc(_ptr(tgt_codes), n_tgt, _ptr(ref_codes), n_ref, nbits, _ptr(idx), _ptr(dist),
+                                  _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(err_flag),
+                                  _stream(stream))
+    _check(st, "semshare_match_tc")
     return idx, dist
 
 

@@ -38,6 +38,7 @@
 
 #include "common.cuh"
 #include "ptx.cuh"
+#include "tma_host.cuh"
 
 namespace semshare {
 namespace {
@@ -620,32 +621,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;  // resolved once per process
-    if (fn == nullptr) {
-        void* p = nullptr;
-        cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-    }
-    return fn;
-}
-
-bool encode_2d(CUtensorMap* map, CUtensorMapDataType type, const void* base, uint64_t inner, uint64_t outer,
-               uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
-    PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
-    if (enc == nullptr) return false;
-    const cuuint64_t dims[2] = {inner, outer};
-    const cuuint64_t strides[1] = {row_bytes};
-    const cuuint32_t box[2] = {box_inner, box_outer};
-    const cuuint32_t estr[2] = {1, 1};
-    return enc(map, type, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-               CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 // Grid and workspace of one call: one CTA per SM (fewer if there are fewer iterations), a
 // 256-byte-aligned array of per-tile counters, then two partial-accumulator slots per CTA.
 struct HashPlan {
@@ -739,11 +714,11 @@ extern "C" semshare_status semshare_hash(const void* emb, semshare_dtype dtype, 
     const size_t smem = fixed + static_cast<size_t>(stages) * a.stage_bytes;
 
     CUtensorMap tm_emb, tm_hyp;
-    if (!encode_2d(&tm_emb, a.is_f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, emb,
+    if (!encode_tma_2d(&tm_emb, a.is_f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, emb,
                    static_cast<uint64_t>(d), static_cast<uint64_t>(n), static_cast<uint64_t>(row_stride * esize),
                    a.is_f32 ? 32u : 64u, kBM))
         return SEMSHARE_ECUDA;
-    if (!encode_2d(&tm_hyp, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, hyperplanes, static_cast<uint64_t>(d),
+    if (!encode_tma_2d(&tm_hyp, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, hyperplanes, static_cast<uint64_t>(d),
                    static_cast<uint64_t>(nbits), static_cast<uint64_t>(d) * 2, 64u, static_cast<uint32_t>(nbits)))
         return SEMSHARE_ECUDA;
 

@@ -25,7 +25,7 @@ import paper_2509_24832_gb300 as ss  # noqa: E402
 
 def main(argv=None):
     p = argparse.ArgumentParser()
-    p.add_argument("--kernel", choices=["hash", "match", "gather"], required=True)
+    p.add_argument("--kernel", choices=["hash", "match", "match_tc", "gather"], required=True)
     p.add_argument("--workload", default="llama8b-5k", choices=sorted(workloads.WORKLOADS))
     p.add_argument("--reps", type=int, default=3)
     a = p.parse_args(argv)
@@ -48,6 +48,9 @@ def main(argv=None):
         if a.kernel == "match":
             for _ in range(a.reps):
                 ss.semshare_match(tc, rc, idx=idx, dist=dist)
+        elif a.kernel == "match_tc":
+            for _ in range(a.reps):
+                ss.semshare_match_tc(tc, rc, idx=idx, dist=dist, err_flag=flag)
         else:
             del e
             segs = [workloads.kv_cache_device(wl, dev, segment=s) for s in range(wl.n_seg)]

@@ -168,6 +168,43 @@ def test_match_parity(ss, orc, nbits, n_tgt, n_ref):
     np.testing.assert_array_equal(dist.cpu().numpy(), od)
 
 
+@pytest.mark.parametrize("nbits", [32, 64, 96, 128, 160, 256])
+@pytest.mark.parametrize("n_tgt,n_ref", [(1, 1), (513, 255), (3000, 1000), (700, 5000), (129, 257)])
+def test_match_tc_parity(ss, orc, nbits, n_tgt, n_ref):
+    g = np.random.default_rng(nbits * 11 + n_ref)
+    ref = workloads.random_codes(n_ref, nbits, seed=nbits + n_ref, stream=3)
+    tgt = workloads.random_codes(n_tgt, nbits, seed=nbits + n_tgt, stream=4)
+    k = n_tgt // 3
+    if k:
+        tgt[:k] = ref[g.integers(0, n_ref, size=k)]
+        tgt[:k, 0] ^= np.uint32(1) << np.uint32(g.integers(0, 32))
+    if n_ref > 4:
+        ref[n_ref - 1] = ref[2]
+    ti = torch.from_numpy(tgt.view(np.int32)).cuda()
+    ri = torch.from_numpy(ref.view(np.int32)).cuda()
+    flag = ss.new_err_flag()
+    idx, dist = ss.semshare_match_tc(ti, ri, err_flag=flag)
+    pi, pd = ss.semshare_match(ti, ri)
+    torch.cuda.synchronize()
+    ss.check_flag(flag, "match_tc")
+    oi, od = orc.match(tgt, ref)
+    np.testing.assert_array_equal(idx.cpu().numpy(), oi)
+    np.testing.assert_array_equal(dist.cpu().numpy(), od)
+    assert torch.equal(idx, pi) and torch.equal(dist, pd)
+
+
+def test_match_tc_ties_and_all_equal(ss):
+    c = torch.randint(-2 ** 31, 2 ** 31 - 1, (3000, 8), dtype=torch.int32, device="cuda")
+    c[2999] = c[7]
+    idx, dist = ss.semshare_match_tc(c, c)
+    want = torch.arange(3000, dtype=torch.int32, device="cuda")
+    want[2999] = 7
+    assert torch.equal(idx, want) and int(dist.max()) == 0
+    same = torch.full((600, 8), 5, dtype=torch.int32, device="cuda")
+    idx2, d2 = ss.semshare_match_tc(c[:100].contiguous(), same)
+    assert int(idx2.max()) == 0
+
+
 def test_match_identity_ties_and_determinism(ss):
     c = torch.randint(-2 ** 31, 2 ** 31 - 1, (4000, 8), dtype=torch.int32, device="cuda")
     c[3999] = c[5]

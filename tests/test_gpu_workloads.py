@@ -47,7 +47,10 @@ def _run_path(ss, wl, emb, pos, want_proj):
     proj = torch.empty((n_rows, wl.nbits), dtype=torch.float32, device=dev) if want_proj else None
     flag = ss.new_err_flag(dev)
     codes = ss.semshare_hash(e, table, R, p, proj_out=proj, err_flag=flag)
-    idx, dist = ss.semshare_match(codes[wl.n_ref:], codes[: wl.n_ref])
+    idx, dist = ss.semshare_match_tc(codes[wl.n_ref:], codes[: wl.n_ref], err_flag=flag)
+    pidx, pdist = ss.semshare_match(codes[wl.n_ref:], codes[: wl.n_ref])
+    torch.cuda.synchronize()
+    assert torch.equal(idx, pidx) and torch.equal(dist, pdist), "tensor-core and popc matchers disagree"
     segs = [workloads.kv_cache_device(wl, dev, segment=s) for s in range(wl.n_seg)]
     out_k, out_v = ss.semshare_gather_kv([s[0] for s in segs], [s[1] for s in segs],
                                          idx.view(wl.n_batch, wl.n_tgt), err_flag=flag)
