@@ -44,8 +44,9 @@ LAUNCHES_PER_STEP = 5  # hash 1, match 3 (tc: expand + key reset, search, split;
 # valid only while the kernel source has the recorded sha256 prefix.
 NCU_TRAFFIC = {
     "gather": {"file": "gather.cu", "sha": "e03583daf19419cb", "bytes_per_launch": 1092.8e6, "targets": 5120},
-    "hash": {"file": "hash.cu", "sha": "6325d4225151e316", "bytes_per_launch": 88.96e6, "targets": 5120},
-    "match": {"file": "match.cu", "sha": "4d2ee4d85f0ed0fc", "bytes_per_launch": 0.3845e6, "targets": 5120},
+    "hash": {"file": "hash.cu", "sha": "7cf51b07f7d5874d", "bytes_per_launch": 92.63e6, "targets": 5120},
+    "match": {"file": "match.cu", "sha": "69ac4b7ce5b193e4", "bytes_per_launch": 0.3845e6, "targets": 5120},
+    "match_tc": {"file": "match_tc.cu", "sha": "3bcc238fb9cfe314", "bytes_per_launch": 2.712e6, "targets": 5120},
 }
 
 
@@ -347,7 +348,7 @@ def run_gpu_arm(args, rank, world, local_rank):
     else:
         roof = {"kernel": "hamming_tc_kernel", "bound": "tensor", "achieved": stages["match"]["tflops_fp8"],
                 "peak": 2.0 * peaks["bf16_tflops"], "unit": "TFLOP/s"}
-        tr = None
+        tr = NCU_TRAFFIC.get("match_tc")
     roof["frac"] = roof["achieved"] / roof["peak"]
     roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"
     if tr and tr.get("sha") == kernel_sha(tr["file"]):
