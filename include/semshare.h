@@ -25,6 +25,10 @@
  *   - Errors found by a kernel while it runs are OR-ed into an optional device word
  *     `err_flag` (SEMSHARE_FLAG_*); the caller reads it after synchronising and may turn it
  *     into a status with semshare_flag_status().  Kernels never trap.
+ *   - Every wait inside a pipelined kernel is bounded (2 s by default; the environment
+ *     variable SEMSHARE_WAIT_LIMIT_NS, read at each call, overrides it for diagnostics).  A
+ *     wait that runs out raises SEMSHARE_FLAG_TIMEOUT; the kernel then lets its copies in
+ *     flight land, frees its tensor memory and returns, and the CUDA context stays usable.
  *   - Results are deterministic: the same inputs give the same bits on every run.
  */
 #ifndef SEMSHARE_H

@@ -4,6 +4,7 @@
 #include <cuda_runtime.h>
 
 #include <cstdint>
+#include <cstdlib>
 
 #include "semshare.h"
 
@@ -30,5 +31,17 @@ inline semshare_status launch_status() {
 
 // Limit of every bounded pipeline wait inside a kernel (the host never sees a longer stall).
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
+
+// The pipeline-wait limit of one call: kWaitLimitNs, or the nanoseconds in the environment
+// variable SEMSHARE_WAIT_LIMIT_NS (a diagnostic knob, read at every call; tests use a tiny
+// value to drive the timeout path).  The waits that let copies in flight land before a CTA
+// exits always keep kWaitLimitNs.
+inline uint64_t wait_limit_ns() {
+    const char* e = getenv("SEMSHARE_WAIT_LIMIT_NS");
+    if (e == nullptr || *e == 0) return kWaitLimitNs;
+    char* end = nullptr;
+    const unsigned long long v = strtoull(e, &end, 10);
+    return (end != e && v > 0) ? static_cast<uint64_t>(v) : kWaitLimitNs;
+}
 
 }  // namespace semshare

@@ -710,7 +710,7 @@ extern "C" semshare_status semshare_hash(const void* emb, semshare_dtype dtype, 
     a.err_flag = err_flag;
     a.tile_count = static_cast<uint32_t*>(workspace);
     a.partials = reinterpret_cast<float4*>(static_cast<uint8_t*>(workspace) + plan.count_bytes);
-    a.wait_limit_ns = kWaitLimitNs;
+    a.wait_limit_ns = wait_limit_ns();
     const size_t smem = fixed + static_cast<size_t>(stages) * a.stage_bytes;
 
     CUtensorMap tm_emb, tm_hyp;

@@ -368,7 +368,7 @@ extern "C" semshare_status semshare_match_tc(const uint32_t* tgt_codes, int64_t 
     a.b_bytes = static_cast<uint32_t>(kTN * plan.kpad);
     a.keys = keys;
     a.err_flag = err_flag;
-    a.wait_limit_ns = kWaitLimitNs;
+    a.wait_limit_ns = wait_limit_ns();
     const size_t smem = kFixedSmem + 2 * static_cast<size_t>(a.a_bytes) + 2 * static_cast<size_t>(a.b_bytes);
     if (smem > static_cast<size_t>(smem_optin)) return SEMSHARE_EUNSUPPORTED;
 

@@ -69,16 +69,14 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
                                                   uint32_t* err, uint32_t timeout_bit, uint64_t limit_ns) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = global_timer_ns();
-    for (uint32_t i = 1;; ++i) {
-        if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
-        if ((i & 3u) == 0u) {
-            if (*abort_flag) return false;
-            if (global_timer_ns() - t0 > limit_ns) {
-                *abort_flag = 1;
-                if (err) atomicOr(err, timeout_bit);
-                return false;
-            }
+    for (;;) {
+        if (*abort_flag) return false;
+        if (global_timer_ns() - t0 > limit_ns) {
+            *abort_flag = 1;
+            if (err) atomicOr(err, timeout_bit);
+            return false;
         }
+        if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
     }
 }
 

@@ -301,3 +301,45 @@ def test_gather_preserves_special_bit_patterns(ss):
     ok, ov = ss.semshare_gather_kv(k, v, idx)
     assert torch.equal(ok[0].view(torch.int16), k.flip(2).view(torch.int16))
     assert torch.equal(ov[0].view(torch.int16), v.flip(2).view(torch.int16))
+
+
+# ---- failure detection: a pipeline wait that runs out ----------------------------------------
+
+def test_wait_timeout_reports_status_and_context_survives(ss, orc, monkeypatch):
+    # a 1 ns wait limit makes the pipelined kernels' waits run out: they must report
+    # SEMSHARE_ETIMEOUT through the error word, return without trapping, and leave the CUDA
+    # context usable (the next calls, with the default limit, give correct results)
+    wl = workloads.WORKLOADS["llama8b-1k"]
+    emb, pos, _ = workloads.prompt_rows(wl)
+    e = emb_dev(emb)
+    p = torch.from_numpy(pos).cuda()
+    R = bf16_dev(workloads.hyperplanes(wl))
+    table = ss.semshare_rope_table(wl.d)
+    ws = torch.zeros(ss.semshare_hash_workspace_size(len(emb), wl.d, wl.nbits) + 256, dtype=torch.uint8,
+                     device="cuda")
+    codes = torch.empty((len(emb), wl.nbits // 32), dtype=torch.int32, device="cuda")
+    monkeypatch.setenv("SEMSHARE_WAIT_LIMIT_NS", "1")
+    flag = ss.new_err_flag()
+    ss.semshare_hash(e, table, R, p, codes=codes, workspace=ws, err_flag=flag)
+    torch.cuda.synchronize()
+    assert ss.flag_status(flag) == 5  # SEMSHARE_ETIMEOUT
+    tgt, ref = codes[wl.n_ref:], codes[: wl.n_ref]
+    flag2 = ss.new_err_flag()
+    ss.semshare_match_tc(tgt, ref, err_flag=flag2)
+    torch.cuda.synchronize()
+    assert ss.flag_status(flag2) == 5
+    monkeypatch.delenv("SEMSHARE_WAIT_LIMIT_NS")
+    # the context is intact: rerun with the default limit (the timed-out hash may have left
+    # its workspace dirty, so it is zeroed first) and compare with the oracle
+    ws.zero_()
+    flag3 = ss.new_err_flag()
+    proj = torch.empty((len(emb), wl.nbits), dtype=torch.float32, device="cuda")
+    codes = ss.semshare_hash(e, table, R, p, codes=codes, proj_out=proj, workspace=ws, err_flag=flag3)
+    idx, dist = ss.semshare_match_tc(codes[wl.n_ref:], codes[: wl.n_ref], err_flag=flag3)
+    torch.cuda.synchronize()
+    ss.check_flag(flag3, "after timeout")
+    oc, op = orc.hash_codes(emb, pos, workloads.hyperplanes(wl))
+    check_hash(codes_host(codes), proj.cpu().numpy(), oc, op)
+    gc = codes_host(codes)
+    oi, od = orc.match(gc[wl.n_ref:], gc[: wl.n_ref])
+    np.testing.assert_array_equal(idx.cpu().numpy(), oi)
