@@ -10,6 +10,8 @@ it follows, is stated in `semshare_oracle.c`:
   hash    random-hyperplane sign codes of the rotated rows; Sec. 3.3, App. A.2
   match   Hamming 1-nearest reference token, ties to the lowest index; Sec. 3.3
   gather  reordered K/V rows, bitwise copies; Sec. 3.3, Sec. 3.3.2
+  retrieve  LSH-distance similarity of whole prompts and the best candidate; Sec. 3.2,
+          App. A.3, Sec. 4.4
 
 Parity pins: every function here is pinned by `tests/test_oracle_*.py` against closed forms,
 invariants, hand-derived golden cases and brute force (none is "parity unpinned").
@@ -65,6 +67,7 @@ def _load():
         lib.oracle_match.argtypes = [P, i64, P, i64, i32, P, P]
         lib.oracle_gather_kv.argtypes = [P, P, P, i32, i32, i32, i64, P, i64, i32, P, P]
         lib.oracle_gather_kv.restype = i64
+        lib.oracle_retrieve.argtypes = [P, i64, P, P, i32, i32, f64, f64, P, P, P, P]
         _lib = lib
         return lib
 
@@ -178,3 +181,24 @@ def gather_kv(seg_k, seg_v, idx: np.ndarray, out_k: np.ndarray | None = None, ou
     bad = _load().oracle_gather_kv(pk, pv, _ptr(offs), len(seg_k), L, H, hd * dt.itemsize, _ptr(idx2), n_tgt, B,
                                    _ptr(out_k), _ptr(out_v))
     return out_k, out_v, int(bad)
+
+
+def retrieve(tgt_codes: np.ndarray, pool_codes: np.ndarray, seg_offsets, nbits: int | None = None,
+             dmax: float = 30.0, threshold: float = 0.8):
+    """Reference retrieval by LSH-distance similarity (Sec. 3.2, App. A.3, Sec. 4.4).
+
+    pool_codes: the candidate prompts' codes concatenated; candidate s is rows
+    seg_offsets[s]..seg_offsets[s+1].  Returns (mean_dist [n_seg] float64, similarity [n_seg]
+    float64, best, applies)."""
+    t = np.ascontiguousarray(tgt_codes, dtype=np.uint32)
+    p = np.ascontiguousarray(pool_codes, dtype=np.uint32)
+    offs = np.ascontiguousarray(np.asarray(seg_offsets, dtype=np.int64))
+    n_seg = len(offs) - 1
+    nbits = 32 * t.shape[1] if nbits is None else nbits
+    mean = np.zeros(n_seg)
+    sim = np.zeros(n_seg)
+    best = np.zeros(1, dtype=np.int32)
+    applies = np.zeros(1, dtype=np.int32)
+    _load().oracle_retrieve(_ptr(t), t.shape[0], _ptr(p), _ptr(offs), n_seg, nbits, float(dmax), float(threshold),
+                            _ptr(mean), _ptr(sim), _ptr(best), _ptr(applies))
+    return mean, sim, int(best[0]), bool(applies[0])

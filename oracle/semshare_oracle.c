@@ -25,6 +25,10 @@
  *              reference cache (Sec. 3.3): out[b][l][h][t] = ref[l][h][idx[b][t]] for every
  *              layer l and KV head h, copied bit for bit (Sec. 3.3.2: KV is stored after RoPE,
  *              so nothing is re-encoded).
+ *   5. retrieve  Reference retrieval (Sec. 3.2, App. A.3, Sec. 4.4): each stored candidate
+ *              prompt's LSH distance to the target -- read as the mean over target tokens of the
+ *              nearest Hamming distance -- is normalised by 30 and turned into a similarity in
+ *              [0, 1]; the most similar candidate wins and is reused if above 0.8.
  *
  * Build: gcc -O2 -fopenmp -ffp-contract=off -shared -fPIC (no fused multiply-add, so x86 and
  * Arm hosts produce the same bits).
@@ -202,4 +206,42 @@ int64_t oracle_gather_kv(const uint8_t* const* seg_k, const uint8_t* const* seg_
                     memcpy(out_v + dst_row * row_bytes, seg_v[s] + src_row * row_bytes, (size_t)row_bytes);
                 }
     return bad;
+}
+
+/* ---- reference retrieval: LSH-distance similarity of whole prompts ------------------------ */
+
+/* Reference retrieval (Sec. 3.2: the stored prompt with the highest LSH-distance-based
+ * similarity to the target is retrieved; App. A.3: Similarity = clip(1 - (LSH_dist - 0)/(30 - 0),
+ * 0, 1); Sec. 4.4: reuse applies when the similarity is above 0.8).  LSH_dist of a candidate
+ * prompt is read here as the mean over the target tokens of each token's Hamming distance to
+ * its nearest token of the candidate.  The pool is one code array; candidate s holds rows
+ * seg_offsets[s] <= j < seg_offsets[s+1] (each non-empty).
+ * Outputs: mean_dist[s], similarity[s] (n_seg doubles), *best = the lowest s of greatest
+ * similarity, *applies = similarity[*best] > threshold. */
+void oracle_retrieve(const uint32_t* tgt, int64_t n_tgt, const uint32_t* pool, const int64_t* seg_offsets,
+                     int32_t n_seg, int32_t nbits, double dmax, double threshold, double* mean_dist,
+                     double* similarity, int32_t* best, int32_t* applies) {
+    const int32_t w = nbits / 32;
+    for (int32_t s = 0; s < n_seg; ++s) {
+        int64_t sum = 0;
+#pragma omp parallel for reduction(+ : sum) schedule(dynamic, 64)
+        for (int64_t t = 0; t < n_tgt; ++t) {
+            int32_t m = nbits + 1;
+            for (int64_t j = seg_offsets[s]; j < seg_offsets[s + 1]; ++j) {
+                const int32_t h = oracle_hamming(tgt + t * w, pool + j * w, w);
+                if (h < m) m = h;
+            }
+            sum += m;
+        }
+        mean_dist[s] = (double)sum / (double)n_tgt;
+        double sim = 1.0 - mean_dist[s] / dmax;
+        if (sim < 0.0) sim = 0.0;
+        if (sim > 1.0) sim = 1.0;
+        similarity[s] = sim;
+    }
+    int32_t b = 0;
+    for (int32_t s = 1; s < n_seg; ++s)
+        if (similarity[s] > similarity[b]) b = s;
+    *best = b;
+    *applies = similarity[b] > threshold ? 1 : 0;
 }
