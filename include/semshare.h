@@ -114,9 +114,10 @@ semshare_status semshare_rope_table(int32_t d, double rope_base, uint64_t* table
  *   proj_out    device or NULL; if given, [n][nbits] float32 projections p_j are written too
  *   workspace   device scratch of at least semshare_hash_workspace_size(n, d, nbits) bytes,
  *               256-byte aligned.  It must be zero-filled before its first use; every call
- *               that completes without an error flag leaves it zero-filled again, so one
- *               workspace serves any number of calls made one after another.  Calls that may
- *               run concurrently need separate workspaces.
+ *               that completes without an error flag leaves the part that must be zero
+ *               zero-filled again, so one workspace (sized for the largest call) serves any
+ *               number of calls of any sizes made one after another on the same device.
+ *               Calls that may run concurrently need separate workspaces.
  *   err_flag    device or NULL; SEMSHARE_FLAG_TIMEOUT is OR-ed in if a pipeline wait of the
  *               kernel exceeds its limit (the kernel then stops, leaves codes incomplete and
  *               the workspace in an unknown state: zero it before the next call)

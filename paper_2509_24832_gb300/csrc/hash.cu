@@ -621,24 +621,30 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-// Grid and workspace of one call: one CTA per SM (fewer if there are fewer iterations), a
-// 256-byte-aligned array of per-tile counters, then two partial-accumulator slots per CTA.
+// Grid and workspace of one call: one CTA per SM (fewer if there are fewer iterations).
+// Workspace layout: the partial-accumulator slots (two per CTA) first, in a region sized for
+// the largest call on this device (one CTA per SM, 256-bit codes), then the per-tile counters.
+// The counters therefore start at the same offset for every call on a device and never overlap
+// the slots of any other call: the counters are the only part that must be zero on entry, the
+// slots are written before they are read, and calls of different sizes can share a workspace.
 struct HashPlan {
     int64_t n_tiles;
     int64_t total_iters;
     int grid;
+    size_t partial_bytes;  // the slot region (fixed per device)
     size_t count_bytes;
-    size_t partial_bytes;
 };
 
-semshare_status plan_hash(int64_t n, int32_t d, int32_t nbits, HashPlan* p) {
+constexpr int kMaxBits = 256;
+
+semshare_status plan_hash(int64_t n, int32_t d, HashPlan* p) {
     int sms = 0;
     if (current_sm_count(&sms, nullptr) != SEMSHARE_OK) return SEMSHARE_ECUDA;
     p->n_tiles = (n + kBM - 1) / kBM;
     p->total_iters = p->n_tiles * (d / kBK);
     p->grid = static_cast<int>(p->total_iters < sms ? p->total_iters : sms);
+    p->partial_bytes = static_cast<size_t>(2) * sms * kBM * static_cast<size_t>(kMaxBits) * 4;
     p->count_bytes = ((static_cast<size_t>(p->n_tiles) * 4 + 255) / 256) * 256;
-    p->partial_bytes = static_cast<size_t>(2) * p->grid * kBM * static_cast<size_t>(nbits) * 4;
     return SEMSHARE_OK;
 }
 
@@ -649,8 +655,8 @@ extern "C" size_t semshare_hash_workspace_size(int64_t n, int32_t d, int32_t nbi
     using namespace semshare;
     if (n <= 0 || d < kBK || d % kBK != 0 || nbits < 32 || nbits > 256 || nbits % 32 != 0) return 0;
     HashPlan p;
-    if (plan_hash(n, d, nbits, &p) != SEMSHARE_OK) return 0;
-    return p.count_bytes + p.partial_bytes;
+    if (plan_hash(n, d, &p) != SEMSHARE_OK) return 0;
+    return p.partial_bytes + p.count_bytes;
 }
 
 extern "C" semshare_status semshare_hash(const void* emb, semshare_dtype dtype, int64_t n, int32_t d,
@@ -676,8 +682,8 @@ extern "C" semshare_status semshare_hash(const void* emb, semshare_dtype dtype, 
         return SEMSHARE_EINVAL;
 
     HashPlan plan;
-    if (plan_hash(n, d, nbits, &plan) != SEMSHARE_OK) return SEMSHARE_ECUDA;
-    if (workspace_bytes < plan.count_bytes + plan.partial_bytes) return SEMSHARE_EINVAL;
+    if (plan_hash(n, d, &plan) != SEMSHARE_OK) return SEMSHARE_ECUDA;
+    if (workspace_bytes < plan.partial_bytes + plan.count_bytes) return SEMSHARE_EINVAL;
     int dev = 0, smem_optin = 0;
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
@@ -708,8 +714,8 @@ extern "C" semshare_status semshare_hash(const void* emb, semshare_dtype dtype, 
     a.codes = codes;
     a.proj = proj_out;
     a.err_flag = err_flag;
-    a.tile_count = static_cast<uint32_t*>(workspace);
-    a.partials = reinterpret_cast<float4*>(static_cast<uint8_t*>(workspace) + plan.count_bytes);
+    a.partials = static_cast<float4*>(workspace);
+    a.tile_count = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(workspace) + plan.partial_bytes);
     a.wait_limit_ns = wait_limit_ns();
     const size_t smem = fixed + static_cast<size_t>(stages) * a.stage_bytes;
 

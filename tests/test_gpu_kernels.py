@@ -132,10 +132,28 @@ def test_hash_empty_and_repeatable(ss):
     a = ss.semshare_hash(x, table, R)
     b = ss.semshare_hash(x, table, R)
     assert torch.equal(a, b)
-    # the shared-tile counters are back at zero after every call
-    ws = ss.hash_workspace(300, 128, 64)
-    torch.cuda.synchronize()
-    assert int(ws[: 256].count_nonzero()) == 0
+
+
+def test_hash_workspace_shared_across_sizes(ss):
+    """One workspace serves calls of different sizes one after another: each call's codes and
+    projections equal those of the same call on a fresh zero-filled workspace (the per-tile
+    counters never land on an earlier call's partial sums)."""
+    g = torch.Generator(device="cuda").manual_seed(3)
+    cases = [(256, 512, 64), (10240, 4096, 256), (300, 4096, 256), (5000, 1024, 128), (70000, 128, 32),
+             (1000, 4096, 96), (129, 64, 256)]
+    big = max(ss.semshare_hash_workspace_size(n, d, nb) for n, d, nb in cases)
+    shared = torch.zeros(big, dtype=torch.uint8, device="cuda")
+    for n, d, nb in cases:
+        x = torch.randn((n, d), generator=g, device="cuda").to(torch.bfloat16)
+        R = torch.randn((nb, d), generator=g, device="cuda").to(torch.bfloat16)
+        table = ss.semshare_rope_table(d)
+        p1 = torch.empty((n, nb), dtype=torch.float32, device="cuda")
+        p2 = torch.empty_like(p1)
+        fresh = torch.zeros(ss.semshare_hash_workspace_size(n, d, nb), dtype=torch.uint8, device="cuda")
+        a = ss.semshare_hash(x, table, R, proj_out=p1, workspace=shared)
+        b = ss.semshare_hash(x, table, R, proj_out=p2, workspace=fresh)
+        torch.cuda.synchronize()
+        assert torch.equal(a, b) and torch.equal(p1, p2), (n, d, nb)
 
 
 def test_hash_stream_k_split_tiles_are_deterministic(ss, orc):
