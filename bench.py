@@ -8,6 +8,12 @@ One step = the whole path over one synthetic matching problem resident in HBM:
   semshare_gather_kv reference K/V rows rearranged into the target's order, all layers/heads
 value = target tokens of all ranks / max over ranks of the mean device time of a step.
 
+`--workload retrieve-16x4096` times the path with reference retrieval in front (Sec. 3.2):
+16 stored prompts whose codes were computed when they were stored; per step the target is
+hashed without rotary encoding, the most similar stored prompt is retrieved
+(semshare_retrieve), the target is hashed with it, matched against the winner's codes and the
+winner's K/V cache is gathered.
+
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl gb300|reference]
 
 With N > 1 it runs under torch.distributed.run, one rank per GPU; every rank solves its own
@@ -35,10 +41,11 @@ if ROOT not in sys.path:
 import workloads  # noqa: E402
 
 METRIC = "target tokens matched+gathered/sec at 5k tokens"
+METRIC_RETRIEVE = "target tokens retrieved+matched+gathered/sec"
 DEFAULT_WORKLOAD = "llama8b-5k"
+ALL_WORKLOADS = {**workloads.WORKLOADS, **workloads.RETRIEVAL_WORKLOADS}
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 L2_FLUSH_BYTES = 256 << 20
-LAUNCHES_PER_STEP = 5  # hash 1, match 3 (tc: expand + key reset, search, split; popc: key init, search, split), gather 1
 
 # DRAM bytes per launch from ncu captures (dram__bytes_read.sum + dram__bytes_write.sum),
 # valid only while the kernel source has the recorded sha256 prefix.
@@ -55,7 +62,7 @@ def parse_args(argv=None):
     p.add_argument("--gpus", type=int, default=1)
     p.add_argument("--steps", type=int, default=1000)
     p.add_argument("--warmup", type=int, default=20)
-    p.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads.WORKLOADS))
+    p.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(ALL_WORKLOADS))
     p.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     p.add_argument("--matcher", default="tc", choices=["tc", "popc"],
                    help="Hamming search: tensor-core GEMM (semshare_match_tc) or xor/popc (semshare_match)")
@@ -96,6 +103,8 @@ def barrier(device=None):
 # ---- algorithmic work per step (roofline numerators) -----------------------------------------
 
 def work(wl: workloads.Workload) -> dict:
+    if wl.recipe == "retrieve":
+        return work_retrieve(wl)
     rows = wl.n_ref + wl.n_batch * wl.n_tgt
     esz = 4 if wl.emb_dtype == "f32" else 2
     L, H, hd = wl.kv
@@ -108,6 +117,25 @@ def work(wl: workloads.Workload) -> dict:
         "gather_bytes": 2.0 * 2.0 * n_t * L * H * hd * 2,  # K and V, read + write
         "targets": n_t,
         "rows": rows,
+    }
+
+
+def work_retrieve(wl: workloads.Workload) -> dict:
+    """Retrieval step: two hashes of the target rows (plain and rotary), the retrieval GEMM over
+    the whole pool, the match against one member, the gather of one member's rows."""
+    n_t = wl.n_tgt
+    esz = 4 if wl.emb_dtype == "f32" else 2
+    L, H, hd = wl.kv
+    kpad = ((wl.nbits + 127) // 128) * 128
+    return {
+        "hash_flops": 2.0 * n_t * wl.d * wl.nbits,
+        "hash_bytes": n_t * wl.d * esz + n_t * wl.nbits / 8 + n_t * 4 + wl.nbits * wl.d * 2,
+        "retrieve_flops": 2.0 * n_t * wl.n_ref * kpad,
+        "match_wordops": float(n_t) * wl.seg_len * (wl.nbits // 32),
+        "match_flops": 2.0 * n_t * wl.seg_len * kpad,
+        "gather_bytes": 2.0 * 2.0 * n_t * L * H * hd * 2,
+        "targets": n_t,
+        "rows": n_t,
     }
 
 
@@ -194,6 +222,10 @@ class ClockSampler:
 class Problem:
     """Device buffers of one matching problem and the three library calls of a step."""
 
+    STAGES = ("hash", "match", "gather")
+    # hash 1, match 3 (tc: expand + key reset, search, split; popc: key init, search, split), gather 1
+    LAUNCHES_PER_STEP = 5
+
     def __init__(self, wl: workloads.Workload, device, seed: int, matcher: str = "tc"):
         import torch
 
@@ -259,6 +291,227 @@ class Problem:
         if ev:
             ev[3].record()
 
+    def e2e_plan(self):
+        """(one, h2d, d2h, read): a step through the public API with host buffers -- the
+        embedding rows, positions and reference K/V cache copied in from pinned host memory,
+        the match result (idx, dist) copied back."""
+        import torch
+
+        h_emb = self.emb.cpu().pin_memory()
+        h_pos = self.pos.cpu().pin_memory()
+        h_k = [t.cpu().pin_memory() for t in self.ref_k]
+        h_v = [t.cpu().pin_memory() for t in self.ref_v]
+        h_idx = torch.empty_like(self.idx, device="cpu").pin_memory()
+        h_dist = torch.empty_like(self.dist, device="cpu").pin_memory()
+        h2d = h_emb.numel() * h_emb.element_size() + h_pos.numel() * 4 + \
+            sum(t.numel() * t.element_size() for t in h_k + h_v)
+        d2h = (h_idx.numel() + h_dist.numel()) * 4
+
+        def one():
+            self.emb.copy_(h_emb, non_blocking=True)
+            self.pos.copy_(h_pos, non_blocking=True)
+            for d, h in zip(self.ref_k + self.ref_v, h_k + h_v):
+                d.copy_(h, non_blocking=True)
+            self.step()
+            h_idx.copy_(self.idx, non_blocking=True)
+            h_dist.copy_(self.dist, non_blocking=True)
+
+        return one, h2d, d2h, lambda: int(h_idx[0])
+
+
+class RetrieveProblem:
+    """Reference retrieval in front of the path (Sec. 3.2).  The stored prompts' codes -- plain
+    for retrieval, rotary-encoded for matching -- are computed once when they are stored; a step
+    handles one new target prompt:
+      hash_plain  codes of the target rows without rotary encoding (retrieval precedes it)
+      retrieve    similarity to every stored prompt, the best one (semshare_retrieve)
+      hash        codes of the target rows with rotary encoding (Sec. 3.3.1)
+      match       1-NN against the winner's rotary codes (the host reads the winner first)
+      gather      the winner's K/V rows in the target's order"""
+
+    STAGES = ("hash_plain", "retrieve", "hash", "match", "gather")
+    # hash 1, retrieve 3 (expand + key reset, search, per-candidate reduction), hash 1, match 3, gather 1
+    LAUNCHES_PER_STEP = 9
+
+    def __init__(self, wl: workloads.Workload, device, seed: int, matcher: str = "tc"):
+        import torch
+
+        import paper_2509_24832_gb300 as ss
+
+        if matcher != "tc":
+            raise ValueError("the retrieval step uses the tensor-core matcher")
+        self.ss, self.wl, self.dev, self.matcher = ss, wl, device, matcher
+        emb, pos, _ = workloads.prompt_rows(wl, seed=seed)
+        self.host_emb, self.host_pos = emb, pos
+        n_pool, n_t, w = wl.n_ref, wl.n_tgt, wl.nbits // 32
+
+        def dev_rows(a):
+            return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(device).view(torch.bfloat16)
+
+        R = workloads.hyperplanes(wl, seed=seed)
+        self.hyp = torch.from_numpy(R.view(np.int16)).to(device).view(torch.bfloat16)
+        self.table = ss.semshare_rope_table(wl.d, 10000.0, device=device)
+        self.flag = ss.new_err_flag(device)
+        self.offsets = [m * wl.seg_len for m in range(wl.n_seg + 1)]
+        # store time: every stored prompt's codes, plain and rotary (its own positions)
+        pool = dev_rows(emb[:n_pool])
+        self.pool_rcodes = ss.semshare_hash(pool, self.table, self.hyp,
+                                            torch.zeros(n_pool, dtype=torch.int32, device=device))
+        self.pool_codes = ss.semshare_hash(pool, self.table, self.hyp, torch.from_numpy(pos[:n_pool]).to(device))
+        del pool
+        self.emb = dev_rows(emb[n_pool:])
+        self.pos = torch.from_numpy(pos[n_pool:]).to(device)
+        self.zeros = torch.zeros(n_t, dtype=torch.int32, device=device)
+        self.t_rcodes = torch.empty((n_t, w), dtype=torch.int32, device=device)
+        self.codes = torch.empty((n_t, w), dtype=torch.int32, device=device)
+        self.hash_ws = torch.zeros(max(256, ss.semshare_hash_workspace_size(n_t, wl.d, wl.nbits)), dtype=torch.uint8,
+                                   device=device)
+        self.ret_ws = torch.empty(ss.semshare_retrieve_workspace_size(n_t, n_pool, wl.n_seg, wl.nbits),
+                                  dtype=torch.uint8, device=device)
+        self.choice = choice = torch.zeros(2, dtype=torch.int32, device=device)  # best, applies
+        self.ret = ss.Retrieval(torch.empty(wl.n_seg, dtype=torch.float64, device=device),
+                                torch.empty(wl.n_seg, dtype=torch.float64, device=device),
+                                choice[:1], choice[1:], None, None)
+        self.h_choice = torch.zeros(2, dtype=torch.int32).pin_memory()
+        self.idx = torch.empty(n_t, dtype=torch.int32, device=device)
+        self.dist = torch.empty(n_t, dtype=torch.int32, device=device)
+        self.tc_ws = torch.empty(ss.semshare_match_tc_workspace_size(n_t, wl.seg_len, wl.nbits), dtype=torch.uint8,
+                                 device=device)
+        segs = [workloads.kv_cache_device(wl, device, seed=seed, segment=m) for m in range(wl.n_seg)]
+        self.ref_k = [m[0] for m in segs]
+        self.ref_v = [m[1] for m in segs]
+        L, H, hd = wl.kv
+        self.out_k = torch.empty((1, L, H, n_t, hd), dtype=torch.bfloat16, device=device)
+        self.out_v = torch.empty_like(self.out_k)
+        self.winner = -1
+        self.load_winner = None  # e2e: copies the winner's K/V cache in from host memory
+
+    def step(self, ev=None):
+        ss, wl = self.ss, self.wl
+        if ev:
+            ev[0].record()
+        ss.semshare_hash(self.emb, self.table, self.hyp, self.zeros, codes=self.t_rcodes, err_flag=self.flag,
+                         workspace=self.hash_ws)
+        if ev:
+            ev[1].record()
+        ss.semshare_retrieve(self.t_rcodes, self.pool_rcodes, self.offsets, workspace=self.ret_ws,
+                             err_flag=self.flag, out=self.ret)
+        self.h_choice.copy_(self.choice, non_blocking=True)  # best, applies
+        if ev:
+            ev[2].record()
+        ss.semshare_hash(self.emb, self.table, self.hyp, self.pos, codes=self.codes, err_flag=self.flag,
+                         workspace=self.hash_ws)
+        if ev:
+            ev[3].record()
+            ev[3].synchronize()
+        else:
+            import torch
+
+            torch.cuda.current_stream().synchronize()
+        m = self.winner = int(self.h_choice[0])
+        if not 0 <= m < wl.n_seg:
+            raise RuntimeError(f"retrieval returned candidate {m}")
+        ss.semshare_match_tc(self.codes, self.pool_codes[self.offsets[m]:self.offsets[m + 1]], idx=self.idx,
+                             dist=self.dist, workspace=self.tc_ws, err_flag=self.flag)
+        if self.load_winner is not None:
+            self.load_winner(m)
+        if ev:
+            ev[4].record()
+        ss.semshare_gather_kv([self.ref_k[m]], [self.ref_v[m]], self.idx.view(1, wl.n_tgt), out_k=self.out_k,
+                              out_v=self.out_v, err_flag=self.flag)
+        if ev:
+            ev[5].record()
+
+    def e2e_plan(self):
+        """(one, h2d, d2h, read): the target's embedding rows and positions copied in, the
+        retrieved prompt's K/V cache loaded from pinned host memory once the winner is known
+        (Sec. 3.2: the reference is loaded onto the GPU with its KV cache), the winner and the
+        match result (idx, dist) copied back."""
+        import torch
+
+        h_emb = self.emb.cpu().pin_memory()
+        h_pos = self.pos.cpu().pin_memory()
+        h_k = [t.cpu().pin_memory() for t in self.ref_k]
+        h_v = [t.cpu().pin_memory() for t in self.ref_v]
+        h_idx = torch.empty_like(self.idx, device="cpu").pin_memory()
+        h_dist = torch.empty_like(self.dist, device="cpu").pin_memory()
+        kv_bytes = h_k[0].numel() * h_k[0].element_size() * 2
+        h2d = h_emb.numel() * h_emb.element_size() + h_pos.numel() * 4 + kv_bytes
+        d2h = (h_idx.numel() + h_dist.numel()) * 4 + self.h_choice.numel() * 4
+
+        def load(m):
+            self.ref_k[m].copy_(h_k[m], non_blocking=True)
+            self.ref_v[m].copy_(h_v[m], non_blocking=True)
+
+        def one():
+            self.emb.copy_(h_emb, non_blocking=True)
+            self.pos.copy_(h_pos, non_blocking=True)
+            self.load_winner = load
+            try:
+                self.step()
+            finally:
+                self.load_winner = None
+            h_idx.copy_(self.idx, non_blocking=True)
+            h_dist.copy_(self.dist, non_blocking=True)
+
+        return one, h2d, d2h, lambda: int(h_idx[0])
+
+
+def make_problem(wl, device, seed, matcher):
+    cls = RetrieveProblem if wl.recipe == "retrieve" else Problem
+    return cls(wl, device, seed, matcher)
+
+
+def stage_report(wl, W, stage_ms, peaks, popc_peak, matcher):
+    """Per-stage throughput and fraction of the relevant peak."""
+    kpad = ((wl.nbits + 127) // 128) * 128
+    fp8_peak = 2.0 * peaks["bf16_tflops"]  # fp8 dense = 2 x bf16 (nominal ratio)
+    out = {}
+    for name, ms in stage_ms.items():
+        sec = ms * 1e-3
+        r = {"ms": ms}
+        if name in ("hash", "hash_plain"):
+            r["tflops"] = W["hash_flops"] / sec / 1e12
+            r["gbs"] = W["hash_bytes"] / sec / 1e9
+            r["frac_tensor"] = r["tflops"] / peaks["bf16_tflops"]
+            r["frac_hbm"] = r["gbs"] / peaks["hbm_gbs"]
+        elif name == "retrieve":
+            r["tflops_fp8"] = W["retrieve_flops"] / sec / 1e12
+            r["frac_fp8_tensor"] = r["tflops_fp8"] / fp8_peak
+        elif name == "match":
+            r["gwordops"] = W["match_wordops"] / sec / 1e9
+            r["matcher"] = matcher
+            if matcher == "popc":
+                r["frac_popc"] = r["gwordops"] * 1e9 / popc_peak
+            else:
+                fl = W.get("match_flops", 2.0 * W["targets"] * wl.n_ref * kpad)
+                r["tflops_fp8"] = fl / sec / 1e12
+                r["frac_fp8_tensor"] = r["tflops_fp8"] / fp8_peak
+        elif name == "gather":
+            r["gbs"] = W["gather_bytes"] / sec / 1e9
+            r["frac_hbm"] = r["gbs"] / peaks["hbm_gbs"]
+        out[name] = r
+    return out
+
+
+def roofline_for(dominant, stages, peaks, matcher):
+    if dominant == "gather":
+        return {"kernel": "kv_gather_kernel", "bound": "hbm", "achieved": stages["gather"]["gbs"],
+                "peak": peaks["hbm_gbs"], "unit": "GB/s"}, NCU_TRAFFIC.get("gather")
+    if dominant in ("hash", "hash_plain"):
+        return {"kernel": "lsh_hash_kernel", "bound": "tensor", "achieved": stages[dominant]["tflops"],
+                "peak": peaks["bf16_tflops"], "unit": "TFLOP/s"}, NCU_TRAFFIC.get("hash")
+    if dominant == "retrieve":
+        return {"kernel": "hamming_tc_kernel<256> (segmented)", "bound": "tensor",
+                "achieved": stages["retrieve"]["tflops_fp8"], "peak": 2.0 * peaks["bf16_tflops"],
+                "unit": "TFLOP/s"}, NCU_TRAFFIC.get("retrieve")
+    if matcher == "popc":
+        return {"kernel": "hamming_nn_kernel", "bound": "alu", "achieved": stages["match"]["gwordops"],
+                "peak": stages["match"]["gwordops"] / stages["match"]["frac_popc"], "unit": "Gwordop/s"}, \
+            NCU_TRAFFIC.get("match")
+    return {"kernel": "hamming_tc_kernel", "bound": "tensor", "achieved": stages["match"]["tflops_fp8"],
+            "peak": 2.0 * peaks["bf16_tflops"], "unit": "TFLOP/s"}, NCU_TRAFFIC.get("match_tc")
+
 
 def run_gpu_arm(args, rank, world, local_rank):
     import torch
@@ -268,10 +521,11 @@ def run_gpu_arm(args, rank, world, local_rank):
     ss.load()
     device = torch.device("cuda", local_rank)
     torch.cuda.set_device(device)
-    wl = workloads.WORKLOADS[args.workload]
+    wl = ALL_WORKLOADS[args.workload]
     seed = wl.base_seed + 7919 * rank
-    prob = Problem(wl, device, seed, args.matcher)
+    prob = make_problem(wl, device, seed, args.matcher)
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
+    n_ev = len(prob.STAGES) + 1
 
     for _ in range(max(args.warmup, 3)):
         prob.step()
@@ -279,7 +533,7 @@ def run_gpu_arm(args, rank, world, local_rank):
     ss.check_flag(prob.flag, "warm-up")
 
     K = args.steps
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(n_ev)] for _ in range(K)]
     gpu_id = None
     try:
         gpu_id = "GPU-" + str(torch.cuda.get_device_properties(device).uuid)
@@ -300,11 +554,10 @@ def run_gpu_arm(args, rank, world, local_rank):
     barrier(device)
     ss.check_flag(prob.flag, "timed steps")
 
-    st = np.array([[evs[k][0].elapsed_time(evs[k][1]), evs[k][1].elapsed_time(evs[k][2]),
-                    evs[k][2].elapsed_time(evs[k][3])] for k in range(K)])
-    ms_local = float(st.sum(axis=1).mean())
+    st = np.array([[evs[k][i].elapsed_time(evs[k][i + 1]) for i in range(n_ev - 1)] for k in range(K)])
+    ms_local = float(evs_total(evs))
     ms_step = reduce_max(ms_local, device)
-    stage_ms = {n: reduce_max(float(st[:, i].mean()), device) for i, n in enumerate(["hash", "match", "gather"])}
+    stage_ms = {n: reduce_max(float(st[:, i].mean()), device) for i, n in enumerate(prob.STAGES)}
     W = work(wl)
     value = world * W["targets"] / (ms_step * 1e-3)
 
@@ -312,43 +565,11 @@ def run_gpu_arm(args, rank, world, local_rank):
     props = torch.cuda.get_device_properties(device)
     clocks = sampler.summary() if not args.no_clocks else None
     sm_mhz = (clocks or {}).get("sm_mhz") or 2070.0
-    stages = {
-        "hash": {"ms": stage_ms["hash"], "tflops": W["hash_flops"] / (stage_ms["hash"] * 1e-3) / 1e12,
-                 "gbs": W["hash_bytes"] / (stage_ms["hash"] * 1e-3) / 1e9},
-        "match": {"ms": stage_ms["match"], "gwordops": W["match_wordops"] / (stage_ms["match"] * 1e-3) / 1e9},
-        "gather": {"ms": stage_ms["gather"], "gbs": W["gather_bytes"] / (stage_ms["gather"] * 1e-3) / 1e9},
-    }
-    stages["hash"]["frac_tensor"] = stages["hash"]["tflops"] / peaks["bf16_tflops"]
-    stages["hash"]["frac_hbm"] = stages["hash"]["gbs"] / peaks["hbm_gbs"]
     popc_peak = popc_peak_wordops(sm_mhz, props.multi_processor_count)
-    stages["match"]["matcher"] = args.matcher
-    if args.matcher == "popc":
-        stages["match"]["frac_popc"] = stages["match"]["gwordops"] * 1e9 / popc_peak
-    else:
-        # the GEMM over padded code bits: 2 * n_t * n_ref * kpad fp8 flops; fp8 peak = 2 x bf16 (nominal ratio)
-        kpad = ((wl.nbits + 127) // 128) * 128
-        fl = 2.0 * W["targets"] * wl.n_ref * kpad
-        stages["match"]["tflops_fp8"] = fl / (stage_ms["match"] * 1e-3) / 1e12
-        stages["match"]["frac_fp8_tensor"] = stages["match"]["tflops_fp8"] / (2.0 * peaks["bf16_tflops"])
-    stages["gather"]["frac_hbm"] = stages["gather"]["gbs"] / peaks["hbm_gbs"]
+    stages = stage_report(wl, W, stage_ms, peaks, popc_peak, args.matcher)
 
     dominant = max(stage_ms, key=stage_ms.get)
-    if dominant == "gather":
-        roof = {"kernel": "kv_gather_kernel", "bound": "hbm", "achieved": stages["gather"]["gbs"],
-                "peak": peaks["hbm_gbs"], "unit": "GB/s"}
-        tr = NCU_TRAFFIC.get("gather")
-    elif dominant == "hash":
-        roof = {"kernel": "lsh_hash_kernel", "bound": "tensor", "achieved": stages["hash"]["tflops"],
-                "peak": peaks["bf16_tflops"], "unit": "TFLOP/s"}
-        tr = NCU_TRAFFIC.get("hash")
-    elif args.matcher == "popc":
-        roof = {"kernel": "hamming_nn_kernel", "bound": "alu", "achieved": stages["match"]["gwordops"],
-                "peak": popc_peak / 1e9, "unit": "Gwordop/s"}
-        tr = NCU_TRAFFIC.get("match")
-    else:
-        roof = {"kernel": "hamming_tc_kernel", "bound": "tensor", "achieved": stages["match"]["tflops_fp8"],
-                "peak": 2.0 * peaks["bf16_tflops"], "unit": "TFLOP/s"}
-        tr = NCU_TRAFFIC.get("match_tc")
+    roof, tr = roofline_for(dominant, stages, peaks, args.matcher)
     roof["frac"] = roof["achieved"] / roof["peak"]
     roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"
     if tr and tr.get("sha") == kernel_sha(tr["file"]):
@@ -362,21 +583,31 @@ def run_gpu_arm(args, rank, world, local_rank):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(wl, prob)
 
+    config = {"workload": wl.name, "n_ref": wl.n_ref, "n_tgt": wl.n_tgt, "n_batch": wl.n_batch,
+              "n_seg": wl.n_seg, "d": wl.d, "nbits": wl.nbits, "kv": list(wl.kv),
+              "parallelism": f"replicas x{world}", "l2": "flushed before every step (256 MB write)",
+              "matcher": args.matcher}
+    if isinstance(prob, RetrieveProblem):
+        config["retrieved"] = prob.winner
+        config["stored_codes"] = "computed when the prompts were stored (outside the timed region)"
     line = {
-        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
+        "metric": METRIC_RETRIEVE if isinstance(prob, RetrieveProblem) else METRIC, "value": value,
+        "unit": "tokens/s", "n_gpus": world, "steps": K,
         "warmup": max(args.warmup, 3), "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16" if wl.emb_dtype == "bf16" else "f32",
         "data": "synthetic (seeded; see workloads.py)",
-        "config": {"workload": wl.name, "n_ref": wl.n_ref, "n_tgt": wl.n_tgt, "n_batch": wl.n_batch,
-                   "n_seg": wl.n_seg, "d": wl.d, "nbits": wl.nbits, "kv": list(wl.kv),
-                   "parallelism": f"replicas x{world}", "l2": "flushed before every step (256 MB write)",
-                   "matcher": args.matcher},
+        "config": config,
         "roofline": roof, "stages": stages, "e2e": e2e, "cpu_baseline": cpu,
-        "gpu_launches": LAUNCHES_PER_STEP * K, "clocks": clocks, "wall_s_timed": reduce_max(t_wall, device),
+        "gpu_launches": prob.LAUNCHES_PER_STEP * K, "clocks": clocks, "wall_s_timed": reduce_max(t_wall, device),
         "impl": "gb300",
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
+
+
+def evs_total(evs):
+    """Mean device time of a step: first to last event of each step."""
+    return float(np.mean([e[0].elapsed_time(e[-1]) for e in evs]))
 
 
 class _Null:
@@ -387,32 +618,13 @@ class _Null:
         return False
 
 
-def run_e2e(args, prob: Problem, device):
-    """Same metric through the public API with host buffers: every step copies its inputs
-    (embedding rows, positions, the reference K/V cache) from pinned host memory, runs the
-    three calls and reads the match result (idx, dist) back."""
+def run_e2e(args, prob, device):
+    """Same metric through the public API with host buffers (the problem's e2e_plan says which
+    inputs are copied in and which results are read back every step)."""
     import torch
 
     wl = prob.wl
-    h_emb = prob.emb.cpu().pin_memory()
-    h_pos = prob.pos.cpu().pin_memory()
-    h_k = [t.cpu().pin_memory() for t in prob.ref_k]
-    h_v = [t.cpu().pin_memory() for t in prob.ref_v]
-    h_idx = torch.empty_like(prob.idx, device="cpu").pin_memory()
-    h_dist = torch.empty_like(prob.dist, device="cpu").pin_memory()
-    h2d = h_emb.numel() * h_emb.element_size() + h_pos.numel() * 4 + \
-        sum(t.numel() * t.element_size() for t in h_k + h_v)
-    d2h = (h_idx.numel() + h_dist.numel()) * 4
-
-    def one():
-        prob.emb.copy_(h_emb, non_blocking=True)
-        prob.pos.copy_(h_pos, non_blocking=True)
-        for d, h in zip(prob.ref_k + prob.ref_v, h_k + h_v):
-            d.copy_(h, non_blocking=True)
-        prob.step()
-        h_idx.copy_(prob.idx, non_blocking=True)
-        h_dist.copy_(prob.dist, non_blocking=True)
-
+    one, h2d, d2h, read = prob.e2e_plan()
     for _ in range(3):
         one()
     torch.cuda.synchronize()
@@ -424,7 +636,7 @@ def run_e2e(args, prob: Problem, device):
         one()
         b.record()
         b.synchronize()
-        _ = int(h_idx[0])  # the host reads the result
+        _ = read()  # the host reads the result
         times.append(a.elapsed_time(b))
     ms = reduce_max(float(np.mean(times)), device)
     _, world, _ = dist_info()
@@ -462,11 +674,73 @@ def _oracle_inputs(oracle, wl, emb, pos, R, k_dev=None, v_dev=None):
     return ref_codes, k_np, v_np
 
 
+def _oracle_retrieve_setup(oracle, wl, emb, pos, R):
+    """Store time for the oracle: every stored prompt's plain and rotary codes."""
+    n_pool = wl.n_ref
+    rcodes, _ = oracle.hash_codes(emb[:n_pool], np.zeros(n_pool, dtype=np.int32), R)
+    codes, _ = oracle.hash_codes(emb[:n_pool], pos[:n_pool], R)
+    return {"rcodes": rcodes, "codes": codes, "offsets": [m * wl.seg_len for m in range(wl.n_seg + 1)]}
+
+
+def _oracle_retrieve_sample(oracle, wl, emb, pos, R, ctx, kv_of, tsel):
+    """The oracle's retrieval step for the target tokens `tsel`: their plain codes, the
+    similarity to every stored prompt and the winner, their rotary codes, the match against the
+    winner's codes, the gather of the winner's K/V rows.  Returns (seconds, winner)."""
+    rows = wl.n_ref + tsel
+    t0 = time.perf_counter()
+    tr, _ = oracle.hash_codes(emb[rows], np.zeros(len(tsel), dtype=np.int32), R)
+    _, _, best, _ = oracle.retrieve(tr, ctx["rcodes"], ctx["offsets"], wl.nbits)
+    tc, _ = oracle.hash_codes(emb[rows], pos[rows], R)
+    o = ctx["offsets"]
+    idx, _ = oracle.match(tc, ctx["codes"][o[best]:o[best + 1]])
+    k, v = kv_of(best)
+    oracle.gather_kv(k, v, idx)
+    return time.perf_counter() - t0, best
+
+
+def _kv_from_device(prob):
+    import torch
+
+    cache = {}
+
+    def kv_of(m):
+        if m not in cache:
+            cache.clear()
+            cache[m] = (prob.ref_k[m].cpu().view(torch.int16).numpy().view(np.uint16),
+                        prob.ref_v[m].cpu().view(torch.int16).numpy().view(np.uint16))
+        return cache[m]
+
+    return kv_of
+
+
+def _kv_from_host(wl):
+    cache = {}
+
+    def kv_of(m):
+        if m not in cache:
+            cache.clear()
+            cache[m] = workloads.kv_cache(wl, segment=m)
+        return cache[m]
+
+    return kv_of
+
+
 def cpu_baseline(wl, prob):
     """The oracle as it stands on the host cores: one bounded sample of the workload."""
     import oracle
 
     oracle.build()
+    if wl.recipe == "retrieve":
+        emb, pos = prob.host_emb, prob.host_pos
+        R = prob.hyp.cpu().view(__import__("torch").int16).numpy().view(np.uint16)
+        ctx = _oracle_retrieve_setup(oracle, wl, emb, pos, R)
+        n_s = wl.n_tgt
+        secs, best = _oracle_retrieve_sample(oracle, wl, emb, pos, R, ctx, _kv_from_device(prob), np.arange(n_s))
+        return {"value": n_s / secs, "unit": "tokens/s", "cores": oracle.num_threads(), "kind": "oracle",
+                "sample": f"all {n_s} target tokens: plain codes, similarity to the {wl.n_seg} stored prompts "
+                          f"({wl.n_ref} stored codes, computed beforehand as on the GPU), rotary codes, match "
+                          f"against the winner ({best}), gather of its {wl.n_layers}x{wl.n_heads} K/V rows; "
+                          f"seconds={secs:.2f}"}
     emb, pos = prob.host_emb, prob.host_pos
     R = prob.hyp.cpu().view(__import__("torch").int16).numpy().view(np.uint16)
     ref_codes, k_np, v_np = _oracle_inputs(oracle, wl, emb, pos, R, prob.ref_k, prob.ref_v)
@@ -485,24 +759,38 @@ def run_reference_arm(args, rank, world):
     import oracle
 
     oracle.build()
-    wl = workloads.WORKLOADS[args.workload]
+    wl = ALL_WORKLOADS[args.workload]
     emb, pos, _ = workloads.prompt_rows(wl, batches=[0])
     R = workloads.hyperplanes(wl)
-    ref_codes, k_np, v_np = _oracle_inputs(oracle, wl, emb, pos, R)
     per_step = 64
     g = np.random.default_rng(wl.base_seed)
+    if wl.recipe == "retrieve":
+        ctx = _oracle_retrieve_setup(oracle, wl, emb, pos, R)
+        kv_of = _kv_from_host(wl)
+
+        def sample_step(tsel):
+            return _oracle_retrieve_sample(oracle, wl, emb, pos, R, ctx, kv_of, tsel)[0]
+
+        sample = (f"per step {per_step} random target tokens: plain codes, similarity to the {wl.n_seg} stored "
+                  f"prompts ({wl.n_ref} stored codes computed beforehand), rotary codes, match against the "
+                  f"winner, gather of its K/V rows")
+    else:
+        ref_codes, k_np, v_np = _oracle_inputs(oracle, wl, emb, pos, R)
+
+        def sample_step(tsel):
+            return _oracle_sample(oracle, wl, emb, pos, R, ref_codes, k_np, v_np, tsel)
+
+        sample = (f"per step {per_step} random target tokens of prompt 0: hash of them plus their share of "
+                  f"reference rows, match against all {wl.n_ref} reference codes, gather of their K/V rows")
     for _ in range(max(args.warmup, 3)):
-        _oracle_sample(oracle, wl, emb, pos, R, ref_codes, k_np, v_np, np.sort(g.choice(wl.n_tgt, per_step, False)))
+        sample_step(np.sort(g.choice(wl.n_tgt, per_step, False)))
     secs = []
     for _ in range(args.steps):
-        secs.append(_oracle_sample(oracle, wl, emb, pos, R, ref_codes, k_np, v_np,
-                                   np.sort(g.choice(wl.n_tgt, per_step, False))))
+        secs.append(sample_step(np.sort(g.choice(wl.n_tgt, per_step, False))))
     ms = 1e3 * float(np.mean(secs))
     value = per_step / (ms * 1e-3)
-    sample = (f"per step {per_step} random target tokens of prompt 0: hash of them plus their share of reference "
-              f"rows, match against all {wl.n_ref} reference codes, gather of their K/V rows")
     line = {
-        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "impl": "reference", "metric": METRIC_RETRIEVE if wl.recipe == "retrieve" else METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded; see workloads.py)",
         "config": {"workload": wl.name, "n_ref": wl.n_ref, "n_tgt": wl.n_tgt, "n_batch": wl.n_batch,

@@ -178,6 +178,49 @@ semshare_status semshare_match_tc(const uint32_t* tgt_codes, int64_t n_tgt, cons
                                   uint32_t* err_flag, void* stream);
 
 /*
+ * semshare_retrieve -- reference retrieval: which stored prompt the target should reuse.
+ *
+ * Sec. 3.2: the stored prompt with the highest LSH-distance-based similarity to the target is
+ * the reference.  App. A.3: Similarity = clip(1 - d_norm, 0, 1) with d_norm = LSH_dist / max_dist
+ * (the paper's min(dist) = 0, max(dist) = 30).  Sec. 4.4: reuse applies only when that
+ * similarity exceeds 0.8.  The paper does not spell out LSH_dist for two prompts; here it is the
+ * mean, over the target's tokens, of each token's Hamming distance to its nearest token of the
+ * candidate (the per-token distance of Sec. 3.3 averaged over the target).
+ *
+ *   tgt_codes     device, [n_tgt][nbits/32] packed codes of the target prompt (4-byte aligned)
+ *   pool_codes    device, the codes of all candidates concatenated, [n_pool][nbits/32]
+ *   cand_offsets  HOST, n_cand + 1 values: candidate c is pool rows
+ *                 [cand_offsets[c], cand_offsets[c+1]); cand_offsets[0] = 0, strictly
+ *                 increasing (no empty candidate), n_pool = cand_offsets[n_cand]; read before
+ *                 the call returns
+ *   n_cand        1 <= n_cand <= SEMSHARE_RETRIEVE_MAX_CANDIDATES (more returns EUNSUPPORTED)
+ *   nbits         32..256, a multiple of 32
+ *   max_dist      the normaliser of d_norm (> 0); threshold: reuse applies when the best
+ *                 similarity is strictly above it
+ *   mean_dist     device double[n_cand] or NULL: LSH_dist of every candidate (exact: the integer
+ *                 sum of nearest distances divided by n_tgt in fp64)
+ *   similarity    device double[n_cand] or NULL: clip(1 - mean_dist/max_dist, 0, 1) in fp64
+ *   best          device int32: the candidate of greatest similarity, lowest index on ties
+ *   applies       device int32 or NULL: 1 if similarity[best] > threshold, else 0
+ *   idx, dist     device int32[n_tgt] or NULL: each target token's nearest row of the best
+ *                 candidate (a global pool row; ties to the lowest row) and its distance --
+ *                 semshare_match against that candidate's rows, shifted by its offset
+ *   workspace     device scratch of at least semshare_retrieve_workspace_size(n_tgt, n_pool,
+ *                 n_cand, nbits) bytes, 256-byte aligned; contents on entry do not matter
+ *   err_flag      as for semshare_match_tc (SEMSHARE_FLAG_TIMEOUT: the outputs are invalid)
+ * n_tgt must be >= 1 (the mean of no distances is undefined).  Returns EINVAL / EUNSUPPORTED
+ * for bad arguments before anything is enqueued, ECUDA if a launch fails.  Outputs are written
+ * in stream order; read them after synchronising the stream.
+ */
+#define SEMSHARE_RETRIEVE_MAX_CANDIDATES 256
+size_t semshare_retrieve_workspace_size(int64_t n_tgt, int64_t n_pool, int32_t n_cand, int32_t nbits);
+semshare_status semshare_retrieve(const uint32_t* tgt_codes, int64_t n_tgt, const uint32_t* pool_codes,
+                                  const int64_t* cand_offsets, int32_t n_cand, int32_t nbits, double max_dist,
+                                  double threshold, double* mean_dist, double* similarity, int32_t* best,
+                                  int32_t* applies, int32_t* idx, int32_t* dist, void* workspace,
+                                  size_t workspace_bytes, uint32_t* err_flag, void* stream);
+
+/*
  * semshare_match_static -- semshare_match without a caller-provided workspace.
  *
  * The paper has no counterpart: this entry point exists for callers that cannot allocate

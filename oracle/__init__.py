@@ -184,7 +184,7 @@ def gather_kv(seg_k, seg_v, idx: np.ndarray, out_k: np.ndarray | None = None, ou
 
 
 def retrieve(tgt_codes: np.ndarray, pool_codes: np.ndarray, seg_offsets, nbits: int | None = None,
-             dmax: float = 30.0, threshold: float = 0.8):
+             max_dist: float = 30.0, threshold: float = 0.8):
     """Reference retrieval by LSH-distance similarity (Sec. 3.2, App. A.3, Sec. 4.4).
 
     pool_codes: the candidate prompts' codes concatenated; candidate s is rows
@@ -199,6 +199,6 @@ def retrieve(tgt_codes: np.ndarray, pool_codes: np.ndarray, seg_offsets, nbits: 
     sim = np.zeros(n_seg)
     best = np.zeros(1, dtype=np.int32)
     applies = np.zeros(1, dtype=np.int32)
-    _load().oracle_retrieve(_ptr(t), t.shape[0], _ptr(p), _ptr(offs), n_seg, nbits, float(dmax), float(threshold),
+    _load().oracle_retrieve(_ptr(t), t.shape[0], _ptr(p), _ptr(offs), n_seg, nbits, float(max_dist), float(threshold),
                             _ptr(mean), _ptr(sim), _ptr(best), _ptr(applies))
     return mean, sim, int(best[0]), bool(applies[0])

@@ -3,7 +3,8 @@
 The path: rotary position encoding of the embedding rows of a target and a reference prompt
 (Sec. 3.3.1, Eq. 1), random-hyperplane LSH sign codes (Sec. 3.3, App. A.2), the Hamming
 nearest reference token of every target token (Sec. 3.3), and the rearrangement of the
-reference K/V cache into the target's order (Sec. 3.3, Sec. 3.3.2).
+reference K/V cache into the target's order (Sec. 3.3, Sec. 3.3.2); before it, the retrieval of
+the stored prompt to reuse by LSH-distance similarity (Sec. 3.2, App. A.3).
 
 The compute lives in libsemshare.so (C ABI: include/semshare.h); this package is its thin
 ctypes binding with the same names.  Build the library with `paper_2509_24832_gb300.build`."""
@@ -13,6 +14,10 @@ from ._native import (  # noqa: F401
     KVLayout,
     LIB_PATH,
     MATCH_STATIC_MAX_TARGETS,
+    RETRIEVE_MAX_CANDIDATES,
+    SIMILARITY_MAX_DIST,
+    SIMILARITY_THRESHOLD,
+    Retrieval,
     SemshareError,
     check_flag,
     flag_status,
@@ -29,6 +34,8 @@ from ._native import (  # noqa: F401
     semshare_match_tc,
     semshare_match_tc_workspace_size,
     semshare_match_workspace_size,
+    semshare_retrieve,
+    semshare_retrieve_workspace_size,
     semshare_rope_table,
     status_string,
 )

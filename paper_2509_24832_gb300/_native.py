@@ -8,6 +8,7 @@ from __future__ import annotations
 import ctypes
 import os
 import threading
+from typing import NamedTuple
 
 import torch
 
@@ -66,6 +67,11 @@ def load():
         lib.semshare_match_tc_workspace_size.restype = ctypes.c_size_t
         lib.semshare_match_tc.argtypes = [P, i64, P, i64, i32, P, P, P, ctypes.c_size_t, P, P]
         lib.semshare_match_tc.restype = ctypes.c_int
+        lib.semshare_retrieve_workspace_size.argtypes = [i64, i64, i32, i32]
+        lib.semshare_retrieve_workspace_size.restype = ctypes.c_size_t
+        lib.semshare_retrieve.argtypes = [P, i64, P, P, i32, i32, ctypes.c_double, ctypes.c_double, P, P, P, P, P, P,
+                                          P, ctypes.c_size_t, P, P]
+        lib.semshare_retrieve.restype = ctypes.c_int
         lib.semshare_match_static.argtypes = [P, i64, P, i64, i32, P, P, P]
         lib.semshare_match_static.restype = ctypes.c_int
         lib.semshare_gather_kv.argtypes = [P, P, P, i32, KVLayout, P, i64, i32, P, P, KVLayout, P, P]
@@ -252,6 +258,74 @@ def semshare_match_tc(tgt_codes: torch.Tensor, ref_codes: torch.Tensor, idx: tor
                                   _stream(stream))
     _check(st, "semshare_match_tc")
     return idx, dist
+
+
+RETRIEVE_MAX_CANDIDATES = 256
+SIMILARITY_MAX_DIST = 30.0   # App. A.3: max(dist) of the normalised LSH distance
+SIMILARITY_THRESHOLD = 0.8   # Sec. 4.4: reuse applies above this similarity
+
+
+def semshare_retrieve_workspace_size(n_tgt: int, n_pool: int, n_cand: int, nbits: int) -> int:
+    return int(load().semshare_retrieve_workspace_size(int(n_tgt), int(n_pool), int(n_cand), int(nbits)))
+
+
+class Retrieval(NamedTuple):
+    """Outputs of semshare_retrieve, all device tensors."""
+    mean_dist: torch.Tensor   # float64 [n_cand]: LSH_dist of every candidate
+    similarity: torch.Tensor  # float64 [n_cand]
+    best: torch.Tensor        # int32 [1]: candidate of greatest similarity
+    applies: torch.Tensor     # int32 [1]: 1 if similarity[best] > threshold
+    idx: torch.Tensor | None  # int32 [n_tgt]: nearest global pool row within the best candidate
+    dist: torch.Tensor | None
+
+
+def semshare_retrieve(tgt_codes: torch.Tensor, pool_codes: torch.Tensor, cand_offsets,
+                      max_dist: float = SIMILARITY_MAX_DIST, threshold: float = SIMILARITY_THRESHOLD,
+                      want_match: bool = True, workspace: torch.Tensor | None = None,
+                      err_flag: torch.Tensor | None = None, nbits: int | None = None, stream=None,
+                      out: Retrieval | None = None) -> Retrieval:
+    """Reference retrieval by LSH-distance similarity (Sec. 3.2, App. A.3, Sec. 4.4).
+
+    pool_codes holds the candidates' codes back to back; cand_offsets (host sequence of
+    n_cand + 1 ints) delimits them.  With want_match, idx/dist are the nearest rows of the
+    best candidate for every target row.  `out` (a Retrieval of preallocated device tensors,
+    idx/dist None to skip the match) is filled instead of allocating."""
+    _need_cuda(tgt_codes, "tgt_codes")
+    _need_cuda(pool_codes, "pool_codes")
+    if not tgt_codes.is_contiguous() or not pool_codes.is_contiguous():
+        raise ValueError("codes must be contiguous")
+    n_tgt, w = tgt_codes.shape
+    if pool_codes.shape[1] != w:
+        raise ValueError("code widths differ")
+    offs = (ctypes.c_int64 * len(cand_offsets))(*[int(o) for o in cand_offsets])
+    n_cand = len(cand_offsets) - 1
+    nbits = 32 * w if nbits is None else nbits
+    dev = tgt_codes.device
+    if out is not None:
+        mean, sim, best, applies, idx, dist = out
+        for t, n in ((mean, n_cand), (sim, n_cand), (best, 1), (applies, 1), (idx, n_tgt), (dist, n_tgt)):
+            if t is not None and (t.device != dev or not t.is_contiguous() or t.numel() < n):
+                raise ValueError("preallocated retrieval output of the wrong size or device")
+    else:
+        mean = torch.empty(max(n_cand, 1), dtype=torch.float64, device=dev)
+        sim = torch.empty(max(n_cand, 1), dtype=torch.float64, device=dev)
+        choice = torch.empty(2, dtype=torch.int32, device=dev)
+        best, applies = choice[:1], choice[1:]
+        idx = dist = None
+        if want_match:
+            idx = torch.empty(n_tgt, dtype=torch.int32, device=dev)
+            dist = torch.empty(n_tgt, dtype=torch.int32, device=dev)
+    if workspace is None:
+        need = semshare_retrieve_workspace_size(n_tgt, int(pool_codes.shape[0]), n_cand, nbits)
+        workspace = torch.empty(max(256, need), dtype=torch.uint8, device=dev)
+    st = load().semshare_retrieve(_ptr(tgt_codes), n_tgt, _ptr(pool_codes), offs, n_cand, nbits, float(max_dist),
+                                  float(threshold), _ptr(mean), _ptr(sim), _ptr(best), _ptr(applies),
+                                  _ptr(idx), _ptr(dist), _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                  _ptr(err_flag), _stream(stream))
+    _check(st, "semshare_retrieve")
+    if out is not None:
+        return out
+    return Retrieval(mean[:n_cand], sim[:n_cand], best, applies, idx, dist)
 
 
 def semshare_match_static(tgt_codes: torch.Tensor, ref_codes: torch.Tensor, idx: torch.Tensor | None = None,

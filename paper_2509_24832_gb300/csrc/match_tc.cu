@@ -20,6 +20,14 @@
 // (tcgen05.ld, lane = target, running arg-max).  The (target block, reference block) tiles are
 // split into one equal contiguous range per CTA, target blocks outermost.  Every pipeline wait
 // is bounded (SEMSHARE_FLAG_TIMEOUT), nothing traps.
+//
+// Segmented mode (semshare_retrieve).  The reference rows are the concatenated codes of several
+// candidate prompts; the epilogue keeps one best key per (candidate, target) instead of one per
+// target.  Candidate boundaries are the same for every lane of a warp (lanes are targets,
+// columns are references), so the boundary tests are warp-uniform: a 32-column chunk without a
+// boundary takes the plain arg-max, one with a boundary is cut into runs and the key of the
+// finished candidate is flushed with the atomicMin.  A reduction over targets then gives each
+// candidate's summed nearest distance, its similarity (App. A.3) and the arg-max candidate.
 #include <cuda.h>
 
 #include "common.cuh"
@@ -37,6 +45,14 @@ constexpr int kEpiWarp0 = 4;
 constexpr unsigned long long kNoKey = ~0ull;
 constexpr size_t kFixedSmem = 1024 + 256;
 
+// Candidate (segment) boundaries of the reference rows, passed by value: off[0] = 0 <
+// off[1] < ... < off[n_seg] = n_ref.  kMax = 1 for the plain search.
+template <int kMax>
+struct SegTable {
+    int32_t n_seg;
+    int64_t off[kMax + 1];
+};
+
 struct TcArgs {
     int64_t n_tgt;
     int64_t n_ref;
@@ -46,7 +62,7 @@ struct TcArgs {
     int32_t kchunks;
     uint32_t a_bytes;  // one A buffer: 128 rows x kchunks*128 bytes
     uint32_t b_bytes;  // one B buffer: 256 rows x kchunks*128 bytes
-    unsigned long long* keys;
+    unsigned long long* keys;  // [n_seg][n_tgt]
     uint32_t* err_flag;
     uint64_t wait_limit_ns;
 };
@@ -55,7 +71,8 @@ struct TcArgs {
 // kpad; the keys of the search are reset on the way.
 __global__ void expand_codes_kernel(const uint32_t* __restrict__ tgt, int64_t n_tgt, const uint32_t* __restrict__ ref,
                                     int64_t n_ref, int32_t nbits, int32_t kpad, uint8_t* __restrict__ tpm,
-                                    uint8_t* __restrict__ rpm, unsigned long long* __restrict__ keys) {
+                                    uint8_t* __restrict__ rpm, unsigned long long* __restrict__ keys, int64_t n_keys,
+                                    unsigned int* __restrict__ counter) {
     const int W = nbits >> 5;
     const int per_row = kpad >> 4;  // 16-byte pieces per row
     const int64_t total = (n_tgt + n_ref) * per_row;
@@ -81,7 +98,8 @@ __global__ void expand_codes_kernel(const uint32_t* __restrict__ tgt, int64_t n_
         uint8_t* dst = row < n_tgt ? tpm + row * kpad : rpm + (row - n_tgt) * kpad;
         *reinterpret_cast<uint4*>(dst + b0) = out;
     }
-    for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < n_tgt; t += stride) keys[t] = kNoKey;
+    for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < n_keys; t += stride) keys[t] = kNoKey;
+    if (counter != nullptr && blockIdx.x == 0 && threadIdx.x == 0) *counter = 0u;
 }
 
 __global__ void tc_keys_split_kernel(const unsigned long long* __restrict__ keys, int64_t n, int32_t* __restrict__ idx,
@@ -102,9 +120,10 @@ __device__ __forceinline__ bool drain_wait(uint32_t bar, uint32_t parity, uint64
     return true;
 }
 
+template <int kMaxSeg>
 __global__ void __launch_bounds__(kThreads, 1)
     hamming_tc_kernel(const __grid_constant__ CUtensorMap tm_t, const __grid_constant__ CUtensorMap tm_r,
-                      const TcArgs a) {
+                      const TcArgs a, const __grid_constant__ SegTable<kMaxSeg> seg) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_addr(smem_raw);
     const uint32_t sbase = (raw + 1023u) & ~1023u;
@@ -235,20 +254,45 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
     } else if (warp >= kEpiWarp0) {
         // ---------------- epilogue: best reference of every target row ----------------
+        // (per candidate in segmented mode; candidate cs covers columns [off[cs], next_b))
         const int ew = warp - kEpiWarp0;
         const int r = ew * 32 + lane;
         uint32_t acc = 0;
-        int64_t cur_tb = -1;
+        int64_t cur_tb = -1, col0 = 0, next_b = 0;
+        int32_t cs = 0;
         unsigned long long best = kNoKey;
+        // fold the tile's best key 256*dot - j (j = column within the tile) into `best`
+        auto fold = [&](float bk) {
+            if (bk > -1.0e38f) {
+                const int ik = __float2int_rn(bk);
+                const int dot = -((-ik) >> 8);  // ceil(ik / 256)
+                const int j = 256 * dot - ik;    // 0..255
+                const unsigned long long dist = static_cast<unsigned long long>((a.nbits - dot) >> 1);
+                const unsigned long long cand = (dist << 32) | static_cast<unsigned long long>(col0 + j);
+                best = cand < best ? cand : best;
+            }
+        };
+        auto flush = [&]() {
+            const int64_t g = cur_tb * kTM + r;
+            if (g < a.n_tgt && best != kNoKey && cs < seg.n_seg)
+                atomicMin(a.keys + static_cast<int64_t>(cs) * a.n_tgt + g, best);
+            best = kNoKey;
+        };
         for (int64_t u = u0; u < u1; ++u, ++acc) {
             const int64_t tb = u / a.n_rb, rb = u - tb * a.n_rb;
+            col0 = rb * kTN;
             if (tb != cur_tb) {
-                if (cur_tb >= 0) {
-                    const int64_t g = cur_tb * kTM + r;
-                    if (g < a.n_tgt && best != kNoKey) atomicMin(a.keys + g, best);
-                }
+                if (cur_tb >= 0) flush();
                 cur_tb = tb;
                 best = kNoKey;
+                // candidate holding column col0: the largest cs with off[cs] <= col0
+                int lo = 0, hi = seg.n_seg - 1;
+                while (lo < hi) {
+                    const int mid = (lo + hi + 1) >> 1;
+                    if (seg.off[mid] <= col0) lo = mid; else hi = mid - 1;
+                }
+                cs = lo;
+                next_b = seg.off[lo + 1];
             }
             const uint32_t buf = acc & 1u;
             const bool got = mbar_wait_bounded(bar_accfull + 8 * buf, (acc >> 1) & 1u, abort_flag, err,
@@ -258,40 +302,48 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             tc_fence_after_sync();
-            const int64_t rem = a.n_ref - rb * kTN;
+            const int64_t rem = a.n_ref - col0;
             const int valid = rem < kTN ? static_cast<int>(rem) : kTN;
             const uint32_t taddr = tmem_base + (static_cast<uint32_t>(ew * 32) << 16) + buf * kTN;
-            float bk = -3.0e38f;  // best key 256*dot - j of this tile
+            float bk = -3.0e38f;  // best key 256*dot - j of this tile (current candidate)
 #pragma unroll
             for (int q = 0; q < kTN / 32; ++q) {
                 uint32_t v[32];
                 tmem_load_32cols(taddr + q * 32, v);
                 tmem_load_wait();
-                if (q * 32 + 32 <= valid) {
+                const int64_t c0 = col0 + q * 32;
+                if (q * 32 + 32 <= valid && c0 + 32 <= next_b) {
 #pragma unroll
                     for (int j = 0; j < 32; ++j)
                         bk = fmaxf(bk, fmaf(__uint_as_float(v[j]), 256.0f, -static_cast<float>(q * 32 + j)));
                 } else if (q * 32 < valid) {
+                    // ragged end and/or candidate boundaries inside the chunk: runs [js, je)
+                    const int jend = valid - q * 32 < 32 ? valid - q * 32 : 32;
+                    int js = 0;
+                    for (;;) {
+                        const int64_t lim_b = next_b - c0;  // >= js: the boundary is not passed yet
+                        const int je = lim_b < jend ? static_cast<int>(lim_b) : jend;
 #pragma unroll
-                    for (int j = 0; j < 32; ++j)
-                        if (q * 32 + j < valid)
-                            bk = fmaxf(bk, fmaf(__uint_as_float(v[j]), 256.0f, -static_cast<float>(q * 32 + j)));
+                        for (int j = 0; j < 32; ++j)
+                            if (j >= js && j < je)
+                                bk = fmaxf(bk, fmaf(__uint_as_float(v[j]), 256.0f, -static_cast<float>(q * 32 + j)));
+                        if (je == jend) break;
+                        // column c0 + je opens candidate cs + 1
+                        fold(bk);
+                        bk = -3.0e38f;
+                        flush();
+                        ++cs;
+                        next_b = cs + 1 <= seg.n_seg ? seg.off[cs + 1] : a.n_ref;
+                        js = je;
+                    }
                 }
             }
             tc_fence_before_sync();
             __syncwarp();
             if (lane == 0) mbar_arrive(bar_accempty + 8 * buf);
-            const int ik = __float2int_rn(bk);
-            const int dot = -((-ik) >> 8);   // ceil(ik / 256)
-            const int j = 256 * dot - ik;     // 0..255
-            const unsigned long long dist = static_cast<unsigned long long>((a.nbits - dot) >> 1);
-            const unsigned long long cand = (dist << 32) | static_cast<unsigned long long>(rb * kTN + j);
-            best = cand < best ? cand : best;
+            fold(bk);
         }
-        if (cur_tb >= 0) {
-            const int64_t g = cur_tb * kTM + r;
-            if (g < a.n_tgt && best != kNoKey) atomicMin(a.keys + g, best);
-        }
+        if (cur_tb >= 0) flush();
     }
 
     tc_fence_before_sync();
@@ -304,58 +356,97 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 struct TcPlan {
     int32_t kpad;
-    size_t keys_bytes, t_bytes, r_bytes;
+    size_t keys_bytes, t_bytes, r_bytes, sums_bytes;
+    size_t total() const { return keys_bytes + t_bytes + r_bytes + sums_bytes; }
 };
 
-void plan_tc(int64_t n_tgt, int64_t n_ref, int32_t nbits, TcPlan* p) {
+size_t round256(size_t x) { return ((x + 255) / 256) * 256; }
+
+// n_seg = 0: the plain search (one key per target, no reduction scratch).
+void plan_tc(int64_t n_tgt, int64_t n_ref, int32_t nbits, int32_t n_seg, TcPlan* p) {
     p->kpad = ((nbits + kChunk - 1) / kChunk) * kChunk;
-    p->keys_bytes = ((static_cast<size_t>(n_tgt) * 8 + 255) / 256) * 256;
-    p->t_bytes = ((static_cast<size_t>(n_tgt) * p->kpad + 255) / 256) * 256;
-    p->r_bytes = ((static_cast<size_t>(n_ref) * p->kpad + 255) / 256) * 256;
+    p->keys_bytes = round256(static_cast<size_t>(n_tgt) * 8 * static_cast<size_t>(n_seg > 0 ? n_seg : 1));
+    p->t_bytes = round256(static_cast<size_t>(n_tgt) * p->kpad);
+    p->r_bytes = round256(static_cast<size_t>(n_ref) * p->kpad);
+    // per-candidate sums, then the arrival counter
+    p->sums_bytes = n_seg > 0 ? round256(static_cast<size_t>(n_seg) * 8 + 8) : 0;
 }
 
-}  // namespace
-}  // namespace semshare
-
-extern "C" size_t semshare_match_tc_workspace_size(int64_t n_tgt, int64_t n_ref, int32_t nbits) {
-    using namespace semshare;
-    if (n_tgt <= 0 || n_ref <= 0 || nbits < 32 || nbits > 256 || nbits % 32 != 0) return 0;
-    TcPlan p;
-    plan_tc(n_tgt, n_ref, nbits, &p);
-    return p.keys_bytes + p.t_bytes + p.r_bytes;
+// Per-candidate reduction (Sec. 3.2, App. A.3, Sec. 4.4): block s sums the nearest distances
+// of all targets to candidate s (exact, int64); the last block to finish turns the sums into
+// mean distances and similarities, picks the arg-max candidate (lowest index on ties) and
+// decides whether reuse applies.  fp64 throughout: the same rounding as a plain host program.
+__global__ void __launch_bounds__(256)
+    retrieve_finalize_kernel(const unsigned long long* __restrict__ keys, int64_t n_tgt, int32_t n_seg,
+                             double max_dist, double threshold, long long* sums, unsigned int* counter,
+                             double* __restrict__ mean_dist, double* __restrict__ similarity,
+                             int32_t* __restrict__ best, int32_t* __restrict__ applies) {
+    __shared__ long long warp_sum[8];
+    __shared__ bool last;
+    const int s = blockIdx.x;
+    long long acc = 0;
+    const unsigned long long* k = keys + static_cast<int64_t>(s) * n_tgt;
+    for (int64_t t = threadIdx.x; t < n_tgt; t += blockDim.x) acc += static_cast<long long>(k[t] >> 32);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, o);
+    if ((threadIdx.x & 31) == 0) warp_sum[threadIdx.x >> 5] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        long long tot = 0;
+        for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) tot += warp_sum[w];
+        sums[s] = tot;
+        __threadfence();
+        last = atomicAdd(counter, 1u) == static_cast<unsigned>(n_seg - 1);
+    }
+    __syncthreads();
+    if (!last || threadIdx.x != 0) return;
+    __threadfence();
+    const volatile long long* vs = sums;
+    int32_t b = 0;
+    double b_sim = 0.0;
+    for (int c = 0; c < n_seg; ++c) {
+        const double m = static_cast<double>(vs[c]) / static_cast<double>(n_tgt);
+        double sim = 1.0 - m / max_dist;
+        sim = sim < 0.0 ? 0.0 : (sim > 1.0 ? 1.0 : sim);
+        if (mean_dist) mean_dist[c] = m;
+        if (similarity) similarity[c] = sim;
+        if (c == 0 || sim > b_sim) {
+            b = c;
+            b_sim = sim;
+        }
+    }
+    *best = b;
+    if (applies) *applies = b_sim > threshold ? 1 : 0;
+    *counter = 0u;
 }
 
-extern "C" semshare_status semshare_match_tc(const uint32_t* tgt_codes, int64_t n_tgt, const uint32_t* ref_codes,
-                                             int64_t n_ref, int32_t nbits, int32_t* idx, int32_t* dist,
-                                             void* workspace, size_t workspace_bytes, uint32_t* err_flag,
-                                             void* stream) {
-    using namespace semshare;
-    if (n_tgt < 0 || n_ref < 1) return SEMSHARE_EINVAL;
-    if (nbits < 32 || nbits > 256 || nbits % 32 != 0) return SEMSHARE_EUNSUPPORTED;
-    if (n_tgt >= (int64_t(1) << 31) || n_ref >= (int64_t(1) << 31)) return SEMSHARE_EUNSUPPORTED;
-    if (n_tgt == 0) return SEMSHARE_OK;
-    if (!tgt_codes || !ref_codes || !idx || !workspace) return SEMSHARE_EINVAL;
-    if (!aligned(tgt_codes, 4) || !aligned(ref_codes, 4) || !aligned(idx, 4) || !aligned(workspace, 256) ||
-        (dist && !aligned(dist, 4)) || (err_flag && !aligned(err_flag, 4)))
-        return SEMSHARE_EINVAL;
-    TcPlan plan;
-    plan_tc(n_tgt, n_ref, nbits, &plan);
-    if (workspace_bytes < plan.keys_bytes + plan.t_bytes + plan.r_bytes) return SEMSHARE_EINVAL;
+// idx/dist of every target against the chosen candidate (global reference rows).
+__global__ void retrieve_select_kernel(const unsigned long long* __restrict__ keys, int64_t n_tgt,
+                                       const int32_t* __restrict__ best, int32_t* __restrict__ idx,
+                                       int32_t* __restrict__ dist) {
+    const unsigned long long* k = keys + static_cast<int64_t>(*best) * n_tgt;
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n_tgt;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const unsigned long long v = k[i];
+        if (idx) idx[i] = static_cast<int32_t>(static_cast<uint32_t>(v));
+        if (dist) dist[i] = static_cast<int32_t>(static_cast<uint32_t>(v >> 32));
+    }
+}
 
-    int sms = 0, dev = 0, smem_optin = 0;
-    if (current_sm_count(&sms, &dev) != SEMSHARE_OK) return SEMSHARE_ECUDA;
+// Expand the codes and run the search; leaves keys[n_seg][n_tgt] in the workspace.
+template <int kMaxSeg>
+semshare_status launch_search(const uint32_t* tgt_codes, int64_t n_tgt, const uint32_t* ref_codes, int64_t n_ref,
+                              int32_t nbits, const SegTable<kMaxSeg>& seg, const TcPlan& plan, void* workspace,
+                              uint32_t* err_flag, cudaStream_t s, int sms, int dev) {
+    int smem_optin = 0;
     if (cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
         return SEMSHARE_ECUDA;
-    cudaStream_t s = as_stream(stream);
     auto* keys = static_cast<unsigned long long*>(workspace);
     uint8_t* tpm = static_cast<uint8_t*>(workspace) + plan.keys_bytes;
     uint8_t* rpm = tpm + plan.t_bytes;
-
-    const int64_t pieces = (n_tgt + n_ref) * (plan.kpad / 16);
-    const int64_t eg = (pieces + 255) / 256;
-    expand_codes_kernel<<<static_cast<unsigned>(eg < sms * 8 ? eg : sms * 8), 256, 0, s>>>(
-        tgt_codes, n_tgt, ref_codes, n_ref, nbits, plan.kpad, tpm, rpm, keys);
-    if (launch_status() != SEMSHARE_OK) return SEMSHARE_ECUDA;
+    unsigned int* counter = nullptr;
+    if (plan.sums_bytes > 0)
+        counter = reinterpret_cast<unsigned int*>(rpm + plan.r_bytes + static_cast<size_t>(seg.n_seg) * 8);
 
     TcArgs a{};
     a.n_tgt = n_tgt;
@@ -378,13 +469,119 @@ extern "C" semshare_status semshare_match_tc(const uint32_t* tgt_codes, int64_t 
         !encode_tma_2d(&tm_r, CU_TENSOR_MAP_DATA_TYPE_UINT8, rpm, static_cast<uint64_t>(plan.kpad),
                        static_cast<uint64_t>(n_ref), static_cast<uint64_t>(plan.kpad), kChunk, kTN))
         return SEMSHARE_ECUDA;
-    if (cudaFuncSetAttribute(hamming_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (cudaFuncSetAttribute(hamming_tc_kernel<kMaxSeg>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(smem)) != cudaSuccess)
         return SEMSHARE_ECUDA;
-    const int64_t grid = a.total < sms ? a.total : sms;
-    hamming_tc_kernel<<<static_cast<unsigned>(grid), kThreads, smem, s>>>(tm_t, tm_r, a);
+
+    const int64_t pieces = (n_tgt + n_ref) * (plan.kpad / 16);
+    const int64_t eg = (pieces + 255) / 256;
+    expand_codes_kernel<<<static_cast<unsigned>(eg < sms * 8 ? eg : sms * 8), 256, 0, s>>>(
+        tgt_codes, n_tgt, ref_codes, n_ref, nbits, plan.kpad, tpm, rpm, keys, n_tgt * seg.n_seg, counter);
     if (launch_status() != SEMSHARE_OK) return SEMSHARE_ECUDA;
-    const int small = static_cast<int>((n_tgt + 255) / 256 < sms * 4 ? (n_tgt + 255) / 256 : sms * 4);
-    tc_keys_split_kernel<<<small, 256, 0, s>>>(keys, n_tgt, idx, dist);
+    const int64_t grid = a.total < sms ? a.total : sms;
+    hamming_tc_kernel<kMaxSeg><<<static_cast<unsigned>(grid), kThreads, smem, s>>>(tm_t, tm_r, a, seg);
     return launch_status();
+}
+
+}  // namespace
+}  // namespace semshare
+
+extern "C" size_t semshare_match_tc_workspace_size(int64_t n_tgt, int64_t n_ref, int32_t nbits) {
+    using namespace semshare;
+    if (n_tgt <= 0 || n_ref <= 0 || nbits < 32 || nbits > 256 || nbits % 32 != 0) return 0;
+    TcPlan p;
+    plan_tc(n_tgt, n_ref, nbits, 0, &p);
+    return p.total();
+}
+
+extern "C" semshare_status semshare_match_tc(const uint32_t* tgt_codes, int64_t n_tgt, const uint32_t* ref_codes,
+                                             int64_t n_ref, int32_t nbits, int32_t* idx, int32_t* dist,
+                                             void* workspace, size_t workspace_bytes, uint32_t* err_flag,
+                                             void* stream) {
+    using namespace semshare;
+    if (n_tgt < 0 || n_ref < 1) return SEMSHARE_EINVAL;
+    if (nbits < 32 || nbits > 256 || nbits % 32 != 0) return SEMSHARE_EUNSUPPORTED;
+    if (n_tgt >= (int64_t(1) << 31) || n_ref >= (int64_t(1) << 31)) return SEMSHARE_EUNSUPPORTED;
+    if (n_tgt == 0) return SEMSHARE_OK;
+    if (!tgt_codes || !ref_codes || !idx || !workspace) return SEMSHARE_EINVAL;
+    if (!aligned(tgt_codes, 4) || !aligned(ref_codes, 4) || !aligned(idx, 4) || !aligned(workspace, 256) ||
+        (dist && !aligned(dist, 4)) || (err_flag && !aligned(err_flag, 4)))
+        return SEMSHARE_EINVAL;
+    TcPlan plan;
+    plan_tc(n_tgt, n_ref, nbits, 0, &plan);
+    if (workspace_bytes < plan.total()) return SEMSHARE_EINVAL;
+
+    int sms = 0, dev = 0;
+    if (current_sm_count(&sms, &dev) != SEMSHARE_OK) return SEMSHARE_ECUDA;
+    cudaStream_t s = as_stream(stream);
+    SegTable<1> seg{};
+    seg.n_seg = 1;
+    seg.off[0] = 0;
+    seg.off[1] = n_ref;
+    const semshare_status st = launch_search(tgt_codes, n_tgt, ref_codes, n_ref, nbits, seg, plan, workspace,
+                                             err_flag, s, sms, dev);
+    if (st != SEMSHARE_OK) return st;
+    const int small = static_cast<int>((n_tgt + 255) / 256 < sms * 4 ? (n_tgt + 255) / 256 : sms * 4);
+    tc_keys_split_kernel<<<small, 256, 0, s>>>(static_cast<const unsigned long long*>(workspace), n_tgt, idx, dist);
+    return launch_status();
+}
+
+extern "C" size_t semshare_retrieve_workspace_size(int64_t n_tgt, int64_t n_pool, int32_t n_cand, int32_t nbits) {
+    using namespace semshare;
+    if (n_tgt <= 0 || n_pool <= 0 || n_cand < 1 || n_cand > SEMSHARE_RETRIEVE_MAX_CANDIDATES || nbits < 32 ||
+        nbits > 256 || nbits % 32 != 0)
+        return 0;
+    TcPlan p;
+    plan_tc(n_tgt, n_pool, nbits, n_cand, &p);
+    return p.total();
+}
+
+extern "C" semshare_status semshare_retrieve(const uint32_t* tgt_codes, int64_t n_tgt, const uint32_t* pool_codes,
+                                             const int64_t* cand_offsets, int32_t n_cand, int32_t nbits,
+                                             double max_dist, double threshold, double* mean_dist,
+                                             double* similarity, int32_t* best, int32_t* applies, int32_t* idx,
+                                             int32_t* dist, void* workspace, size_t workspace_bytes,
+                                             uint32_t* err_flag, void* stream) {
+    using namespace semshare;
+    if (n_cand < 1 || !cand_offsets || n_tgt < 1) return SEMSHARE_EINVAL;
+    if (n_cand > SEMSHARE_RETRIEVE_MAX_CANDIDATES) return SEMSHARE_EUNSUPPORTED;
+    if (nbits < 32 || nbits > 256 || nbits % 32 != 0) return SEMSHARE_EUNSUPPORTED;
+    if (!(max_dist > 0.0) || !(max_dist <= 1.0e300) || threshold != threshold) return SEMSHARE_EINVAL;
+    if (cand_offsets[0] != 0) return SEMSHARE_EINVAL;
+    for (int32_t c = 0; c < n_cand; ++c)
+        if (cand_offsets[c + 1] <= cand_offsets[c]) return SEMSHARE_EINVAL;
+    const int64_t n_pool = cand_offsets[n_cand];
+    if (n_tgt >= (int64_t(1) << 31) || n_pool >= (int64_t(1) << 31)) return SEMSHARE_EUNSUPPORTED;
+    if (!tgt_codes || !pool_codes || !best || !workspace) return SEMSHARE_EINVAL;
+    if (!aligned(tgt_codes, 4) || !aligned(pool_codes, 4) || !aligned(best, 4) || !aligned(workspace, 256) ||
+        (applies && !aligned(applies, 4)) || (mean_dist && !aligned(mean_dist, 8)) ||
+        (similarity && !aligned(similarity, 8)) || (idx && !aligned(idx, 4)) || (dist && !aligned(dist, 4)) ||
+        (err_flag && !aligned(err_flag, 4)))
+        return SEMSHARE_EINVAL;
+    TcPlan plan;
+    plan_tc(n_tgt, n_pool, nbits, n_cand, &plan);
+    if (workspace_bytes < plan.total()) return SEMSHARE_EINVAL;
+
+    int sms = 0, dev = 0;
+    if (current_sm_count(&sms, &dev) != SEMSHARE_OK) return SEMSHARE_ECUDA;
+    cudaStream_t s = as_stream(stream);
+    SegTable<SEMSHARE_RETRIEVE_MAX_CANDIDATES> seg{};
+    seg.n_seg = n_cand;
+    for (int32_t c = 0; c <= n_cand; ++c) seg.off[c] = cand_offsets[c];
+    semshare_status st = launch_search(tgt_codes, n_tgt, pool_codes, n_pool, nbits, seg, plan, workspace, err_flag,
+                                       s, sms, dev);
+    if (st != SEMSHARE_OK) return st;
+    auto* keys = static_cast<const unsigned long long*>(workspace);
+    auto* sums = reinterpret_cast<long long*>(static_cast<uint8_t*>(workspace) + plan.keys_bytes + plan.t_bytes +
+                                              plan.r_bytes);
+    auto* counter = reinterpret_cast<unsigned int*>(sums + n_cand);
+    retrieve_finalize_kernel<<<n_cand, 256, 0, s>>>(keys, n_tgt, n_cand, max_dist, threshold, sums, counter,
+                                                    mean_dist, similarity, best, applies);
+    if (launch_status() != SEMSHARE_OK) return SEMSHARE_ECUDA;
+    if (idx || dist) {
+        const int small = static_cast<int>((n_tgt + 255) / 256 < sms * 4 ? (n_tgt + 255) / 256 : sms * 4);
+        retrieve_select_kernel<<<small, 256, 0, s>>>(keys, n_tgt, best, idx, dist);
+        st = launch_status();
+    }
+    return st;
 }

@@ -102,6 +102,30 @@ def test_gather_argument_errors(lib):
     assert g(pk, pk, offs, 1, lay, None, 0, 1, None, None, out, None, None) == 0        # empty
 
 
+def test_retrieve_argument_errors(lib):
+    r = lib.semshare_retrieve
+
+    def call(offs, n_cand=None, n_tgt=10, nbits=64, max_dist=30.0, thr=0.8, best=FAKE, ws_bytes=1 << 30):
+        o = (ctypes.c_int64 * len(offs))(*offs)
+        n_cand = len(offs) - 1 if n_cand is None else n_cand
+        return r(FAKE, n_tgt, FAKE, o, n_cand, nbits, max_dist, thr, None, None, best, None, None, None, FAKE,
+                 ws_bytes, None, None)
+
+    assert call([0]) == 1                              # no candidate
+    assert call([0, 5, 5, 9]) == 1                     # empty candidate
+    assert call([1, 5]) == 1                           # does not start at row 0
+    assert call([0, 5, 3]) == 1                        # decreasing
+    assert call(list(range(258))) == 2                 # 257 candidates: above the maximum
+    assert call([0, 5], nbits=40) == 2
+    assert call([0, 5], n_tgt=0) == 1                  # the mean over no target token
+    assert call([0, 5], max_dist=0.0) == 1
+    assert call([0, 5], thr=float("nan")) == 1
+    assert call([0, 5], best=None) == 1
+    assert call([0, 5], ws_bytes=100) == 1             # workspace too small
+    assert lib.semshare_retrieve_workspace_size(10, 5, 0, 64) == 0
+    assert lib.semshare_retrieve_workspace_size(10, 5, 1, 64) > lib.semshare_match_tc_workspace_size(10, 5, 64)
+
+
 def test_rope_table_argument_errors(lib):
     t = lib.semshare_rope_table
     assert t(7, 10000.0, FAKE, None) == 1

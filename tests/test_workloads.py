@@ -61,3 +61,14 @@ def test_kv_cache_segments():
     assert k.shape == (1, 2, 4, 256, 64) and k.dtype == np.uint16
     k0, _ = workloads.kv_cache(wl, segment=0)
     np.testing.assert_array_equal(k0, k[0])
+
+
+def test_retrieve_recipe_rewrites_one_member():
+    wl = workloads.RETRIEVAL_WORKLOADS["retrieve-16x4096"].scaled(d=64)
+    m = workloads.retrieval_member(wl)
+    _, _, src = workloads.target_prompt(wl)
+    copied = np.nonzero(src >= 0)[0]
+    # copied rows come from the one member, in order, at their own position
+    np.testing.assert_array_equal(src[copied], m * wl.seg_len + copied)
+    assert abs(len(copied) / wl.n_tgt - wl.reuse) < 1e-3
+    assert 0 <= m < wl.n_seg

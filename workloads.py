@@ -58,7 +58,9 @@ class Workload:
     noise     standard deviation of the Gaussian noise added to copied rows
     recipe    how copied rows are placed: 'perm' (global random permutation),
               'window' (local shuffle of +-window positions), 'subset' (sorted random
-              subset, order kept), 'pool' (uniform pool member and row)
+              subset, order kept), 'pool' (uniform pool member and row),
+              'retrieve' (the rows of one pool member in order: the target is a rewrite of
+              one stored prompt, the reference retrieval case of Sec. 3.2 and Sec. 4.4)
     """
     name: str
     n_ref: int
@@ -113,6 +115,21 @@ WORKLOADS = {
                              base_seed=0x5E4D5AE0 + 4),
 }
 
+# Reference retrieval (Sec. 3.2): 16 stored prompts of 4096 tokens, and a target that is one of
+# them with 3% of its rows replaced and light noise on the rest (the replace study of Sec. 4.4);
+# its retrieval codes are taken without rotary encoding (retrieval precedes it in Sec. 3.2).
+RETRIEVAL_WORKLOADS = {
+    "retrieve-16x4096": Workload("retrieve-16x4096", n_ref=65536, n_seg=16, n_tgt=4096, d=4096, emb_dtype="bf16",
+                                 nbits=256, kv=(32, 8, 128), reuse=0.97, noise=0.02, recipe="retrieve",
+                                 base_seed=0x5E4D5AE0 + 5),
+}
+
+
+def retrieval_member(wl: Workload, seed: int | None = None, b: int = 0) -> int:
+    """The pool member target prompt `b` of a 'retrieve' workload was rewritten from."""
+    seed = wl.base_seed if seed is None else seed
+    return int(rng(seed, _S_POOL, b).integers(0, wl.n_seg))
+
 
 def _emb_out(x: np.ndarray, emb_dtype: str) -> np.ndarray:
     return x.astype(np.float32) if emb_dtype == "f32" else f32_to_bf16_bits(x)
@@ -146,6 +163,10 @@ def _source_rows(wl: Workload, seed: int, b: int) -> np.ndarray:
         src = np.argsort(key, kind="stable").astype(np.int64) % wl.n_ref
     elif wl.recipe == "subset":
         src = np.sort(g.choice(wl.n_ref, size=n, replace=False)).astype(np.int64)
+    elif wl.recipe == "retrieve":
+        if n > wl.seg_len:
+            raise ValueError("a rewritten prompt is at most one member long")
+        src = (retrieval_member(wl, seed, b) * wl.seg_len + np.arange(n)).astype(np.int64)
     elif wl.recipe == "pool":
         member = g.integers(0, wl.n_seg, size=n)
         row = g.integers(0, wl.seg_len, size=n)
