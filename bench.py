@@ -47,13 +47,16 @@ ALL_WORKLOADS = {**workloads.WORKLOADS, **workloads.RETRIEVAL_WORKLOADS}
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 L2_FLUSH_BYTES = 256 << 20
 
-# DRAM bytes per launch from ncu captures (dram__bytes_read.sum + dram__bytes_write.sum),
-# valid only while the kernel source has the recorded sha256 prefix.
+# DRAM bytes per launch from ncu captures (dram__bytes_read.sum + dram__bytes_write.sum) on a
+# workload, valid only for that workload and while the kernel source has the recorded sha256
+# prefix (the traffic depends on the index pattern, e.g. how often a gathered row repeats).
 NCU_TRAFFIC = {
-    "gather": {"file": "gather.cu", "sha": "e03583daf19419cb", "bytes_per_launch": 1092.8e6, "targets": 5120},
-    "hash": {"file": "hash.cu", "sha": "7cf51b07f7d5874d", "bytes_per_launch": 92.63e6, "targets": 5120},
-    "match": {"file": "match.cu", "sha": "69ac4b7ce5b193e4", "bytes_per_launch": 0.3845e6, "targets": 5120},
-    "match_tc": {"file": "match_tc.cu", "sha": "3bcc238fb9cfe314", "bytes_per_launch": 2.712e6, "targets": 5120},
+    ("gather", "llama8b-5k"): {"file": "gather.cu", "sha": "e03583daf19419cb", "bytes_per_launch": 1092.8e6},
+    ("gather", "retrieve-16x4096"): {"file": "gather.cu", "sha": "e03583daf19419cb", "bytes_per_launch": 1000.5e6},
+    ("hash", "llama8b-5k"): {"file": "hash.cu", "sha": "0fc6e508c36def23", "bytes_per_launch": 90.65e6},
+    ("match", "llama8b-5k"): {"file": "match.cu", "sha": "69ac4b7ce5b193e4", "bytes_per_launch": 0.3845e6},
+    ("match_tc", "llama8b-5k"): {"file": "match_tc.cu", "sha": "c494ec8dce435f1b", "bytes_per_launch": 2.736e6},
+    ("retrieve", "retrieve-16x4096"): {"file": "match_tc.cu", "sha": "c494ec8dce435f1b", "bytes_per_launch": 18.42e6},
 }
 
 
@@ -494,23 +497,23 @@ def stage_report(wl, W, stage_ms, peaks, popc_peak, matcher):
     return out
 
 
-def roofline_for(dominant, stages, peaks, matcher):
+def roofline_for(dominant, stages, peaks, matcher, workload):
     if dominant == "gather":
         return {"kernel": "kv_gather_kernel", "bound": "hbm", "achieved": stages["gather"]["gbs"],
-                "peak": peaks["hbm_gbs"], "unit": "GB/s"}, NCU_TRAFFIC.get("gather")
+                "peak": peaks["hbm_gbs"], "unit": "GB/s"}, NCU_TRAFFIC.get(("gather", workload))
     if dominant in ("hash", "hash_plain"):
         return {"kernel": "lsh_hash_kernel", "bound": "tensor", "achieved": stages[dominant]["tflops"],
-                "peak": peaks["bf16_tflops"], "unit": "TFLOP/s"}, NCU_TRAFFIC.get("hash")
+                "peak": peaks["bf16_tflops"], "unit": "TFLOP/s"}, NCU_TRAFFIC.get(("hash", workload))
     if dominant == "retrieve":
         return {"kernel": "hamming_tc_kernel<256> (segmented)", "bound": "tensor",
                 "achieved": stages["retrieve"]["tflops_fp8"], "peak": 2.0 * peaks["bf16_tflops"],
-                "unit": "TFLOP/s"}, NCU_TRAFFIC.get("retrieve")
+                "unit": "TFLOP/s"}, NCU_TRAFFIC.get(("retrieve", workload))
     if matcher == "popc":
         return {"kernel": "hamming_nn_kernel", "bound": "alu", "achieved": stages["match"]["gwordops"],
                 "peak": stages["match"]["gwordops"] / stages["match"]["frac_popc"], "unit": "Gwordop/s"}, \
-            NCU_TRAFFIC.get("match")
+            NCU_TRAFFIC.get(("match", workload))
     return {"kernel": "hamming_tc_kernel", "bound": "tensor", "achieved": stages["match"]["tflops_fp8"],
-            "peak": 2.0 * peaks["bf16_tflops"], "unit": "TFLOP/s"}, NCU_TRAFFIC.get("match_tc")
+            "peak": 2.0 * peaks["bf16_tflops"], "unit": "TFLOP/s"}, NCU_TRAFFIC.get(("match_tc", workload))
 
 
 def run_gpu_arm(args, rank, world, local_rank):
@@ -569,13 +572,10 @@ def run_gpu_arm(args, rank, world, local_rank):
     stages = stage_report(wl, W, stage_ms, peaks, popc_peak, args.matcher)
 
     dominant = max(stage_ms, key=stage_ms.get)
-    roof, tr = roofline_for(dominant, stages, peaks, args.matcher)
+    roof, tr = roofline_for(dominant, stages, peaks, args.matcher, wl.name)
     roof["frac"] = roof["achieved"] / roof["peak"]
     roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"
-    if tr and tr.get("sha") == kernel_sha(tr["file"]):
-        roof["traffic"] = tr["bytes_per_launch"] * (W["targets"] / tr["targets"])
-    else:
-        roof["traffic"] = None
+    roof["traffic"] = tr["bytes_per_launch"] if tr and tr.get("sha") == kernel_sha(tr["file"]) else None
 
     e2e = run_e2e(args, prob, device)
 

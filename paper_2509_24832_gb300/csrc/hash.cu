@@ -469,7 +469,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (qq < W) {
                         uint32_t v[32];
                         tmem_load_32cols(taddr + qq * 32, v);
-                        tmem_load_wait();
+                        tmem_load_wait_fence(v);
                         words[qq] = sign_word(v);
                         if (a.proj != nullptr && row < a.n) store_proj(a.proj, row, a.nbits, qq, v);
                     }
@@ -488,7 +488,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (qq < W) {
                         uint32_t v[32];
                         tmem_load_32cols(taddr + qq * 32, v);
-                        tmem_load_wait();
+                        tmem_load_wait_fence(v);
 #pragma unroll
                         for (int j = 0; j < 8; ++j)
                             dst[(qq * 8 + j) * kBM + r] =

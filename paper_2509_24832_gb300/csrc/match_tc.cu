@@ -306,16 +306,28 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int valid = rem < kTN ? static_cast<int>(rem) : kTN;
             const uint32_t taddr = tmem_base + (static_cast<uint32_t>(ew * 32) << 16) + buf * kTN;
             float bk = -3.0e38f;  // best key 256*dot - j of this tile (current candidate)
+            // 32-column chunks, double-buffered: the load of chunk q+1 is in flight while chunk
+            // q is reduced
+            uint32_t va[32], vb[32];
+            tmem_load_32cols(taddr, va);
+            tmem_load_wait_fence(va);
 #pragma unroll
             for (int q = 0; q < kTN / 32; ++q) {
-                uint32_t v[32];
-                tmem_load_32cols(taddr + q * 32, v);
-                tmem_load_wait();
+                uint32_t(&v)[32] = (q & 1) ? vb : va;
+                uint32_t(&vn)[32] = (q & 1) ? va : vb;
+                if (q + 1 < kTN / 32) tmem_load_32cols(taddr + (q + 1) * 32, vn);
                 const int64_t c0 = col0 + q * 32;
                 if (q * 32 + 32 <= valid && c0 + 32 <= next_b) {
+                    // four independent max chains (the keys are distinct: order does not matter)
+                    float m0 = -3.0e38f, m1 = -3.0e38f, m2 = -3.0e38f, m3 = -3.0e38f;
 #pragma unroll
-                    for (int j = 0; j < 32; ++j)
-                        bk = fmaxf(bk, fmaf(__uint_as_float(v[j]), 256.0f, -static_cast<float>(q * 32 + j)));
+                    for (int j = 0; j < 32; j += 4) {
+                        m0 = fmaxf(m0, fmaf(__uint_as_float(v[j]), 256.0f, -static_cast<float>(q * 32 + j)));
+                        m1 = fmaxf(m1, fmaf(__uint_as_float(v[j + 1]), 256.0f, -static_cast<float>(q * 32 + j + 1)));
+                        m2 = fmaxf(m2, fmaf(__uint_as_float(v[j + 2]), 256.0f, -static_cast<float>(q * 32 + j + 2)));
+                        m3 = fmaxf(m3, fmaf(__uint_as_float(v[j + 3]), 256.0f, -static_cast<float>(q * 32 + j + 3)));
+                    }
+                    bk = fmaxf(bk, fmaxf(fmaxf(m0, m1), fmaxf(m2, m3)));
                 } else if (q * 32 < valid) {
                     // ragged end and/or candidate boundaries inside the chunk: runs [js, je)
                     const int jend = valid - q * 32 < 32 ? valid - q * 32 : 32;
@@ -337,6 +349,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         js = je;
                     }
                 }
+                if (q + 1 < kTN / 32) tmem_load_wait_fence(vn);
             }
             tc_fence_before_sync();
             __syncwarp();
@@ -399,25 +412,41 @@ __global__ void __launch_bounds__(256)
         last = atomicAdd(counter, 1u) == static_cast<unsigned>(n_seg - 1);
     }
     __syncthreads();
-    if (!last || threadIdx.x != 0) return;
+    if (!last) return;
+    // the last block: thread c handles candidate c (fp64 is slow on this part: run the
+    // divisions side by side), then a tree arg-max over (similarity, lowest index)
+    __shared__ double red_sim[256];
+    __shared__ int red_idx[256];
     __threadfence();
     const volatile long long* vs = sums;
-    int32_t b = 0;
-    double b_sim = 0.0;
-    for (int c = 0; c < n_seg; ++c) {
+    const int c = threadIdx.x;
+    double sim = -1.0;
+    if (c < n_seg) {
         const double m = static_cast<double>(vs[c]) / static_cast<double>(n_tgt);
-        double sim = 1.0 - m / max_dist;
+        sim = 1.0 - m / max_dist;
         sim = sim < 0.0 ? 0.0 : (sim > 1.0 ? 1.0 : sim);
         if (mean_dist) mean_dist[c] = m;
         if (similarity) similarity[c] = sim;
-        if (c == 0 || sim > b_sim) {
-            b = c;
-            b_sim = sim;
-        }
     }
-    *best = b;
-    if (applies) *applies = b_sim > threshold ? 1 : 0;
-    *counter = 0u;
+    red_sim[c] = sim;
+    red_idx[c] = c;
+    __syncthreads();
+    for (int o = 128; o > 0; o >>= 1) {
+        if (c < o) {
+            const double s2 = red_sim[c + o];
+            const int i2 = red_idx[c + o];
+            if (s2 > red_sim[c] || (s2 == red_sim[c] && i2 < red_idx[c])) {
+                red_sim[c] = s2;
+                red_idx[c] = i2;
+            }
+        }
+        __syncthreads();
+    }
+    if (c == 0) {
+        *best = red_idx[0];
+        if (applies) *applies = red_sim[0] > threshold ? 1 : 0;
+        *counter = 0u;
+    }
 }
 
 // idx/dist of every target against the chosen candidate (global reference rows).

@@ -180,6 +180,20 @@ __device__ __forceinline__ void tmem_load_32cols(uint32_t taddr, uint32_t (&v)[3
 
 __device__ __forceinline__ void tmem_load_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 
+// tcgen05.wait::ld that also marks the 32 destination registers of an earlier tmem_load_32cols
+// as written here, so the compiler cannot move their uses above the wait (the load's asm
+// statement hands the registers back before the data has arrived).
+__device__ __forceinline__ void tmem_load_wait_fence(uint32_t (&v)[32]) {
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(v[0]), "+r"(v[1]), "+r"(v[2]), "+r"(v[3]), "+r"(v[4]), "+r"(v[5]), "+r"(v[6]), "+r"(v[7]),
+                   "+r"(v[8]), "+r"(v[9]), "+r"(v[10]), "+r"(v[11]), "+r"(v[12]), "+r"(v[13]), "+r"(v[14]),
+                   "+r"(v[15]), "+r"(v[16]), "+r"(v[17]), "+r"(v[18]), "+r"(v[19]), "+r"(v[20]), "+r"(v[21]),
+                   "+r"(v[22]), "+r"(v[23]), "+r"(v[24]), "+r"(v[25]), "+r"(v[26]), "+r"(v[27]), "+r"(v[28]),
+                   "+r"(v[29]), "+r"(v[30]), "+r"(v[31])
+                 :
+                 : "memory");
+}
+
 // Shared-memory matrix descriptor of a K-major operand tile stored with the 128-byte
 // swizzle: rows of 128 bytes, 8-row groups 1024 bytes apart (the layout TMA writes with
 // CU_TENSOR_MAP_SWIZZLE_128B).  The tile must start on a 1024-byte boundary; steps along K

@@ -1,10 +1,14 @@
 """Runs one library call on a workload's synthetic inputs, a few times, for profilers.
 
-    python -m paper_2509_24832_gb300.kernel_runner --kernel hash|match|gather --workload NAME [--reps N]
+    python -m paper_2509_24832_gb300.kernel_runner --kernel hash|match|match_tc|gather|retrieve
+        --workload NAME [--reps N]
 
 Only the buffers that call needs are allocated (e.g. the 5k-token hash holds ~100 MB, the
 5k-token gather ~1.4 GB), which keeps a profiler's capture small.  Inputs come from workloads.py;
-the match and gather run on the codes and indices the library computes for that workload."""
+the match and gather run on the codes and indices the library computes for that workload.  On
+a retrieval workload the calls follow the retrieval step: `retrieve` searches the plain codes of
+the stored prompts, `match_tc` matches the target against the winner's rotary codes and
+`gather` moves the winner's K/V rows (only the winner's cache is allocated)."""
 from __future__ import annotations
 
 import argparse
@@ -22,15 +26,50 @@ import workloads  # noqa: E402
 
 import paper_2509_24832_gb300 as ss  # noqa: E402
 
+ALL = {**workloads.WORKLOADS, **workloads.RETRIEVAL_WORKLOADS}
+
+
+def _retrieval(a, wl, e, pd, R, table, flag, dev):
+    n_pool = wl.n_ref
+    offs = [m * wl.seg_len for m in range(wl.n_seg + 1)]
+    zeros = torch.zeros(e.shape[0], dtype=torch.int32, device=dev)
+    plain = ss.semshare_hash(e, table, R, zeros, err_flag=flag)
+    ws = torch.empty(ss.semshare_retrieve_workspace_size(wl.n_tgt, n_pool, wl.n_seg, wl.nbits), dtype=torch.uint8,
+                     device=dev)
+    reps = a.reps if a.kernel == "retrieve" else 1
+    for _ in range(reps):
+        res = ss.semshare_retrieve(plain[n_pool:], plain[:n_pool], offs, workspace=ws, err_flag=flag,
+                                   want_match=False)
+    if a.kernel == "retrieve":
+        return
+    m = int(res.best.item())
+    codes = ss.semshare_hash(e, table, R, pd, err_flag=flag)
+    del plain, zeros
+    tc, rc = codes[n_pool:], codes[offs[m]:offs[m + 1]]
+    idx = torch.empty(wl.n_tgt, dtype=torch.int32, device=dev)
+    dist = torch.empty_like(idx)
+    reps = a.reps if a.kernel == "match_tc" else 1
+    for _ in range(reps):
+        ss.semshare_match_tc(tc, rc, idx=idx, dist=dist, err_flag=flag)
+    if a.kernel != "gather":
+        return
+    del e, codes
+    k, v = workloads.kv_cache_device(wl, dev, segment=m)
+    L, H, hd = wl.kv
+    out_k = torch.empty((1, L, H, wl.n_tgt, hd), dtype=torch.bfloat16, device=dev)
+    out_v = torch.empty_like(out_k)
+    for _ in range(a.reps):
+        ss.semshare_gather_kv([k], [v], idx.view(1, wl.n_tgt), out_k=out_k, out_v=out_v, err_flag=flag)
+
 
 def main(argv=None):
     p = argparse.ArgumentParser()
-    p.add_argument("--kernel", choices=["hash", "match", "match_tc", "gather"], required=True)
-    p.add_argument("--workload", default="llama8b-5k", choices=sorted(workloads.WORKLOADS))
+    p.add_argument("--kernel", choices=["hash", "match", "match_tc", "gather", "retrieve"], required=True)
+    p.add_argument("--workload", default="llama8b-5k", choices=sorted(ALL))
     p.add_argument("--reps", type=int, default=3)
     a = p.parse_args(argv)
     dev = torch.device("cuda")
-    wl = workloads.WORKLOADS[a.workload]
+    wl = ALL[a.workload]
     emb, pos, _ = workloads.prompt_rows(wl)
     e = torch.from_numpy(emb).to(dev) if emb.dtype == np.float32 else \
         torch.from_numpy(emb.view(np.int16)).to(dev).view(torch.bfloat16)
@@ -38,28 +77,35 @@ def main(argv=None):
     R = torch.from_numpy(workloads.hyperplanes(wl).view(np.int16)).to(dev).view(torch.bfloat16)
     table = ss.semshare_rope_table(wl.d, 10000.0, device=dev)
     flag = ss.new_err_flag(dev)
-    codes = ss.semshare_hash(e, table, R, pd, err_flag=flag)
-    if a.kernel == "hash":
-        for _ in range(a.reps):
-            ss.semshare_hash(e, table, R, pd, codes=codes, err_flag=flag)
+    if wl.recipe == "retrieve":
+        if a.kernel not in ("retrieve", "match_tc", "gather"):
+            raise SystemExit("a retrieval workload runs retrieve, match_tc or gather")
+        _retrieval(a, wl, e, pd, R, table, flag, dev)
+    elif a.kernel == "retrieve":
+        raise SystemExit("retrieve needs a retrieval workload")
     else:
-        tc, rc = codes[wl.n_ref:], codes[: wl.n_ref]
-        idx, dist = ss.semshare_match(tc, rc)
-        if a.kernel == "match":
+        codes = ss.semshare_hash(e, table, R, pd, err_flag=flag)
+        if a.kernel == "hash":
             for _ in range(a.reps):
-                ss.semshare_match(tc, rc, idx=idx, dist=dist)
-        elif a.kernel == "match_tc":
-            for _ in range(a.reps):
-                ss.semshare_match_tc(tc, rc, idx=idx, dist=dist, err_flag=flag)
+                ss.semshare_hash(e, table, R, pd, codes=codes, err_flag=flag)
         else:
-            del e
-            segs = [workloads.kv_cache_device(wl, dev, segment=s) for s in range(wl.n_seg)]
-            L, H, hd = wl.kv
-            out_k = torch.empty((wl.n_batch, L, H, wl.n_tgt, hd), dtype=torch.bfloat16, device=dev)
-            out_v = torch.empty_like(out_k)
-            for _ in range(a.reps):
-                ss.semshare_gather_kv([s[0] for s in segs], [s[1] for s in segs], idx.view(wl.n_batch, wl.n_tgt),
-                                      out_k=out_k, out_v=out_v, err_flag=flag)
+            tc, rc = codes[wl.n_ref:], codes[: wl.n_ref]
+            idx, dist = ss.semshare_match(tc, rc)
+            if a.kernel == "match":
+                for _ in range(a.reps):
+                    ss.semshare_match(tc, rc, idx=idx, dist=dist)
+            elif a.kernel == "match_tc":
+                for _ in range(a.reps):
+                    ss.semshare_match_tc(tc, rc, idx=idx, dist=dist, err_flag=flag)
+            else:
+                del e
+                segs = [workloads.kv_cache_device(wl, dev, segment=s) for s in range(wl.n_seg)]
+                L, H, hd = wl.kv
+                out_k = torch.empty((wl.n_batch, L, H, wl.n_tgt, hd), dtype=torch.bfloat16, device=dev)
+                out_v = torch.empty_like(out_k)
+                for _ in range(a.reps):
+                    ss.semshare_gather_kv([s[0] for s in segs], [s[1] for s in segs],
+                                          idx.view(wl.n_batch, wl.n_tgt), out_k=out_k, out_v=out_v, err_flag=flag)
     torch.cuda.synchronize()
     ss.check_flag(flag, a.kernel)
     print(f"{a.kernel} on {wl.name}: {a.reps} launches ok")
