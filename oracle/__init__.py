@@ -12,6 +12,8 @@ it follows, is stated in `semshare_oracle.c`:
   gather  reordered K/V rows, bitwise copies; Sec. 3.3, Sec. 3.3.2
   retrieve  LSH-distance similarity of whole prompts and the best candidate; Sec. 3.2,
           App. A.3, Sec. 4.4
+  kv_deviation  sigma_K + sigma_V per layer and token; App. A.4
+  select_hd     the k highest-deviation tokens per layer; Insight 1, Sec. 3.2
 
 Parity pins: every function here is pinned by `tests/test_oracle_*.py` against closed forms,
 invariants, hand-derived golden cases and brute force (none is "parity unpinned").
@@ -68,6 +70,8 @@ def _load():
         lib.oracle_gather_kv.argtypes = [P, P, P, i32, i32, i32, i64, P, i64, i32, P, P]
         lib.oracle_gather_kv.restype = i64
         lib.oracle_retrieve.argtypes = [P, i64, P, P, i32, i32, f64, f64, P, P, P, P]
+        lib.oracle_kv_deviation.argtypes = [P, P, P, P, i32, i32, i32, i64, i32, P, P, P]
+        lib.oracle_select_hd.argtypes = [P, i32, i64, i64, P]
         _lib = lib
         return lib
 
@@ -202,3 +206,31 @@ def retrieve(tgt_codes: np.ndarray, pool_codes: np.ndarray, seg_offsets, nbits: 
     _load().oracle_retrieve(_ptr(t), t.shape[0], _ptr(p), _ptr(offs), n_seg, nbits, float(max_dist), float(threshold),
                             _ptr(mean), _ptr(sim), _ptr(best), _ptr(applies))
     return mean, sim, int(best[0]), bool(applies[0])
+
+
+def kv_deviation(k_re, v_re, k_rc, v_rc):
+    """Key-Value deviation (App. A.4) of [L][H][T][hd] arrays (bf16 bit patterns as uint16, or
+    float32): returns (sigma_k, sigma_v, sigma_kv), each [L][T] float64."""
+    arrs = [np.ascontiguousarray(a) for a in (k_re, v_re, k_rc, v_rc)]
+    dt = arrs[0].dtype
+    if dt not in (np.uint16, np.float32) or any(a.dtype != dt or a.shape != arrs[0].shape for a in arrs):
+        raise ValueError("four [L][H][T][hd] arrays of one dtype (uint16 bf16 bits or float32)")
+    L, H, T, hd = arrs[0].shape
+    sk = np.zeros((L, T))
+    sv = np.zeros((L, T))
+    skv = np.zeros((L, T))
+    _load().oracle_kv_deviation(*[_ptr(a) for a in arrs], 1 if dt == np.float32 else 0, L, H, T, hd, _ptr(sk),
+                                _ptr(sv), _ptr(skv))
+    return sk, sv, skv
+
+
+def select_hd(sigma, k: int):
+    """The k highest-deviation tokens of every layer (ties to the lower index), ascending:
+    sigma [L][T] (any float type; taken as float64) -> int32 [L][k]."""
+    s = np.ascontiguousarray(np.atleast_2d(np.asarray(sigma, dtype=np.float64)))
+    L, T = s.shape
+    if not 0 <= k <= T:
+        raise ValueError("k outside [0, T]")
+    out = np.zeros((L, k), dtype=np.int32)
+    _load().oracle_select_hd(_ptr(s), L, T, int(k), _ptr(out))
+    return out

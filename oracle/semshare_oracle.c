@@ -29,6 +29,10 @@
  *              prompt's LSH distance to the target -- read as the mean over target tokens of the
  *              nearest Hamming distance -- is normalised by 30 and turned into a similarity in
  *              [0, 1]; the most similar candidate wins and is reused if above 0.8.
+ *   6. kv_deviation / select_hd  Key-Value deviation (App. A.4): per layer and token,
+ *              ||K_reused - K_recomputed||_2 + ||V_reused - V_recomputed||_2 over all heads; the
+ *              tokens of highest deviation (40% in the paper, Insight 1) are the HD tokens that
+ *              the first layer's comparison hands to recomputation (Sec. 3.2).
  *
  * Build: gcc -O2 -fopenmp -ffp-contract=off -shared -fPIC (no fused multiply-add, so x86 and
  * Arm hosts produce the same bits).
@@ -244,4 +248,64 @@ void oracle_retrieve(const uint32_t* tgt, int64_t n_tgt, const uint32_t* pool, c
         if (similarity[s] > similarity[b]) b = s;
     *best = b;
     *applies = similarity[b] > threshold ? 1 : 0;
+}
+
+/* ---- KV deviation and high-deviation tokens -------------------------------------------- */
+
+/* Value of element e of a K/V array: bf16 bit patterns (is_f32 = 0) or float32. */
+static double kv_elem(const void* base, int32_t is_f32, int64_t e) {
+    return is_f32 ? (double)((const float*)base)[e] : oracle_bf16_value(((const uint16_t*)base)[e]);
+}
+
+/* Key-Value deviation (App. A.4): sigma_K = ||K_reused - K_recomputed||_2, sigma_V likewise,
+ * sigma_KV = sigma_K + sigma_V.  Read per layer l and token t, the norm running over all heads
+ * and head dimensions of that token's K (V) rows.  Arrays are [L][H][T][hd] contiguous.
+ * Outputs [L][T] (sigma_k, sigma_v nullable). */
+void oracle_kv_deviation(const void* k_re, const void* v_re, const void* k_rc, const void* v_rc, int32_t is_f32,
+                         int32_t L, int32_t H, int64_t T, int32_t hd, double* sigma_k, double* sigma_v,
+                         double* sigma_kv) {
+#pragma omp parallel for collapse(2) schedule(static)
+    for (int32_t l = 0; l < L; ++l)
+        for (int64_t t = 0; t < T; ++t) {
+            double sk = 0.0, sv = 0.0;
+            for (int32_t h = 0; h < H; ++h)
+                for (int32_t e = 0; e < hd; ++e) {
+                    const int64_t i = (((int64_t)l * H + h) * T + t) * hd + e;
+                    const double dk = kv_elem(k_re, is_f32, i) - kv_elem(k_rc, is_f32, i);
+                    const double dv = kv_elem(v_re, is_f32, i) - kv_elem(v_rc, is_f32, i);
+                    sk += dk * dk;
+                    sv += dv * dv;
+                }
+            const double a = sqrt(sk), b = sqrt(sv);
+            if (sigma_k) sigma_k[(int64_t)l * T + t] = a;
+            if (sigma_v) sigma_v[(int64_t)l * T + t] = b;
+            sigma_kv[(int64_t)l * T + t] = a + b;
+        }
+}
+
+/* High-deviation tokens (Insight 1: the tokens of highest deviation, 40% of them in the paper):
+ * for each layer, the k tokens of largest sigma (ties to the lower token index), listed in
+ * ascending token order in hd_idx[l][0..k).  A plain sort of (-sigma, t). */
+static const double* g_sort_sigma;
+static int cmp_desc_sigma(const void* a, const void* b) {
+    const int64_t i = *(const int64_t*)a, j = *(const int64_t*)b;
+    if (g_sort_sigma[i] > g_sort_sigma[j]) return -1;
+    if (g_sort_sigma[i] < g_sort_sigma[j]) return 1;
+    return i < j ? -1 : (i > j ? 1 : 0);
+}
+static int cmp_i64(const void* a, const void* b) {
+    const int64_t i = *(const int64_t*)a, j = *(const int64_t*)b;
+    return i < j ? -1 : (i > j ? 1 : 0);
+}
+
+void oracle_select_hd(const double* sigma, int32_t L, int64_t T, int64_t k, int32_t* hd_idx) {
+    int64_t* order = (int64_t*)malloc(sizeof(int64_t) * (size_t)(T > 0 ? T : 1));
+    for (int32_t l = 0; l < L; ++l) {
+        for (int64_t t = 0; t < T; ++t) order[t] = t;
+        g_sort_sigma = sigma + (int64_t)l * T;
+        qsort(order, (size_t)T, sizeof(int64_t), cmp_desc_sigma);
+        qsort(order, (size_t)k, sizeof(int64_t), cmp_i64);
+        for (int64_t i = 0; i < k; ++i) hd_idx[(int64_t)l * k + i] = (int32_t)order[i];
+    }
+    free(order);
 }
