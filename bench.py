@@ -70,6 +70,9 @@ def parse_args(argv=None):
     p.add_argument("--matcher", default="tc", choices=["tc", "popc"],
                    help="Hamming search: tensor-core GEMM (semshare_match_tc) or xor/popc (semshare_match)")
     p.add_argument("--e2e-steps", type=int, default=20)
+    p.add_argument("--hd", action="store_true",
+                   help="append the first layer's KV deviation against a (synthetic) recomputed first layer "
+                        "and the HD-token selection (App. A.4, Insight 1) to the step")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-clocks", action="store_true")
     return p.parse_args(argv)
@@ -118,6 +121,9 @@ def work(wl: workloads.Workload) -> dict:
         "match_wordops": float(n_t) * wl.n_ref * (wl.nbits // 32),
         "match_bytes": (n_t + wl.n_ref) * wl.nbits / 8 + n_t * 8,
         "gather_bytes": 2.0 * 2.0 * n_t * L * H * hd * 2,  # K and V, read + write
+        # first layer of every target prompt: reused and recomputed K and V read, 3 floats out
+        "deviation_bytes": 4.0 * n_t * H * hd * 2 + 3.0 * 4 * n_t,
+        "select_bytes": 4.0 * n_t + 4.0 * ((n_t * 40 + 99) // 100),
         "targets": n_t,
         "rows": rows,
     }
@@ -229,13 +235,13 @@ class Problem:
     # hash 1, match 3 (tc: expand + key reset, search, split; popc: key init, search, split), gather 1
     LAUNCHES_PER_STEP = 5
 
-    def __init__(self, wl: workloads.Workload, device, seed: int, matcher: str = "tc"):
+    def __init__(self, wl: workloads.Workload, device, seed: int, matcher: str = "tc", with_hd: bool = False):
         import torch
 
         import paper_2509_24832_gb300 as ss
 
         self.ss, self.wl, self.dev, self.matcher = ss, wl, device, matcher
-        emb, pos, _ = workloads.prompt_rows(wl, seed=seed)
+        emb, pos, src = workloads.prompt_rows(wl, seed=seed)
         self.host_emb, self.host_pos = emb, pos
         if wl.emb_dtype == "f32":
             self.emb = torch.from_numpy(emb).to(device)
@@ -263,6 +269,30 @@ class Problem:
         self.out_k = torch.empty((wl.n_batch, L, H, wl.n_tgt, hd), dtype=torch.bfloat16, device=device)
         self.out_v = torch.empty_like(self.out_k)
         self.flag = ss.new_err_flag(device)
+        self.hd = with_hd
+        if with_hd:
+            # a synthetic recomputed first layer per target prompt, [B][H][T][hd] (the layer-0 view
+            # of the gathered cache has the same shape, batch standing in for the layer index)
+            ks, vs = [], []
+            k0 = torch.cat([t[:1] for t in self.ref_k], dim=2)  # first layer of every member: global rows
+            v0 = torch.cat([t[:1] for t in self.ref_v], dim=2)
+            for b in range(wl.n_batch):
+                k_rc, v_rc = workloads.recomputed_kv_device(wl, device, k0, v0, src[b], seed=seed + b)
+                ks.append(k_rc[0])
+                vs.append(v_rc[0])
+            self.rc_k, self.rc_v = torch.stack(ks), torch.stack(vs)
+            del ks, vs, k0, v0
+            self.sigma = torch.empty((wl.n_batch, wl.n_tgt), dtype=torch.float32, device=device)
+            self.hd_k = ss.hd_count(wl.n_tgt)
+            self.hd_idx = torch.empty((wl.n_batch, self.hd_k), dtype=torch.int32, device=device)
+            self.STAGES = Problem.STAGES + ("deviation", "select")
+            self.LAUNCHES_PER_STEP = Problem.LAUNCHES_PER_STEP + 2
+
+    def deviation(self):
+        self.ss.semshare_kv_deviation(self.out_k[:, 0], self.out_v[:, 0], self.rc_k, self.rc_v, sigma_kv=self.sigma)
+
+    def select(self):
+        self.ss.semshare_select_hd(self.sigma, self.hd_k, hd_idx=self.hd_idx)
 
     def hash(self):
         self.ss.semshare_hash(self.emb, self.table, self.hyp, self.pos, codes=self.codes, err_flag=self.flag,
@@ -293,6 +323,13 @@ class Problem:
         self.gather()
         if ev:
             ev[3].record()
+        if self.hd:
+            self.deviation()
+            if ev:
+                ev[4].record()
+            self.select()
+            if ev:
+                ev[5].record()
 
     def e2e_plan(self):
         """(one, h2d, d2h, read): a step through the public API with host buffers -- the
@@ -460,9 +497,12 @@ class RetrieveProblem:
         return one, h2d, d2h, lambda: int(h_idx[0])
 
 
-def make_problem(wl, device, seed, matcher):
-    cls = RetrieveProblem if wl.recipe == "retrieve" else Problem
-    return cls(wl, device, seed, matcher)
+def make_problem(wl, device, seed, matcher, with_hd=False):
+    if wl.recipe == "retrieve":
+        if with_hd:
+            raise ValueError("--hd applies to the matching workloads")
+        return RetrieveProblem(wl, device, seed, matcher)
+    return Problem(wl, device, seed, matcher, with_hd=with_hd)
 
 
 def stage_report(wl, W, stage_ms, peaks, popc_peak, matcher):
@@ -492,6 +532,9 @@ def stage_report(wl, W, stage_ms, peaks, popc_peak, matcher):
                 r["frac_fp8_tensor"] = r["tflops_fp8"] / fp8_peak
         elif name == "gather":
             r["gbs"] = W["gather_bytes"] / sec / 1e9
+            r["frac_hbm"] = r["gbs"] / peaks["hbm_gbs"]
+        elif name in ("deviation", "select"):
+            r["gbs"] = W[name + "_bytes"] / sec / 1e9
             r["frac_hbm"] = r["gbs"] / peaks["hbm_gbs"]
         out[name] = r
     return out
@@ -526,7 +569,7 @@ def run_gpu_arm(args, rank, world, local_rank):
     torch.cuda.set_device(device)
     wl = ALL_WORKLOADS[args.workload]
     seed = wl.base_seed + 7919 * rank
-    prob = make_problem(wl, device, seed, args.matcher)
+    prob = make_problem(wl, device, seed, args.matcher, with_hd=args.hd)
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
     n_ev = len(prob.STAGES) + 1
 
@@ -587,6 +630,9 @@ def run_gpu_arm(args, rank, world, local_rank):
               "n_seg": wl.n_seg, "d": wl.d, "nbits": wl.nbits, "kv": list(wl.kv),
               "parallelism": f"replicas x{world}", "l2": "flushed before every step (256 MB write)",
               "matcher": args.matcher}
+    if args.hd:
+        config["hd"] = (f"first-layer KV deviation against a synthetic recomputed first layer, "
+                        f"top {workloads_hd_percent()}% tokens per prompt")
     if isinstance(prob, RetrieveProblem):
         config["retrieved"] = prob.winner
         config["stored_codes"] = "computed when the prompts were stored (outside the timed region)"
@@ -603,6 +649,12 @@ def run_gpu_arm(args, rank, world, local_rank):
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
+
+
+def workloads_hd_percent():
+    import paper_2509_24832_gb300 as ss
+
+    return ss.HD_PERCENT
 
 
 def evs_total(evs):

@@ -292,6 +292,50 @@ semshare_status semshare_gather_kv(const void* const* ref_k, const void* const* 
                                    int32_t n_batch, void* out_k, void* out_v, semshare_kv_layout dst,
                                    uint32_t* err_flag, void* stream);
 
+/*
+ * semshare_kv_deviation -- Key-Value deviation of the reused cache (App. A.4).
+ *
+ * sigma_K = ||K_reused - K_recomputed||_2, sigma_V likewise, sigma_KV = sigma_K + sigma_V
+ * (App. A.4), computed for every layer l < n_layers and token t < n_tok, the norm running over
+ * all n_heads x head_dim values of that token:
+ *     sigma_k[l][t] = sqrt(sum_h sum_e (k_reused[l][h][t][e] - k_recomp[l][h][t][e])^2)
+ * On the first layer every token is recomputed and this comparison picks the tokens for
+ * recomputation (Sec. 3.2); pass one layer (n_layers = 1) for that, more for per-layer analysis.
+ *
+ *   k_reused, v_reused  device, the rearranged cache (e.g. semshare_gather_kv's output for one
+ *                       target prompt), layout `reused` (stride_batch ignored)
+ *   k_recomp, v_recomp  device, the recomputed cache, layout `recomp`; n_layers, n_heads,
+ *                       head_dim and elem_bytes equal to `reused`'s
+ *   dtype               SEMSHARE_BF16 (elem_bytes 2) or SEMSHARE_F32 (elem_bytes 4)
+ *   n_tok               tokens; 0 launches nothing
+ *   sigma_k, sigma_v    device float[n_layers][n_tok] or NULL
+ *   sigma_kv            device float[n_layers][n_tok]
+ * Differences are squared and summed in fp32 in a fixed order (the same bits on every call);
+ * sqrt is correctly rounded.  Base pointers, strides (in bytes) and head_dim*elem_bytes must be
+ * multiples of 16.  Returns EINVAL for bad arguments, ECUDA if the launch fails.
+ */
+semshare_status semshare_kv_deviation(const void* k_reused, const void* v_reused, semshare_kv_layout reused,
+                                      const void* k_recomp, const void* v_recomp, semshare_kv_layout recomp,
+                                      semshare_dtype dtype, int64_t n_tok, float* sigma_k, float* sigma_v,
+                                      float* sigma_kv, void* stream);
+
+/*
+ * semshare_select_hd -- the high-deviation (HD) tokens of every layer.
+ *
+ * Insight 1 calls the tokens of highest KV deviation (40% of them) HD tokens; Sec. 3.2 hands
+ * the ones found on the first layer to recomputation.  For each layer l < n_layers: the k tokens
+ * with the largest sigma[l][t], ties at the k-th value going to the lower token index, listed in
+ * ascending token order.  NaN counts as larger than every number.
+ *
+ *   sigma     device float[n_layers][n_tok] (e.g. semshare_kv_deviation's sigma_kv)
+ *   k         0 <= k <= n_tok (the paper's 40%: k = ceil(0.4 * n_tok))
+ *   hd_idx    device int32[n_layers][k]
+ *   hd_mask   device uint8[n_layers][n_tok] or NULL: 1 for an HD token, else 0
+ * n_tok < 2^31, n_layers <= 65535.  Returns EINVAL for bad arguments, ECUDA if the launch fails.
+ */
+semshare_status semshare_select_hd(const float* sigma, int32_t n_layers, int64_t n_tok, int64_t k, int32_t* hd_idx,
+                                   uint8_t* hd_mask, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -4,12 +4,15 @@ The path: rotary position encoding of the embedding rows of a target and a refer
 (Sec. 3.3.1, Eq. 1), random-hyperplane LSH sign codes (Sec. 3.3, App. A.2), the Hamming
 nearest reference token of every target token (Sec. 3.3), and the rearrangement of the
 reference K/V cache into the target's order (Sec. 3.3, Sec. 3.3.2); before it, the retrieval of
-the stored prompt to reuse by LSH-distance similarity (Sec. 3.2, App. A.3).
+the stored prompt to reuse by LSH-distance similarity (Sec. 3.2, App. A.3); after it, the
+Key-Value deviation against the recomputed first layer and the high-deviation tokens (App. A.4,
+Insight 1).
 
 The compute lives in libsemshare.so (C ABI: include/semshare.h); this package is its thin
 ctypes binding with the same names.  Build the library with `paper_2509_24832_gb300.build`."""
 from ._native import (  # noqa: F401
     FLAG_INDEX,
+    HD_PERCENT,
     FLAG_TIMEOUT,
     KVLayout,
     LIB_PATH,
@@ -21,6 +24,7 @@ from ._native import (  # noqa: F401
     SemshareError,
     check_flag,
     flag_status,
+    hd_count,
     hash_workspace,
     kv_layout,
     load,
@@ -29,6 +33,7 @@ from ._native import (  # noqa: F401
     semshare_gather_kv,
     semshare_hash,
     semshare_hash_workspace_size,
+    semshare_kv_deviation,
     semshare_match,
     semshare_match_static,
     semshare_match_tc,
@@ -37,5 +42,6 @@ from ._native import (  # noqa: F401
     semshare_retrieve,
     semshare_retrieve_workspace_size,
     semshare_rope_table,
+    semshare_select_hd,
     status_string,
 )

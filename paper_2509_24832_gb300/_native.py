@@ -76,6 +76,10 @@ def load():
         lib.semshare_match_static.restype = ctypes.c_int
         lib.semshare_gather_kv.argtypes = [P, P, P, i32, KVLayout, P, i64, i32, P, P, KVLayout, P, P]
         lib.semshare_gather_kv.restype = ctypes.c_int
+        lib.semshare_kv_deviation.argtypes = [P, P, KVLayout, P, P, KVLayout, ctypes.c_int, i64, P, P, P, P]
+        lib.semshare_kv_deviation.restype = ctypes.c_int
+        lib.semshare_select_hd.argtypes = [P, i32, i64, i64, P, P, P]
+        lib.semshare_select_hd.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -414,3 +418,65 @@ def semshare_gather_kv(ref_k, ref_v, idx: torch.Tensor, out_k: torch.Tensor | No
                                    _ptr(err_flag), _stream(stream))
     _check(st, "semshare_gather_kv")
     return out_k, out_v
+
+
+HD_PERCENT = 40  # Insight 1: the 40% of tokens with the highest deviation are HD tokens
+
+
+def hd_count(n_tok: int, percent: int = HD_PERCENT) -> int:
+    """Number of HD tokens: ceil(percent% of n_tok), in integer arithmetic."""
+    return (int(n_tok) * int(percent) + 99) // 100
+
+
+def semshare_kv_deviation(k_reused: torch.Tensor, v_reused: torch.Tensor, k_recomp: torch.Tensor,
+                          v_recomp: torch.Tensor, sigma_kv: torch.Tensor | None = None,
+                          sigma_k: torch.Tensor | None = None, sigma_v: torch.Tensor | None = None,
+                          want_parts: bool = False, stream=None):
+    """Key-Value deviation (App. A.4) per layer and token of [L][H][T][hd] caches (bf16 or fp32;
+    strided views allowed, head_dim contiguous).  Returns sigma_kv, or (sigma_k, sigma_v,
+    sigma_kv) with want_parts; each float32 [L][T]."""
+    ts = (k_reused, v_reused, k_recomp, v_recomp)
+    for t, n in zip(ts, ("k_reused", "v_reused", "k_recomp", "v_recomp")):
+        _need_cuda(t, n)
+    if k_reused.dtype == torch.bfloat16:
+        dt = BF16
+    elif k_reused.dtype == torch.float32:
+        dt = F32
+    else:
+        raise TypeError("caches must be bfloat16 or float32")
+    if any(t.dtype != k_reused.dtype or t.shape != k_reused.shape for t in ts) or k_reused.dim() != 4:
+        raise ValueError("four [L][H][T][hd] caches of one shape and dtype")
+    if v_reused.stride() != k_reused.stride() or v_recomp.stride() != k_recomp.stride():
+        raise ValueError("K and V of a cache must share strides")
+    L, _, T, _ = k_reused.shape
+    dev = k_reused.device
+    if sigma_kv is None:
+        sigma_kv = torch.empty((L, T), dtype=torch.float32, device=dev)
+    if want_parts:
+        sigma_k = torch.empty((L, T), dtype=torch.float32, device=dev) if sigma_k is None else sigma_k
+        sigma_v = torch.empty((L, T), dtype=torch.float32, device=dev) if sigma_v is None else sigma_v
+    st = load().semshare_kv_deviation(_ptr(k_reused), _ptr(v_reused), kv_layout(k_reused, False), _ptr(k_recomp),
+                                      _ptr(v_recomp), kv_layout(k_recomp, False), dt, T, _ptr(sigma_k),
+                                      _ptr(sigma_v), _ptr(sigma_kv), _stream(stream))
+    _check(st, "semshare_kv_deviation")
+    return (sigma_k, sigma_v, sigma_kv) if want_parts else sigma_kv
+
+
+def semshare_select_hd(sigma: torch.Tensor, k: int | None = None, hd_idx: torch.Tensor | None = None,
+                       want_mask: bool = False, hd_mask: torch.Tensor | None = None, stream=None):
+    """The k highest-deviation tokens of every layer (default k = hd_count(T)), ascending, ties
+    to the lower index.  sigma: float32 [L][T] (or [T]).  Returns hd_idx int32 [L][k] (and the
+    uint8 [L][T] mask with want_mask)."""
+    _need_cuda(sigma, "sigma")
+    if sigma.dtype != torch.float32 or not sigma.is_contiguous():
+        raise ValueError("sigma must be a contiguous float32 tensor")
+    s2 = sigma.view(1, -1) if sigma.dim() == 1 else sigma
+    L, T = s2.shape
+    k = hd_count(T) if k is None else int(k)
+    if hd_idx is None:
+        hd_idx = torch.empty((L, k), dtype=torch.int32, device=sigma.device)
+    if want_mask and hd_mask is None:
+        hd_mask = torch.empty((L, T), dtype=torch.uint8, device=sigma.device)
+    st = load().semshare_select_hd(_ptr(s2), L, T, k, _ptr(hd_idx), _ptr(hd_mask), _stream(stream))
+    _check(st, "semshare_select_hd")
+    return (hd_idx, hd_mask) if want_mask else hd_idx

@@ -16,7 +16,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "libsemshare.so")
-SOURCES = ["api.cu", "hash.cu", "match.cu", "match_tc.cu", "gather.cu"]
+SOURCES = ["api.cu", "hash.cu", "match.cu", "match_tc.cu", "gather.cu", "deviation.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2", "-I", INCLUDE, "-I", CSRC]
 

@@ -64,13 +64,14 @@ def _retrieval(a, wl, e, pd, R, table, flag, dev):
 
 def main(argv=None):
     p = argparse.ArgumentParser()
-    p.add_argument("--kernel", choices=["hash", "match", "match_tc", "gather", "retrieve"], required=True)
+    p.add_argument("--kernel", choices=["hash", "match", "match_tc", "gather", "retrieve", "deviation", "select"],
+                   required=True)
     p.add_argument("--workload", default="llama8b-5k", choices=sorted(ALL))
     p.add_argument("--reps", type=int, default=3)
     a = p.parse_args(argv)
     dev = torch.device("cuda")
     wl = ALL[a.workload]
-    emb, pos, _ = workloads.prompt_rows(wl)
+    emb, pos, src = workloads.prompt_rows(wl)
     e = torch.from_numpy(emb).to(dev) if emb.dtype == np.float32 else \
         torch.from_numpy(emb.view(np.int16)).to(dev).view(torch.bfloat16)
     pd = torch.from_numpy(pos).to(dev)
@@ -97,7 +98,7 @@ def main(argv=None):
             elif a.kernel == "match_tc":
                 for _ in range(a.reps):
                     ss.semshare_match_tc(tc, rc, idx=idx, dist=dist, err_flag=flag)
-            else:
+            elif a.kernel == "gather":
                 del e
                 segs = [workloads.kv_cache_device(wl, dev, segment=s) for s in range(wl.n_seg)]
                 L, H, hd = wl.kv
@@ -106,6 +107,29 @@ def main(argv=None):
                 for _ in range(a.reps):
                     ss.semshare_gather_kv([s[0] for s in segs], [s[1] for s in segs],
                                           idx.view(wl.n_batch, wl.n_tgt), out_k=out_k, out_v=out_v, err_flag=flag)
+            else:
+                # first layer only: gather it, compare with a synthetic recomputed first layer
+                del e
+                segs = [workloads.kv_cache_device(wl, dev, segment=s) for s in range(wl.n_seg)]
+                k0 = torch.cat([s[0][:1] for s in segs], dim=2)
+                v0 = torch.cat([s[1][:1] for s in segs], dim=2)
+                del segs
+                _, H, _, hd = k0.shape
+                out_k = torch.empty((wl.n_batch, 1, H, wl.n_tgt, hd), dtype=torch.bfloat16, device=dev)
+                out_v = torch.empty_like(out_k)
+                ss.semshare_gather_kv(k0, v0, idx.view(wl.n_batch, wl.n_tgt), out_k=out_k, out_v=out_v,
+                                      err_flag=flag)
+                rc = [workloads.recomputed_kv_device(wl, dev, k0, v0, src[b], seed=wl.base_seed + b)
+                      for b in range(wl.n_batch)]
+                rc_k = torch.stack([r[0][0] for r in rc])
+                rc_v = torch.stack([r[1][0] for r in rc])
+                sigma = ss.semshare_kv_deviation(out_k[:, 0], out_v[:, 0], rc_k, rc_v)
+                reps = a.reps if a.kernel == "deviation" else 1
+                for _ in range(reps - 1):
+                    ss.semshare_kv_deviation(out_k[:, 0], out_v[:, 0], rc_k, rc_v, sigma_kv=sigma)
+                if a.kernel == "select":
+                    for _ in range(a.reps):
+                        ss.semshare_select_hd(sigma)
     torch.cuda.synchronize()
     ss.check_flag(flag, a.kernel)
     print(f"{a.kernel} on {wl.name}: {a.reps} launches ok")

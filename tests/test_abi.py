@@ -126,6 +126,28 @@ def test_retrieve_argument_errors(lib):
     assert lib.semshare_retrieve_workspace_size(10, 5, 1, 64) > lib.semshare_match_tc_workspace_size(10, 5, 64)
 
 
+def test_deviation_and_select_argument_errors(lib):
+    import paper_2509_24832_gb300 as ss
+
+    lay = ss.KVLayout(1, 8, 128, 2, 0, 8 * 100 * 128, 100 * 128, 128)
+    d = lib.semshare_kv_deviation
+    assert d(FAKE, FAKE, lay, FAKE, FAKE, lay, 7, 100, None, None, FAKE, None) == 1       # dtype
+    assert d(FAKE, FAKE, lay, FAKE, FAKE, lay, 1, 100, None, None, FAKE, None) == 1       # f32 vs 2-byte elements
+    other = ss.KVLayout(1, 4, 128, 2, 0, 4 * 100 * 128, 100 * 128, 128)
+    assert d(FAKE, FAKE, lay, FAKE, FAKE, other, 0, 100, None, None, FAKE, None) == 1     # head mismatch
+    odd = ss.KVLayout(1, 8, 60, 2, 0, 8 * 100 * 60, 100 * 60, 60)                         # 120-byte rows
+    assert d(FAKE, FAKE, odd, FAKE, FAKE, odd, 0, 100, None, None, FAKE, None) == 1
+    assert d(FAKE, FAKE, lay, FAKE, FAKE, lay, 0, 100, None, None, None, None) == 1       # no sigma_kv
+    assert d(ctypes.c_void_p((1 << 20) + 8), FAKE, lay, FAKE, FAKE, lay, 0, 100, None, None, FAKE, None) == 1
+    assert d(None, None, lay, None, None, lay, 0, 0, None, None, None, None) == 0         # empty
+    s = lib.semshare_select_hd
+    assert s(FAKE, 1, 100, 101, FAKE, None, None) == 1                                    # k > n_tok
+    assert s(FAKE, 1, 100, -1, FAKE, None, None) == 1
+    assert s(FAKE, 1, 100, 10, None, None, None) == 1                                     # no output
+    assert s(FAKE, 70000, 100, 10, FAKE, None, None) == 2                                 # too many layers
+    assert s(None, 1, 0, 0, None, None, None) == 0                                        # empty
+
+
 def test_rope_table_argument_errors(lib):
     t = lib.semshare_rope_table
     assert t(7, 10000.0, FAKE, None) == 1

@@ -257,3 +257,24 @@ def prompt_rows(wl: Workload, seed: int | None = None, batches=None):
         pos.append(p)
         src.append(s)
     return np.concatenate(rows), np.concatenate(pos).astype(np.int32), np.stack(src)
+
+
+def recomputed_kv_device(wl: Workload, device, k_ref, v_ref, src, seed: int | None = None, noise: float = 0.05):
+    """A synthetic recomputed cache for the target prompt, [L][H][n_tgt][hd] bf16 each: a target
+    token copied from reference row src[t] gets that row's K/V plus N(0, noise^2); a fresh token
+    (src[t] = -1) gets fresh N(0,1) values.  k_ref/v_ref: the reference cache's layers to
+    recompute ([L][H][N][hd]); seeded through a device generator."""
+    import torch
+
+    seed = wl.base_seed if seed is None else seed
+    g = torch.Generator(device=device).manual_seed((seed * 7919 + 104729) & 0x7FFFFFFFFFFFFFFF)
+    s = torch.as_tensor(np.asarray(src), device=device).long()
+    copied = s >= 0
+    out = []
+    for ref in (k_ref, v_ref):
+        L, H, _, hd = ref.shape
+        x = torch.randn((L, H, len(s), hd), generator=g, device=device)
+        base = ref.float()[:, :, s.clamp(min=0)]
+        x = torch.where(copied.view(1, 1, -1, 1), base + noise * x, x)
+        out.append(x.to(torch.bfloat16).contiguous())
+    return out[0], out[1]
