@@ -14,6 +14,7 @@ it follows, is stated in `semshare_oracle.c`:
           App. A.3, Sec. 4.4
   kv_deviation  sigma_K + sigma_V per layer and token; App. A.4
   select_hd     the k highest-deviation tokens per layer; Insight 1, Sec. 3.2
+  gather_kv_retained  the rearranged rows of each layer's retained tokens only; Sec. 3.3.4, App. A
 
 Parity pins: every function here is pinned by `tests/test_oracle_*.py` against closed forms,
 invariants, hand-derived golden cases and brute force (none is "parity unpinned").
@@ -72,6 +73,8 @@ def _load():
         lib.oracle_retrieve.argtypes = [P, i64, P, P, i32, i32, f64, f64, P, P, P, P]
         lib.oracle_kv_deviation.argtypes = [P, P, P, P, i32, i32, i32, i64, i32, P, P, P]
         lib.oracle_select_hd.argtypes = [P, i32, i64, i64, P]
+        lib.oracle_gather_kv_retained.argtypes = [P, P, i32, i32, i64, i64, P, i64, P, P, i64, P, P]
+        lib.oracle_gather_kv_retained.restype = i64
         _lib = lib
         return lib
 
@@ -234,3 +237,30 @@ def select_hd(sigma, k: int):
     out = np.zeros((L, k), dtype=np.int32)
     _load().oracle_select_hd(_ptr(s), L, T, int(k), _ptr(out))
     return out
+
+
+def gather_kv_retained(ref_k, ref_v, idx, retained, cap: int | None = None, out_k=None, out_v=None):
+    """Retention-aware rearrangement (Sec. 3.3.4, App. A): ref_k/ref_v [L][H][N][hd] (one
+    reference prompt), idx [n_tgt], retained: L sequences of target tokens (layer l keeps
+    retained[l]).  out[l][h][r] = ref[l][h][idx[retained[l][r]]], out [L][H][cap][hd] (cap
+    defaults to the longest list; other rows stay as given, zeros when allocated here).
+    Returns (out_k, out_v, n_bad)."""
+    ref_k = np.ascontiguousarray(ref_k)
+    ref_v = np.ascontiguousarray(ref_v)
+    L, H, N, hd = ref_k.shape
+    idx = np.ascontiguousarray(np.asarray(idx, dtype=np.int32))
+    if len(retained) != L:
+        raise ValueError("one retained list per layer")
+    off = np.zeros(L + 1, dtype=np.int64)
+    for l, r in enumerate(retained):
+        off[l + 1] = off[l] + len(r)
+    flat = np.ascontiguousarray(np.concatenate([np.asarray(r, dtype=np.int32) for r in retained])
+                                if off[-1] else np.zeros(1, dtype=np.int32))
+    cap = int(max((len(r) for r in retained), default=0)) if cap is None else int(cap)
+    if out_k is None:
+        out_k = np.zeros((L, H, cap, hd), dtype=ref_k.dtype)
+    if out_v is None:
+        out_v = np.zeros((L, H, cap, hd), dtype=ref_v.dtype)
+    bad = _load().oracle_gather_kv_retained(_ptr(ref_k), _ptr(ref_v), L, H, N, hd * ref_k.dtype.itemsize, _ptr(idx),
+                                            len(idx), _ptr(flat), _ptr(off), cap, _ptr(out_k), _ptr(out_v))
+    return out_k, out_v, int(bad)

@@ -33,6 +33,8 @@
  *              ||K_reused - K_recomputed||_2 + ||V_reused - V_recomputed||_2 over all heads; the
  *              tokens of highest deviation (40% in the paper, Insight 1) are the HD tokens that
  *              the first layer's comparison hands to recomputation (Sec. 3.2).
+ *   7. gather_kv_retained  Retention (Sec. 3.3.4, App. A): each layer keeps only its retained
+ *              target tokens; its rearranged cache holds just their rows, packed in list order.
  *
  * Build: gcc -O2 -fopenmp -ffp-contract=off -shared -fPIC (no fused multiply-add, so x86 and
  * Arm hosts produce the same bits).
@@ -308,4 +310,34 @@ void oracle_select_hd(const double* sigma, int32_t L, int64_t T, int64_t k, int3
         for (int64_t i = 0; i < k; ++i) hd_idx[(int64_t)l * k + i] = (int32_t)order[i];
     }
     free(order);
+}
+
+/* ---- retention-aware rearrangement --------------------------------------------------------- */
+
+/* Retention (Sec. 3.3.4; App. A: Retain[i] = T * prod_{j<=i} alpha_retain[j], tokens not retained
+ * are evicted): layer l keeps only the target tokens ret[ret_off[l] .. ret_off[l+1]) and its
+ * rearranged cache holds just those rows, packed in list order:
+ *     out[l][h][r] = ref[l][h][idx[ret[ret_off[l] + r]]]
+ * One reference prompt [L][H][N][row_bytes], idx [n_tgt], out [L][H][cap][row_bytes] (cap >= the
+ * longest list; rows past a layer's count are left as they were).  A retained token outside
+ * [0, n_tgt) or an idx outside [0, N) leaves its row untouched and is counted; returns the count. */
+int64_t oracle_gather_kv_retained(const uint8_t* ref_k, const uint8_t* ref_v, int32_t L, int32_t H, int64_t N,
+                                  int64_t row_bytes, const int32_t* idx, int64_t n_tgt, const int32_t* ret,
+                                  const int64_t* ret_off, int64_t cap, uint8_t* out_k, uint8_t* out_v) {
+    int64_t bad = 0;
+    for (int32_t l = 0; l < L; ++l)
+        for (int64_t r = 0; r < ret_off[l + 1] - ret_off[l]; ++r) {
+            const int64_t t = ret[ret_off[l] + r];
+            if (t < 0 || t >= n_tgt || idx[t] < 0 || idx[t] >= N) {
+                ++bad;
+                continue;
+            }
+            for (int32_t h = 0; h < H; ++h) {
+                const int64_t src = (((int64_t)l * H + h) * N + idx[t]) * row_bytes;
+                const int64_t dst = (((int64_t)l * H + h) * cap + r) * row_bytes;
+                memcpy(out_k + dst, ref_k + src, (size_t)row_bytes);
+                memcpy(out_v + dst, ref_v + src, (size_t)row_bytes);
+            }
+        }
+    return bad;
 }
