@@ -51,8 +51,8 @@ L2_FLUSH_BYTES = 256 << 20
 # workload, valid only for that workload and while the kernel source has the recorded sha256
 # prefix (the traffic depends on the index pattern, e.g. how often a gathered row repeats).
 NCU_TRAFFIC = {
-    ("gather", "llama8b-5k"): {"file": "gather.cu", "sha": "e03583daf19419cb", "bytes_per_launch": 1092.8e6},
-    ("gather", "retrieve-16x4096"): {"file": "gather.cu", "sha": "e03583daf19419cb", "bytes_per_launch": 1000.5e6},
+    ("gather", "llama8b-5k"): {"file": "gather.cu", "sha": "7d05bda6e8a70170", "bytes_per_launch": 1092.7e6},
+    ("gather_retained", "llama8b-5k"): {"file": "gather.cu", "sha": "7d05bda6e8a70170", "bytes_per_launch": 663.2e6},
     ("hash", "llama8b-5k"): {"file": "hash.cu", "sha": "0fc6e508c36def23", "bytes_per_launch": 90.65e6},
     ("match", "llama8b-5k"): {"file": "match.cu", "sha": "69ac4b7ce5b193e4", "bytes_per_launch": 0.3845e6},
     ("match_tc", "llama8b-5k"): {"file": "match_tc.cu", "sha": "c494ec8dce435f1b", "bytes_per_launch": 2.736e6},
@@ -70,6 +70,9 @@ def parse_args(argv=None):
     p.add_argument("--matcher", default="tc", choices=["tc", "popc"],
                    help="Hamming search: tensor-core GEMM (semshare_match_tc) or xor/popc (semshare_match)")
     p.add_argument("--e2e-steps", type=int, default=20)
+    p.add_argument("--retain", action="store_true",
+                   help="gather only each layer's retained tokens (Sec. 3.3.4; synthetic schedule: 0.8 on the "
+                        "first layer, then 0.98 per layer; one-prompt workloads)")
     p.add_argument("--hd", action="store_true",
                    help="append the first layer's KV deviation against a (synthetic) recomputed first layer "
                         "and the HD-token selection (App. A.4, Insight 1) to the step")
@@ -235,7 +238,8 @@ class Problem:
     # hash 1, match 3 (tc: expand + key reset, search, split; popc: key init, search, split), gather 1
     LAUNCHES_PER_STEP = 5
 
-    def __init__(self, wl: workloads.Workload, device, seed: int, matcher: str = "tc", with_hd: bool = False):
+    def __init__(self, wl: workloads.Workload, device, seed: int, matcher: str = "tc", with_hd: bool = False,
+                 with_retain: bool = False):
         import torch
 
         import paper_2509_24832_gb300 as ss
@@ -269,6 +273,16 @@ class Problem:
         self.out_k = torch.empty((wl.n_batch, L, H, wl.n_tgt, hd), dtype=torch.bfloat16, device=device)
         self.out_v = torch.empty_like(self.out_k)
         self.flag = ss.new_err_flag(device)
+        self.retain = with_retain
+        if with_retain:
+            if wl.n_batch != 1 or with_hd:
+                raise ValueError("--retain takes a one-prompt workload and no --hd")
+            self.counts = ss.retain_counts(wl.n_tgt, workloads.retain_alphas(L))
+            ret = workloads.retained_tokens(wl.n_tgt, self.counts, seed)
+            self.ret = torch.from_numpy(np.concatenate(ret)).to(device)
+            self.ret_off = [0] + list(np.cumsum(self.counts))
+            self.out_k = torch.empty((L, H, self.counts[0], hd), dtype=torch.bfloat16, device=device)
+            self.out_v = torch.empty_like(self.out_k)
         self.hd = with_hd
         if with_hd:
             # a synthetic recomputed first layer per target prompt, [B][H][T][hd] (the layer-0 view
@@ -308,6 +322,10 @@ class Problem:
                                    workspace=self.ws)
 
     def gather(self):
+        if self.retain:
+            self.ss.semshare_gather_kv_retained(self.ref_k, self.ref_v, self.idx, self.ret, self.ret_off,
+                                                out_k=self.out_k, out_v=self.out_v, err_flag=self.flag)
+            return
         self.ss.semshare_gather_kv(self.ref_k, self.ref_v, self.idx.view(self.wl.n_batch, self.wl.n_tgt),
                                    out_k=self.out_k, out_v=self.out_v, err_flag=self.flag)
 
@@ -497,12 +515,12 @@ class RetrieveProblem:
         return one, h2d, d2h, lambda: int(h_idx[0])
 
 
-def make_problem(wl, device, seed, matcher, with_hd=False):
+def make_problem(wl, device, seed, matcher, with_hd=False, with_retain=False):
     if wl.recipe == "retrieve":
-        if with_hd:
-            raise ValueError("--hd applies to the matching workloads")
+        if with_hd or with_retain:
+            raise ValueError("--hd and --retain apply to the matching workloads")
         return RetrieveProblem(wl, device, seed, matcher)
-    return Problem(wl, device, seed, matcher, with_hd=with_hd)
+    return Problem(wl, device, seed, matcher, with_hd=with_hd, with_retain=with_retain)
 
 
 def stage_report(wl, W, stage_ms, peaks, popc_peak, matcher):
@@ -569,7 +587,7 @@ def run_gpu_arm(args, rank, world, local_rank):
     torch.cuda.set_device(device)
     wl = ALL_WORKLOADS[args.workload]
     seed = wl.base_seed + 7919 * rank
-    prob = make_problem(wl, device, seed, args.matcher, with_hd=args.hd)
+    prob = make_problem(wl, device, seed, args.matcher, with_hd=args.hd, with_retain=args.retain)
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
     n_ev = len(prob.STAGES) + 1
 
@@ -605,6 +623,9 @@ def run_gpu_arm(args, rank, world, local_rank):
     ms_step = reduce_max(ms_local, device)
     stage_ms = {n: reduce_max(float(st[:, i].mean()), device) for i, n in enumerate(prob.STAGES)}
     W = work(wl)
+    if getattr(prob, "retain", False):
+        L, H, hd = wl.kv
+        W["gather_bytes"] = 2.0 * 2.0 * float(sum(prob.counts)) * H * hd * 2
     value = world * W["targets"] / (ms_step * 1e-3)
 
     peaks, peak_src = load_peaks()
@@ -616,6 +637,9 @@ def run_gpu_arm(args, rank, world, local_rank):
 
     dominant = max(stage_ms, key=stage_ms.get)
     roof, tr = roofline_for(dominant, stages, peaks, args.matcher, wl.name)
+    if getattr(prob, "retain", False) and dominant == "gather":
+        roof["kernel"] = "kv_gather_kernel (retained rows)"
+        tr = NCU_TRAFFIC.get(("gather_retained", wl.name))
     roof["frac"] = roof["achieved"] / roof["peak"]
     roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"
     roof["traffic"] = tr["bytes_per_launch"] if tr and tr.get("sha") == kernel_sha(tr["file"]) else None
@@ -630,6 +654,9 @@ def run_gpu_arm(args, rank, world, local_rank):
               "n_seg": wl.n_seg, "d": wl.d, "nbits": wl.nbits, "kv": list(wl.kv),
               "parallelism": f"replicas x{world}", "l2": "flushed before every step (256 MB write)",
               "matcher": args.matcher}
+    if args.retain:
+        config["retain"] = (f"per-layer retained tokens, first {prob.counts[0]}, last {prob.counts[-1]}, "
+                            f"{sum(prob.counts)} rows of {wl.n_layers * wl.n_tgt} (0.8, then 0.98 per layer)")
     if args.hd:
         config["hd"] = (f"first-layer KV deviation against a synthetic recomputed first layer, "
                         f"top {workloads_hd_percent()}% tokens per prompt")

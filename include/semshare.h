@@ -293,6 +293,36 @@ semshare_status semshare_gather_kv(const void* const* ref_k, const void* const* 
                                    uint32_t* err_flag, void* stream);
 
 /*
+ * semshare_gather_kv_retained -- step 4 with retention: each layer keeps only its retained tokens.
+ *
+ * Sec. 3.3.4 and App. A: layer i retains Retain[i] = T * prod_{j<=i} alpha_retain[j] of the T
+ * target tokens and evicts the rest.  Given each layer's retained target tokens (chosen from
+ * attention scores by the caller), the layer's rearranged cache holds only their rows, packed in
+ * list order, for one target prompt:
+ *     out_k[l][h][r][:] = ref_k[l][h][idx[retained[ret_offsets[l] + r]]][:]    (same for V)
+ * for r < ret_offsets[l+1] - ret_offsets[l].  Evicted tokens are neither read nor written.
+ *
+ *   ref_k, ref_v, seg_offsets, n_seg, src   as for semshare_gather_kv
+ *   idx          device int32[n_tgt]: the target prompt's global reference rows
+ *   retained     device int32: the layers' retained target tokens back to back (values in
+ *                [0, n_tgt); conventionally ascending within a layer)
+ *   ret_offsets  HOST int64[n_layers + 1], ret_offsets[0] = 0, non-decreasing; read before the
+ *                call returns.  n_layers <= SEMSHARE_RETAIN_MAX_LAYERS
+ *   out_k, out_v device destination, layout `dst` (stride_batch ignored); its token dimension must
+ *                hold the longest list; rows past a layer's count are left untouched
+ *   err_flag     device or NULL; a retained token outside [0, n_tgt) or an idx outside the
+ *                reference leaves its row untouched and sets SEMSHARE_FLAG_INDEX
+ * Alignment rules as for semshare_gather_kv.  Returns EINVAL / EUNSUPPORTED for bad arguments,
+ * ECUDA if the launch fails.
+ */
+#define SEMSHARE_RETAIN_MAX_LAYERS 128
+semshare_status semshare_gather_kv_retained(const void* const* ref_k, const void* const* ref_v,
+                                            const int64_t* seg_offsets, int32_t n_seg, semshare_kv_layout src,
+                                            const int32_t* idx, int64_t n_tgt, const int32_t* retained,
+                                            const int64_t* ret_offsets, void* out_k, void* out_v,
+                                            semshare_kv_layout dst, uint32_t* err_flag, void* stream);
+
+/*
  * semshare_kv_deviation -- Key-Value deviation of the reused cache (App. A.4).
  *
  * sigma_K = ||K_reused - K_recomputed||_2, sigma_V likewise, sigma_KV = sigma_K + sigma_V

@@ -17,6 +17,7 @@ from ._native import (  # noqa: F401
     KVLayout,
     LIB_PATH,
     MATCH_STATIC_MAX_TARGETS,
+    RETAIN_MAX_LAYERS,
     RETRIEVE_MAX_CANDIDATES,
     SIMILARITY_MAX_DIST,
     SIMILARITY_THRESHOLD,
@@ -29,8 +30,10 @@ from ._native import (  # noqa: F401
     kv_layout,
     load,
     new_err_flag,
+    retain_counts,
     semshare_abi_version,
     semshare_gather_kv,
+    semshare_gather_kv_retained,
     semshare_hash,
     semshare_hash_workspace_size,
     semshare_kv_deviation,

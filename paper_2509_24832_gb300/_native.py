@@ -6,6 +6,7 @@ library is missing the call raises."""
 from __future__ import annotations
 
 import ctypes
+import math
 import os
 import threading
 from typing import NamedTuple
@@ -76,6 +77,8 @@ def load():
         lib.semshare_match_static.restype = ctypes.c_int
         lib.semshare_gather_kv.argtypes = [P, P, P, i32, KVLayout, P, i64, i32, P, P, KVLayout, P, P]
         lib.semshare_gather_kv.restype = ctypes.c_int
+        lib.semshare_gather_kv_retained.argtypes = [P, P, P, i32, KVLayout, P, i64, P, P, P, P, KVLayout, P, P]
+        lib.semshare_gather_kv_retained.restype = ctypes.c_int
         lib.semshare_kv_deviation.argtypes = [P, P, KVLayout, P, P, KVLayout, ctypes.c_int, i64, P, P, P, P]
         lib.semshare_kv_deviation.restype = ctypes.c_int
         lib.semshare_select_hd.argtypes = [P, i32, i64, i64, P, P, P]
@@ -480,3 +483,66 @@ def semshare_select_hd(sigma: torch.Tensor, k: int | None = None, hd_idx: torch.
     st = load().semshare_select_hd(_ptr(s2), L, T, k, _ptr(hd_idx), _ptr(hd_mask), _stream(stream))
     _check(st, "semshare_select_hd")
     return (hd_idx, hd_mask) if want_mask else hd_idx
+
+
+RETAIN_MAX_LAYERS = 128
+
+
+def retain_counts(n_tok: int, alphas) -> list:
+    """Retained tokens per layer, Retain[i] = T * prod_{j<=i} alpha_retain[j] (App. A), rounded
+    down (a product within 1e-9 of an integer counts as that integer)."""
+    out, p = [], 1.0
+    for a in alphas:
+        p *= float(a)
+        out.append(int(math.floor(n_tok * p + 1e-9)))
+    return out
+
+
+def semshare_gather_kv_retained(ref_k, ref_v, idx: torch.Tensor, retained, ret_offsets,
+                                out_k: torch.Tensor | None = None, out_v: torch.Tensor | None = None,
+                                err_flag: torch.Tensor | None = None, stream=None):
+    """Retention-aware rearrangement (Sec. 3.3.4): out[l][h][r] = ref[l][h][idx[retained_l[r]]].
+
+    ref_k/ref_v: a [L][H][N][hd] CUDA tensor or a list of them (a pool, as semshare_gather_kv).
+    idx: int32 [n_tgt].  retained: int32 CUDA tensor, the layers' lists back to back;
+    ret_offsets: host sequence of L + 1 ints.  Returns (out_k, out_v), [L][H][longest][hd]."""
+    seg_k = list(ref_k) if isinstance(ref_k, (list, tuple)) else [ref_k]
+    seg_v = list(ref_v) if isinstance(ref_v, (list, tuple)) else [ref_v]
+    if len(seg_k) != len(seg_v) or not seg_k:
+        raise ValueError("ref_k and ref_v must have the same number of segments")
+    for t in seg_k + seg_v:
+        _need_cuda(t, "ref")
+    src = kv_layout(seg_k[0], batched=False)
+    for t in seg_k[1:] + seg_v:
+        o = kv_layout(t, batched=False)
+        if (o.stride_layer, o.stride_head, o.stride_token, o.head_dim, o.elem_bytes) != \
+                (src.stride_layer, src.stride_head, src.stride_token, src.head_dim, src.elem_bytes):
+            raise ValueError("all segments must share one layout")
+    _need_cuda(idx, "idx")
+    _need_cuda(retained, "retained")
+    if idx.dtype != torch.int32 or not idx.is_contiguous() or retained.dtype != torch.int32 or \
+            not retained.is_contiguous():
+        raise ValueError("idx and retained must be contiguous int32")
+    L, H, hd = src.n_layers, src.n_heads, src.head_dim
+    if len(ret_offsets) != L + 1:
+        raise ValueError("ret_offsets needs n_layers + 1 entries")
+    longest = max(int(ret_offsets[l + 1]) - int(ret_offsets[l]) for l in range(L))
+    if out_k is None:
+        out_k = torch.empty((L, H, max(longest, 0), hd), dtype=seg_k[0].dtype, device=seg_k[0].device)
+    if out_v is None:
+        out_v = torch.empty((L, H, max(longest, 0), hd), dtype=seg_v[0].dtype, device=seg_v[0].device)
+    dst = kv_layout(out_k, batched=False)
+    if kv_layout(out_v, batched=False).stride_token != dst.stride_token or out_v.stride() != out_k.stride():
+        raise ValueError("out_k and out_v must share one layout")
+    offs = [0]
+    for t in seg_k:
+        offs.append(offs[-1] + t.shape[2])
+    n_seg = len(seg_k)
+    pk = (ctypes.c_void_p * n_seg)(*[t.data_ptr() for t in seg_k])
+    pv = (ctypes.c_void_p * n_seg)(*[t.data_ptr() for t in seg_v])
+    po = (ctypes.c_int64 * (n_seg + 1))(*offs)
+    ro = (ctypes.c_int64 * (L + 1))(*[int(o) for o in ret_offsets])
+    st = load().semshare_gather_kv_retained(pk, pv, po, n_seg, src, _ptr(idx), idx.numel(), _ptr(retained), ro,
+                                            _ptr(out_k), _ptr(out_v), dst, _ptr(err_flag), _stream(stream))
+    _check(st, "semshare_gather_kv_retained")
+    return out_k, out_v

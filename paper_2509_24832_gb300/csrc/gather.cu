@@ -12,6 +12,12 @@
 // all of its 16-byte loads (read-only path, no L1 allocation) before any of its stores, so
 // each thread keeps 2*64*row_bytes/(16*256) requests in flight.  Consecutive threads touch
 // consecutive 16-byte chunks of a row and consecutive rows of the destination.
+//
+// Retention (semshare_gather_kv_retained; Sec. 3.3.4, App. A: Retain[i] = T * prod alpha_retain,
+// evicted tokens dropped): each layer keeps only the target tokens of its list, and its cache
+// holds just their rows, packed in list order -- out[l][h][r] = ref[l][h][idx[ret_l[r]]].  The
+// same kernels run with the token index remapped through the layer's list; CTAs past a layer's
+// count exit at once, so evicted tokens cost neither reads nor writes.
 #include "common.cuh"
 
 namespace semshare {
@@ -20,6 +26,15 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kTokens = 64;  // target tokens per CTA
 constexpr int kMaxSeg = 64;
+
+// Per-layer retained-token lists (ret[off[l] .. off[l+1]) for layer l), passed by value.
+template <int kMax>
+struct RetTable {
+    const int32_t* ret;
+    int64_t off[kMax + 1];
+};
+using NoRet = RetTable<1>;
+using Ret = RetTable<SEMSHARE_RETAIN_MAX_LAYERS>;
 
 struct GatherArgs {
     const uint8_t* src_k[kMaxSeg];
@@ -51,9 +66,48 @@ __device__ __forceinline__ void store_vec(void* p, const uint4& v) {
                  : "memory");
 }
 
+// Resolves the CTA's kTokens rows (segment, source offset; -1 = skip) into shared memory.
+// Returns false when the CTA has nothing to move (past its layer's retained count).
+template <bool kRetain, typename RT>
+__device__ __forceinline__ bool resolve_rows(const GatherArgs& a, const RT& rt, int l, int h, int64_t b, int64_t t0,
+                                             int64_t* s_src_off, int32_t* s_seg) {
+    int64_t count = a.n_tgt, base = 0;
+    if (kRetain) {
+        base = rt.off[l];
+        count = rt.off[l + 1] - base;
+        if (t0 >= count) return false;  // uniform over the CTA
+    }
+    if (threadIdx.x < kTokens) {
+        const int64_t t = t0 + threadIdx.x;
+        int32_t seg = -1;
+        int64_t off = 0;
+        if (t < count) {
+            int64_t tok = t;
+            bool ok = true;
+            if (kRetain) {
+                tok = __ldg(rt.ret + base + t);
+                ok = tok >= 0 && tok < a.n_tgt;
+            }
+            const int64_t r = ok ? __ldg(a.idx + b * a.n_tgt + tok) : -1;
+            if (ok && r >= 0 && r < a.seg_off[a.n_seg]) {
+                seg = 0;
+                while (r >= a.seg_off[seg + 1]) ++seg;
+                off = l * a.s_layer + h * a.s_head + (r - a.seg_off[seg]) * a.s_token;
+            } else if (a.err_flag) {
+                atomicOr(a.err_flag, SEMSHARE_FLAG_INDEX);
+            }
+        }
+        s_seg[threadIdx.x] = seg;
+        s_src_off[threadIdx.x] = off;
+    }
+    __syncthreads();
+    return true;
+}
+
 // C = 16-byte chunks per row (row_bytes / 16).
-template <int C>
-__global__ void __launch_bounds__(kThreads) kv_gather_kernel(const __grid_constant__ GatherArgs a) {
+template <int C, bool kRetain, typename RT>
+__global__ void __launch_bounds__(kThreads)
+    kv_gather_kernel(const __grid_constant__ GatherArgs a, const __grid_constant__ RT rt) {
     constexpr int kRowsPerPass = kThreads / C;
     constexpr int kPasses = 2 * kTokens / kRowsPerPass;  // K rows then V rows
     static_assert(kThreads % C == 0 && (2 * kTokens) % kRowsPerPass == 0, "row split");
@@ -66,25 +120,7 @@ __global__ void __launch_bounds__(kThreads) kv_gather_kernel(const __grid_consta
     const int l = static_cast<int>((plane / a.n_heads) % a.n_layers);
     const int64_t b = plane / (static_cast<int64_t>(a.n_heads) * a.n_layers);
     const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kTokens;
-
-    if (threadIdx.x < kTokens) {
-        const int64_t t = t0 + threadIdx.x;
-        int32_t seg = -1;
-        int64_t off = 0;
-        if (t < a.n_tgt) {
-            const int64_t r = __ldg(a.idx + b * a.n_tgt + t);
-            if (r >= 0 && r < a.seg_off[a.n_seg]) {
-                seg = 0;
-                while (r >= a.seg_off[seg + 1]) ++seg;
-                off = l * a.s_layer + h * a.s_head + (r - a.seg_off[seg]) * a.s_token;
-            } else if (a.err_flag) {
-                atomicOr(a.err_flag, SEMSHARE_FLAG_INDEX);
-            }
-        }
-        s_seg[threadIdx.x] = seg;
-        s_src_off[threadIdx.x] = off;
-    }
-    __syncthreads();
+    if (!resolve_rows<kRetain>(a, rt, l, h, b, t0, s_src_off, s_seg)) return;
 
     const int c = threadIdx.x % C;
     const int rr = threadIdx.x / C;
@@ -113,7 +149,9 @@ __global__ void __launch_bounds__(kThreads) kv_gather_kernel(const __grid_consta
 
 // Rows whose size is not a power-of-two number of 16-byte chunks: one chunk per thread per
 // step over the CTA's rows.
-__global__ void __launch_bounds__(kThreads) kv_gather_generic_kernel(const __grid_constant__ GatherArgs a, int chunks) {
+template <bool kRetain, typename RT>
+__global__ void __launch_bounds__(kThreads)
+    kv_gather_generic_kernel(const __grid_constant__ GatherArgs a, const __grid_constant__ RT rt, int chunks) {
     __shared__ int64_t s_src_off[kTokens];
     __shared__ int32_t s_seg[kTokens];
     const int64_t plane = blockIdx.y + static_cast<int64_t>(gridDim.y) * blockIdx.z;
@@ -121,24 +159,7 @@ __global__ void __launch_bounds__(kThreads) kv_gather_generic_kernel(const __gri
     const int l = static_cast<int>((plane / a.n_heads) % a.n_layers);
     const int64_t b = plane / (static_cast<int64_t>(a.n_heads) * a.n_layers);
     const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kTokens;
-    if (threadIdx.x < kTokens) {
-        const int64_t t = t0 + threadIdx.x;
-        int32_t seg = -1;
-        int64_t off = 0;
-        if (t < a.n_tgt) {
-            const int64_t r = __ldg(a.idx + b * a.n_tgt + t);
-            if (r >= 0 && r < a.seg_off[a.n_seg]) {
-                seg = 0;
-                while (r >= a.seg_off[seg + 1]) ++seg;
-                off = l * a.s_layer + h * a.s_head + (r - a.seg_off[seg]) * a.s_token;
-            } else if (a.err_flag) {
-                atomicOr(a.err_flag, SEMSHARE_FLAG_INDEX);
-            }
-        }
-        s_seg[threadIdx.x] = seg;
-        s_src_off[threadIdx.x] = off;
-    }
-    __syncthreads();
+    if (!resolve_rows<kRetain>(a, rt, l, h, b, t0, s_src_off, s_seg)) return;
     const int64_t dst_plane = b * a.d_batch + l * a.d_layer + h * a.d_head;
     const int total = 2 * kTokens * chunks;
     for (int e = threadIdx.x; e < total; e += kThreads) {
@@ -154,17 +175,12 @@ __global__ void __launch_bounds__(kThreads) kv_gather_generic_kernel(const __gri
 
 bool stride_ok(int64_t s, int64_t elem) { return s >= 0 && ((s * elem) % 16) == 0; }
 
-}  // namespace
-}  // namespace semshare
-
-extern "C" semshare_status semshare_gather_kv(const void* const* ref_k, const void* const* ref_v,
-                                              const int64_t* seg_offsets, int32_t n_seg, semshare_kv_layout src,
-                                              const int32_t* idx, int64_t n_tgt, int32_t n_batch, void* out_k,
-                                              void* out_v, semshare_kv_layout dst, uint32_t* err_flag,
-                                              void* stream) {
-    using namespace semshare;
+// Validates the arguments shared by both entry points and fills `a` (n_batch, n_tgt, idx set
+// by the caller).
+semshare_status build_args(const void* const* ref_k, const void* const* ref_v, const int64_t* seg_offsets,
+                           int32_t n_seg, const semshare_kv_layout& src, void* out_k, void* out_v,
+                           const semshare_kv_layout& dst, uint32_t* err_flag, GatherArgs* a) {
     if (n_seg < 1 || n_seg > kMaxSeg || !ref_k || !ref_v || !seg_offsets) return SEMSHARE_EINVAL;
-    if (n_tgt < 0 || n_batch < 0) return SEMSHARE_EINVAL;
     if (src.n_layers < 1 || src.n_heads < 1 || src.head_dim < 1) return SEMSHARE_EINVAL;
     if (src.elem_bytes != 1 && src.elem_bytes != 2 && src.elem_bytes != 4 && src.elem_bytes != 8)
         return SEMSHARE_EINVAL;
@@ -185,36 +201,31 @@ extern "C" semshare_status semshare_gather_kv(const void* const* ref_k, const vo
             return SEMSHARE_EINVAL;
     }
     if (seg_offsets[n_seg] >= (int64_t(1) << 31)) return SEMSHARE_EUNSUPPORTED;
-    if (n_tgt == 0 || n_batch == 0) return SEMSHARE_OK;
-    if (!idx || !out_k || !out_v || !aligned(idx, 4) || !aligned(out_k, 16) || !aligned(out_v, 16) ||
-        (err_flag && !aligned(err_flag, 4)))
-        return SEMSHARE_EINVAL;
-
-    GatherArgs a{};
     for (int s = 0; s < n_seg; ++s) {
-        a.src_k[s] = static_cast<const uint8_t*>(ref_k[s]);
-        a.src_v[s] = static_cast<const uint8_t*>(ref_v[s]);
+        a->src_k[s] = static_cast<const uint8_t*>(ref_k[s]);
+        a->src_v[s] = static_cast<const uint8_t*>(ref_v[s]);
     }
-    for (int s = 0; s <= n_seg; ++s) a.seg_off[s] = seg_offsets[s];
-    a.n_seg = n_seg;
-    a.n_layers = src.n_layers;
-    a.n_heads = src.n_heads;
-    a.n_batch = n_batch;
-    a.n_tgt = n_tgt;
-    a.s_layer = src.stride_layer * eb;
-    a.s_head = src.stride_head * eb;
-    a.s_token = src.stride_token * eb;
-    a.d_batch = dst.stride_batch * eb;
-    a.d_layer = dst.stride_layer * eb;
-    a.d_head = dst.stride_head * eb;
-    a.d_token = dst.stride_token * eb;
-    a.idx = idx;
-    a.dst_k = static_cast<uint8_t*>(out_k);
-    a.dst_v = static_cast<uint8_t*>(out_v);
-    a.err_flag = err_flag;
+    for (int s = 0; s <= n_seg; ++s) a->seg_off[s] = seg_offsets[s];
+    a->n_seg = n_seg;
+    a->n_layers = src.n_layers;
+    a->n_heads = src.n_heads;
+    a->s_layer = src.stride_layer * eb;
+    a->s_head = src.stride_head * eb;
+    a->s_token = src.stride_token * eb;
+    a->d_batch = dst.stride_batch * eb;
+    a->d_layer = dst.stride_layer * eb;
+    a->d_head = dst.stride_head * eb;
+    a->d_token = dst.stride_token * eb;
+    a->dst_k = static_cast<uint8_t*>(out_k);
+    a->dst_v = static_cast<uint8_t*>(out_v);
+    a->err_flag = err_flag;
+    return SEMSHARE_OK;
+}
 
-    const int64_t planes = static_cast<int64_t>(n_batch) * src.n_layers * src.n_heads;
-    const int64_t tblocks = (n_tgt + kTokens - 1) / kTokens;
+template <bool kRetain, typename RT>
+semshare_status launch_gather(const GatherArgs& a, const RT& rt, int64_t planes, int64_t tokens, int64_t row_bytes,
+                              cudaStream_t s) {
+    const int64_t tblocks = (tokens + kTokens - 1) / kTokens;
     if (tblocks > 0x7FFFFFFF) return SEMSHARE_EUNSUPPORTED;
     // planes tile the (y, z) grid exactly: y = the largest divisor of planes within 65535
     int64_t gy = planes < 65535 ? planes : 65535;
@@ -222,13 +233,72 @@ extern "C" semshare_status semshare_gather_kv(const void* const* ref_k, const vo
     if (planes / gy > 65535) return SEMSHARE_EUNSUPPORTED;
     const dim3 grid(static_cast<unsigned>(tblocks), static_cast<unsigned>(gy), static_cast<unsigned>(planes / gy));
     const int chunks = static_cast<int>(row_bytes / 16);
-    cudaStream_t s = as_stream(stream);
     switch (chunks) {
-        case 4: kv_gather_kernel<4><<<grid, kThreads, 0, s>>>(a); break;
-        case 8: kv_gather_kernel<8><<<grid, kThreads, 0, s>>>(a); break;
-        case 16: kv_gather_kernel<16><<<grid, kThreads, 0, s>>>(a); break;
-        case 32: kv_gather_kernel<32><<<grid, kThreads, 0, s>>>(a); break;
-        default: kv_gather_generic_kernel<<<grid, kThreads, 0, s>>>(a, chunks); break;
+        case 4: kv_gather_kernel<4, kRetain><<<grid, kThreads, 0, s>>>(a, rt); break;
+        case 8: kv_gather_kernel<8, kRetain><<<grid, kThreads, 0, s>>>(a, rt); break;
+        case 16: kv_gather_kernel<16, kRetain><<<grid, kThreads, 0, s>>>(a, rt); break;
+        case 32: kv_gather_kernel<32, kRetain><<<grid, kThreads, 0, s>>>(a, rt); break;
+        default: kv_gather_generic_kernel<kRetain><<<grid, kThreads, 0, s>>>(a, rt, chunks); break;
     }
     return launch_status();
+}
+
+}  // namespace
+}  // namespace semshare
+
+extern "C" semshare_status semshare_gather_kv(const void* const* ref_k, const void* const* ref_v,
+                                              const int64_t* seg_offsets, int32_t n_seg, semshare_kv_layout src,
+                                              const int32_t* idx, int64_t n_tgt, int32_t n_batch, void* out_k,
+                                              void* out_v, semshare_kv_layout dst, uint32_t* err_flag,
+                                              void* stream) {
+    using namespace semshare;
+    if (n_tgt < 0 || n_batch < 0) return SEMSHARE_EINVAL;
+    GatherArgs a{};
+    const semshare_status st = build_args(ref_k, ref_v, seg_offsets, n_seg, src, out_k, out_v, dst, err_flag, &a);
+    if (st != SEMSHARE_OK) return st;
+    if (n_tgt == 0 || n_batch == 0) return SEMSHARE_OK;
+    if (!idx || !out_k || !out_v || !aligned(idx, 4) || !aligned(out_k, 16) || !aligned(out_v, 16) ||
+        (err_flag && !aligned(err_flag, 4)))
+        return SEMSHARE_EINVAL;
+    a.n_batch = n_batch;
+    a.n_tgt = n_tgt;
+    a.idx = idx;
+    NoRet none{};
+    const int64_t planes = static_cast<int64_t>(n_batch) * src.n_layers * src.n_heads;
+    return launch_gather<false>(a, none, planes, n_tgt, static_cast<int64_t>(src.head_dim) * src.elem_bytes,
+                                as_stream(stream));
+}
+
+extern "C" semshare_status semshare_gather_kv_retained(const void* const* ref_k, const void* const* ref_v,
+                                                       const int64_t* seg_offsets, int32_t n_seg,
+                                                       semshare_kv_layout src, const int32_t* idx, int64_t n_tgt,
+                                                       const int32_t* retained, const int64_t* ret_offsets,
+                                                       void* out_k, void* out_v, semshare_kv_layout dst,
+                                                       uint32_t* err_flag, void* stream) {
+    using namespace semshare;
+    if (n_tgt < 0 || !ret_offsets) return SEMSHARE_EINVAL;
+    if (src.n_layers > SEMSHARE_RETAIN_MAX_LAYERS) return SEMSHARE_EUNSUPPORTED;
+    GatherArgs a{};
+    const semshare_status st = build_args(ref_k, ref_v, seg_offsets, n_seg, src, out_k, out_v, dst, err_flag, &a);
+    if (st != SEMSHARE_OK) return st;
+    Ret rt{};
+    if (ret_offsets[0] != 0) return SEMSHARE_EINVAL;
+    int64_t longest = 0;
+    for (int l = 0; l < src.n_layers; ++l) {
+        const int64_t c = ret_offsets[l + 1] - ret_offsets[l];
+        if (c < 0) return SEMSHARE_EINVAL;
+        longest = c > longest ? c : longest;
+    }
+    for (int l = 0; l <= src.n_layers; ++l) rt.off[l] = ret_offsets[l];
+    if (longest == 0) return SEMSHARE_OK;
+    if (!retained || !idx || !out_k || !out_v || !aligned(retained, 4) || !aligned(idx, 4) || !aligned(out_k, 16) ||
+        !aligned(out_v, 16) || (err_flag && !aligned(err_flag, 4)))
+        return SEMSHARE_EINVAL;
+    rt.ret = retained;
+    a.n_batch = 1;
+    a.n_tgt = n_tgt;
+    a.idx = idx;
+    const int64_t planes = static_cast<int64_t>(src.n_layers) * src.n_heads;
+    return launch_gather<true>(a, rt, planes, longest, static_cast<int64_t>(src.head_dim) * src.elem_bytes,
+                               as_stream(stream));
 }

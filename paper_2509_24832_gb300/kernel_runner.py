@@ -64,8 +64,8 @@ def _retrieval(a, wl, e, pd, R, table, flag, dev):
 
 def main(argv=None):
     p = argparse.ArgumentParser()
-    p.add_argument("--kernel", choices=["hash", "match", "match_tc", "gather", "retrieve", "deviation", "select"],
-                   required=True)
+    p.add_argument("--kernel", choices=["hash", "match", "match_tc", "gather", "gather_retained", "retrieve",
+                                        "deviation", "select"], required=True)
     p.add_argument("--workload", default="llama8b-5k", choices=sorted(ALL))
     p.add_argument("--reps", type=int, default=3)
     a = p.parse_args(argv)
@@ -98,6 +98,19 @@ def main(argv=None):
             elif a.kernel == "match_tc":
                 for _ in range(a.reps):
                     ss.semshare_match_tc(tc, rc, idx=idx, dist=dist, err_flag=flag)
+            elif a.kernel == "gather_retained":
+                # the synthetic retention schedule of bench.py --retain (one prompt)
+                del e
+                k, v = workloads.kv_cache_device(wl, dev)
+                counts = ss.retain_counts(wl.n_tgt, workloads.retain_alphas(wl.n_layers))
+                ret = workloads.retained_tokens(wl.n_tgt, counts, wl.base_seed)
+                flat = torch.from_numpy(np.concatenate(ret)).to(dev)
+                offs = [0] + list(np.cumsum(counts))
+                out_k = torch.empty((wl.n_layers, wl.n_heads, counts[0], wl.head_dim), dtype=torch.bfloat16,
+                                    device=dev)
+                out_v = torch.empty_like(out_k)
+                for _ in range(a.reps):
+                    ss.semshare_gather_kv_retained(k, v, idx, flat, offs, out_k=out_k, out_v=out_v, err_flag=flag)
             elif a.kernel == "gather":
                 del e
                 segs = [workloads.kv_cache_device(wl, dev, segment=s) for s in range(wl.n_seg)]

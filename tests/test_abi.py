@@ -126,6 +126,27 @@ def test_retrieve_argument_errors(lib):
     assert lib.semshare_retrieve_workspace_size(10, 5, 1, 64) > lib.semshare_match_tc_workspace_size(10, 5, 64)
 
 
+def test_gather_retained_argument_errors(lib):
+    import paper_2509_24832_gb300 as ss
+
+    lay = ss.KVLayout(2, 4, 64, 2, 0, 4 * 100 * 64, 100 * 64, 64)
+    out = ss.KVLayout(2, 4, 64, 2, 0, 4 * 10 * 64, 10 * 64, 64)
+    pk = (ctypes.c_void_p * 1)(1 << 20)
+    offs = (ctypes.c_int64 * 2)(0, 100)
+    g = lib.semshare_gather_kv_retained
+
+    def ro(*v):
+        return (ctypes.c_int64 * len(v))(*v)
+
+    assert g(pk, pk, offs, 1, lay, FAKE, 10, FAKE, None, FAKE, FAKE, out, None, None) == 1        # no offsets
+    assert g(pk, pk, offs, 1, lay, FAKE, 10, FAKE, ro(1, 5, 9), FAKE, FAKE, out, None, None) == 1  # not from 0
+    assert g(pk, pk, offs, 1, lay, FAKE, 10, FAKE, ro(0, 5, 3), FAKE, FAKE, out, None, None) == 1  # decreasing
+    assert g(pk, pk, offs, 1, lay, None, 10, FAKE, ro(0, 5, 9), FAKE, FAKE, out, None, None) == 1  # no idx
+    deep = ss.KVLayout(129, 4, 64, 2, 0, 4 * 100 * 64, 100 * 64, 64)
+    assert g(pk, pk, offs, 1, deep, FAKE, 10, FAKE, ro(*([0] * 130)), FAKE, FAKE, deep, None, None) == 2
+    assert g(pk, pk, offs, 1, lay, None, 10, None, ro(0, 0, 0), None, None, out, None, None) == 0  # nothing kept
+
+
 def test_deviation_and_select_argument_errors(lib):
     import paper_2509_24832_gb300 as ss
 

@@ -278,3 +278,17 @@ def recomputed_kv_device(wl: Workload, device, k_ref, v_ref, src, seed: int | No
         x = torch.where(copied.view(1, 1, -1, 1), base + noise * x, x)
         out.append(x.to(torch.bfloat16).contiguous())
     return out[0], out[1]
+
+
+# Retention schedule for the synthetic workloads (Sec. 3.3.4, App. A: alpha_retain larger in
+# shallow layers, smaller in deep ones; the first layer keeps max(0.8, r_dynamic)): 0.8 on the
+# first layer, then 0.98 per layer.
+def retain_alphas(n_layers: int) -> list:
+    return [0.8] + [0.98] * (n_layers - 1)
+
+
+def retained_tokens(n_tok: int, counts, seed: int) -> list:
+    """Nested retained sets: a seeded ranking of the target tokens stands in for the attention
+    scores; layer l keeps the counts[l] best-ranked tokens, listed in ascending order."""
+    rank = rng(seed, 200).permutation(n_tok)
+    return [np.sort(rank[:c]).astype(np.int32) for c in counts]
