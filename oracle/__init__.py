@@ -64,7 +64,9 @@ def _load():
         lib.oracle_theta.argtypes = [i32, i32, f64]
         lib.oracle_theta.restype = f64
         lib.oracle_rope.argtypes = [P, i64, i32, P, f64, P]
+        lib.oracle_rope_layout.argtypes = [P, i64, i32, P, f64, P, i32]
         lib.oracle_hash.argtypes = [P, i32, i64, i32, i64, P, f64, P, i32, P, P, i32]
+        lib.oracle_hash_layout.argtypes = [P, i32, i64, i32, i64, P, f64, P, i32, P, P, i32, i32]
         lib.oracle_hamming.argtypes = [P, P, i32]
         lib.oracle_hamming.restype = i32
         lib.oracle_match.argtypes = [P, i64, P, i64, i32, P, P]
@@ -102,18 +104,22 @@ def theta(k: int, d: int, base: float = 10000.0) -> float:
     return float(_load().oracle_theta(k, d, base))
 
 
-def rope(x: np.ndarray, positions, base: float = 10000.0) -> np.ndarray:
-    """fp64 rotary encoding of rows x[n][d] at the given positions (Eq. 1, Sec. 3.3.1)."""
+LAYOUTS = {"interleaved": 0, "half": 1}
+
+
+def rope(x: np.ndarray, positions, base: float = 10000.0, layout: str = "interleaved") -> np.ndarray:
+    """fp64 rotary encoding of rows x[n][d] at the given positions (Eq. 1, Sec. 3.3.1); pairs
+    (2k, 2k+1) as Eq. 1 prints them, or (k, k + d/2) with layout="half"."""
     x = np.ascontiguousarray(x, dtype=np.float64)
     n, d = x.shape
     pos = np.ascontiguousarray(np.broadcast_to(np.asarray(positions, dtype=np.int32), (n,)))
     y = np.empty_like(x)
-    _load().oracle_rope(_ptr(x), n, d, _ptr(pos), base, _ptr(y))
+    _load().oracle_rope_layout(_ptr(x), n, d, _ptr(pos), base, _ptr(y), LAYOUTS[layout])
     return y
 
 
 def hash_codes(emb: np.ndarray, positions, hyperplanes: np.ndarray, base: float = 10000.0,
-               round_operand: bool = True):
+               round_operand: bool = True, layout: str = "interleaved"):
     """LSH codes of embedding rows (Sec. 3.3, App. A.2).
 
     emb: [n][d] float32 rows, or uint16 bf16 bit patterns.  hyperplanes: [nbits][d] uint16 bf16.
@@ -133,8 +139,8 @@ def hash_codes(emb: np.ndarray, positions, hyperplanes: np.ndarray, base: float 
     pos = None if positions is None else np.ascontiguousarray(np.asarray(positions, dtype=np.int32).reshape(n))
     codes = np.zeros((n, nbits // 32), dtype=np.uint32)
     proj = np.zeros((n, nbits), dtype=np.float32)
-    _load().oracle_hash(_ptr(emb), f32, n, d, d, _ptr(pos), base, _ptr(R), nbits, _ptr(codes), _ptr(proj),
-                        1 if round_operand else 0)
+    _load().oracle_hash_layout(_ptr(emb), f32, n, d, d, _ptr(pos), base, _ptr(R), nbits, _ptr(codes), _ptr(proj),
+                               1 if round_operand else 0, LAYOUTS[layout])
     return codes, proj
 
 

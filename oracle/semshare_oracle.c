@@ -12,6 +12,7 @@
  *              to the E cache of both the reference and the target prompt; formula Eq. 1,
  *              App. A.1).  Pair (x[2k], x[2k+1]) of the row at position m is rotated by the
  *              angle m * theta_k, theta_k = base^(-2k/d), d = the embedding dimension.
+ *              A second pairing, (k, k + d/2) ("rotate-half"), is available as an option.
  *   2. hash    Random-hyperplane LSH (Sec. 3.3 "we use LSH", App. A.2, App. D "LSH from
  *              FAISS"): p_j = <r_j, y> for each of nbits hyperplanes r_j, code bit j = [p_j > 0],
  *              packed LSB-first into 32-bit words (bit j -> word j/32, bit j%32).
@@ -88,24 +89,33 @@ double oracle_theta(int32_t k, int32_t d, double base) {
     return pow(base, -2.0 * (double)k / (double)d);
 }
 
-static void rope_row(const double* x, int32_t d, double m, const double* theta, double* y) {
+/* Pair k of a row is (2k, 2k+1) as Eq. 1 prints it (half = 0), or (k, k + d/2), the
+ * "rotate-half" arrangement of common implementations (half = 1); either way it turns by
+ * m * theta_k. */
+static void rope_row(const double* x, int32_t d, double m, const double* theta, double* y, int32_t half) {
     for (int32_t k = 0; k < d / 2; ++k) {
         const double a = m * theta[k];
         const double c = cos(a), s = sin(a);
-        const double x0 = x[2 * k], x1 = x[2 * k + 1];
-        y[2 * k] = x0 * c - x1 * s;
-        y[2 * k + 1] = x0 * s + x1 * c;
+        const int32_t i0 = half ? k : 2 * k, i1 = half ? k + d / 2 : 2 * k + 1;
+        const double x0 = x[i0], x1 = x[i1];
+        y[i0] = x0 * c - x1 * s;
+        y[i1] = x0 * s + x1 * c;
     }
 }
 
-/* y[i] = RoPE(x[i], pos[i]) for n rows of width d (row-major, fp64). */
-void oracle_rope(const double* x, int64_t n, int32_t d, const int32_t* pos, double base, double* y) {
+/* y[i] = RoPE(x[i], pos[i]) for n rows of width d (row-major, fp64); half selects the pairing. */
+void oracle_rope_layout(const double* x, int64_t n, int32_t d, const int32_t* pos, double base, double* y,
+                        int32_t half) {
     double* theta = (double*)malloc(sizeof(double) * (size_t)(d / 2));
     for (int32_t k = 0; k < d / 2; ++k) theta[k] = oracle_theta(k, d, base);
 #pragma omp parallel for schedule(static)
     for (int64_t i = 0; i < n; ++i)
-        rope_row(x + i * d, d, (double)pos[i], theta, y + i * d);
+        rope_row(x + i * d, d, (double)pos[i], theta, y + i * d, half);
     free(theta);
+}
+
+void oracle_rope(const double* x, int64_t n, int32_t d, const int32_t* pos, double base, double* y) {
+    oracle_rope_layout(x, n, d, pos, base, y, 0);
 }
 
 /* ---- step 2: random-hyperplane LSH codes ----------------------------------------------- */
@@ -115,9 +125,9 @@ void oracle_rope(const double* x, int64_t n, int32_t d, const int32_t* pos, doub
  * hyperplanes: [nbits][d] bf16 bit patterns.  codes: [n][nbits/32] words.
  * proj (nullable): [n][nbits] float projections (the fp64 sum rounded to float).
  * round_operand = 1 applies the bf16 operand contract to y; 0 keeps y in fp64 (diagnostic). */
-void oracle_hash(const void* emb, int32_t emb_f32, int64_t n, int32_t d, int64_t row_stride,
-                 const int32_t* positions, double base, const uint16_t* hyperplanes, int32_t nbits,
-                 uint32_t* codes, float* proj, int32_t round_operand) {
+void oracle_hash_layout(const void* emb, int32_t emb_f32, int64_t n, int32_t d, int64_t row_stride,
+                        const int32_t* positions, double base, const uint16_t* hyperplanes, int32_t nbits,
+                        uint32_t* codes, float* proj, int32_t round_operand, int32_t half) {
     const int32_t w = nbits / 32;
     double* theta = (double*)malloc(sizeof(double) * (size_t)(d / 2));
     double* r = (double*)malloc(sizeof(double) * (size_t)nbits * (size_t)d);
@@ -134,7 +144,7 @@ void oracle_hash(const void* emb, int32_t emb_f32, int64_t n, int32_t d, int64_t
                 x[c] = emb_f32 ? (double)((const float*)emb)[i * row_stride + c]
                                : oracle_bf16_value(((const uint16_t*)emb)[i * row_stride + c]);
             const double m = positions ? (double)positions[i] : (double)i;
-            rope_row(x, d, m, theta, y);
+            rope_row(x, d, m, theta, y, half);
             if (round_operand)
                 for (int32_t c = 0; c < d; ++c) y[c] = oracle_bf16_value(oracle_bf16_round(y[c]));
             for (int32_t q = 0; q < w; ++q) codes[i * w + q] = 0u;
@@ -150,6 +160,13 @@ void oracle_hash(const void* emb, int32_t emb_f32, int64_t n, int32_t d, int64_t
     }
     free(theta);
     free(r);
+}
+
+void oracle_hash(const void* emb, int32_t emb_f32, int64_t n, int32_t d, int64_t row_stride,
+                 const int32_t* positions, double base, const uint16_t* hyperplanes, int32_t nbits,
+                 uint32_t* codes, float* proj, int32_t round_operand) {
+    oracle_hash_layout(emb, emb_f32, n, d, row_stride, positions, base, hyperplanes, nbits, codes, proj,
+                       round_operand, 0);
 }
 
 /* ---- step 3: Hamming nearest neighbour ------------------------------------------------- */
