@@ -53,7 +53,7 @@ L2_FLUSH_BYTES = 256 << 20
 NCU_TRAFFIC = {
     ("gather", "llama8b-5k"): {"file": "gather.cu", "sha": "7d05bda6e8a70170", "bytes_per_launch": 1092.7e6},
     ("gather_retained", "llama8b-5k"): {"file": "gather.cu", "sha": "7d05bda6e8a70170", "bytes_per_launch": 663.2e6},
-    ("hash", "llama8b-5k"): {"file": "hash.cu", "sha": "0fc6e508c36def23", "bytes_per_launch": 90.65e6},
+    ("hash", "llama8b-5k"): {"file": "hash.cu", "sha": "c9f57175642e48ea", "bytes_per_launch": 90.85e6},
     ("match", "llama8b-5k"): {"file": "match.cu", "sha": "69ac4b7ce5b193e4", "bytes_per_launch": 0.3845e6},
     ("match_tc", "llama8b-5k"): {"file": "match_tc.cu", "sha": "c494ec8dce435f1b", "bytes_per_launch": 2.736e6},
     ("retrieve", "retrieve-16x4096"): {"file": "match_tc.cu", "sha": "c494ec8dce435f1b", "bytes_per_launch": 18.42e6},
@@ -70,6 +70,8 @@ def parse_args(argv=None):
     p.add_argument("--matcher", default="tc", choices=["tc", "popc"],
                    help="Hamming search: tensor-core GEMM (semshare_match_tc) or xor/popc (semshare_match)")
     p.add_argument("--e2e-steps", type=int, default=20)
+    p.add_argument("--rope", default="interleaved", choices=["interleaved", "half"],
+                   help="rotary pairing: (2k, 2k+1) as Eq. 1 prints it, or (k, k + d/2)")
     p.add_argument("--retain", action="store_true",
                    help="gather only each layer's retained tokens (Sec. 3.3.4; synthetic schedule: 0.8 on the "
                         "first layer, then 0.98 per layer; one-prompt workloads)")
@@ -245,6 +247,7 @@ class Problem:
         import paper_2509_24832_gb300 as ss
 
         self.ss, self.wl, self.dev, self.matcher = ss, wl, device, matcher
+        self.rope_layout = "interleaved"
         emb, pos, src = workloads.prompt_rows(wl, seed=seed)
         self.host_emb, self.host_pos = emb, pos
         if wl.emb_dtype == "f32":
@@ -310,7 +313,7 @@ class Problem:
 
     def hash(self):
         self.ss.semshare_hash(self.emb, self.table, self.hyp, self.pos, codes=self.codes, err_flag=self.flag,
-                              workspace=self.hash_ws)
+                              workspace=self.hash_ws, rope_layout=self.rope_layout)
 
     def match(self):
         n_ref = self.wl.n_ref
@@ -588,6 +591,10 @@ def run_gpu_arm(args, rank, world, local_rank):
     wl = ALL_WORKLOADS[args.workload]
     seed = wl.base_seed + 7919 * rank
     prob = make_problem(wl, device, seed, args.matcher, with_hd=args.hd, with_retain=args.retain)
+    if args.rope != "interleaved":
+        if not isinstance(prob, Problem):
+            raise ValueError("--rope applies to the matching workloads")
+        prob.rope_layout = args.rope
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
     n_ev = len(prob.STAGES) + 1
 
@@ -654,6 +661,8 @@ def run_gpu_arm(args, rank, world, local_rank):
               "n_seg": wl.n_seg, "d": wl.d, "nbits": wl.nbits, "kv": list(wl.kv),
               "parallelism": f"replicas x{world}", "l2": "flushed before every step (256 MB write)",
               "matcher": args.matcher}
+    if args.rope != "interleaved":
+        config["rope"] = "pairs (k, k + d/2)"
     if args.retain:
         config["retain"] = (f"per-layer retained tokens, first {prob.counts[0]}, last {prob.counts[-1]}, "
                             f"{sum(prob.counts)} rows of {wl.n_layers * wl.n_tgt} (0.8, then 0.98 per layer)")

@@ -126,6 +126,23 @@ semshare_status semshare_rope_table(int32_t d, double rope_base, uint64_t* table
  * it depends on the current device (its SM count).
  */
 size_t semshare_hash_workspace_size(int64_t n, int32_t d, int32_t nbits);
+
+/*
+ * semshare_hash_ex -- semshare_hash with a choice of rotary pairing.
+ *
+ * rope_layout SEMSHARE_ROPE_INTERLEAVED: pairs (2k, 2k+1), as Eq. 1 prints them (semshare_hash);
+ *             SEMSHARE_ROPE_HALF: pairs (k, k + d/2) ("rotate-half", the arrangement of many
+ *             model implementations), each turned by the same angle m * theta_k and rounded to
+ *             bf16 the same way.  The rotation table is the same for both.
+ * SEMSHARE_ROPE_HALF takes bf16 rows and d a multiple of 128 (else EUNSUPPORTED).  Every other
+ * argument, and the result for SEMSHARE_ROPE_INTERLEAVED, as for semshare_hash.
+ */
+#define SEMSHARE_ROPE_INTERLEAVED 0u
+#define SEMSHARE_ROPE_HALF 1u
+semshare_status semshare_hash_ex(const void* emb, semshare_dtype dtype, int64_t n, int32_t d, int64_t row_stride,
+                                 const int32_t* positions, const uint64_t* rope_table, const uint16_t* hyperplanes,
+                                 int32_t nbits, uint32_t rope_layout, uint32_t* codes, float* proj_out,
+                                 void* workspace, size_t workspace_bytes, uint32_t* err_flag, void* stream);
 semshare_status semshare_hash(const void* emb, semshare_dtype dtype, int64_t n, int32_t d, int64_t row_stride,
                               const int32_t* positions, const uint64_t* rope_table, const uint16_t* hyperplanes,
                               int32_t nbits, uint32_t* codes, float* proj_out, void* workspace,

@@ -20,6 +20,7 @@ OK, EINVAL, EUNSUPPORTED, ECUDA, EINDEX, ETIMEOUT, ETOOLARGE = range(7)
 MATCH_STATIC_MAX_TARGETS = 262144
 FLAG_INDEX, FLAG_TIMEOUT = 1, 2
 BF16, F32 = 0, 1
+ROPE_LAYOUTS = {"interleaved": 0, "half": 1}
 
 _lock = threading.Lock()
 _lib = None
@@ -60,6 +61,9 @@ def load():
         lib.semshare_hash_workspace_size.restype = ctypes.c_size_t
         lib.semshare_hash.argtypes = [P, ctypes.c_int, i64, i32, i64, P, P, P, i32, P, P, P, ctypes.c_size_t, P, P]
         lib.semshare_hash.restype = ctypes.c_int
+        lib.semshare_hash_ex.argtypes = [P, ctypes.c_int, i64, i32, i64, P, P, P, i32, u32, P, P, P, ctypes.c_size_t,
+                                         P, P]
+        lib.semshare_hash_ex.restype = ctypes.c_int
         lib.semshare_match_workspace_size.argtypes = [i64]
         lib.semshare_match_workspace_size.restype = ctypes.c_size_t
         lib.semshare_match.argtypes = [P, i64, P, i64, i32, P, P, P, ctypes.c_size_t, P]
@@ -167,11 +171,12 @@ def hash_workspace(n: int, d: int, nbits: int, device=None) -> torch.Tensor:
 def semshare_hash(emb: torch.Tensor, rope_table: torch.Tensor, hyperplanes: torch.Tensor,
                   positions: torch.Tensor | None = None, codes: torch.Tensor | None = None,
                   proj_out: torch.Tensor | None = None, err_flag: torch.Tensor | None = None,
-                  workspace: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+                  workspace: torch.Tensor | None = None, stream=None, rope_layout: str = "interleaved") -> torch.Tensor:
     """LSH codes of RoPE-encoded rows.  emb [n][d] bf16/fp32 (rows may be strided),
     hyperplanes [nbits][d] bf16, positions [n] int32 (None: 0..n-1).  workspace: a zero-filled
-    uint8 device buffer (default: the per-device one of hash_workspace()).
-    Returns codes [n][nbits/32] int32 (uint32 bit patterns)."""
+    uint8 device buffer (default: the per-device one of hash_workspace()).  rope_layout:
+    "interleaved" (pairs (2k, 2k+1), Eq. 1) or "half" (pairs (k, k + d/2); bf16 rows, d a
+    multiple of 128).  Returns codes [n][nbits/32] int32 (uint32 bit patterns)."""
     _need_cuda(emb, "emb")
     _need_cuda(hyperplanes, "hyperplanes")
     if emb.dim() != 2 or emb.stride(1) != 1:
@@ -196,9 +201,11 @@ def semshare_hash(emb: torch.Tensor, rope_table: torch.Tensor, hyperplanes: torc
     if workspace is None:
         workspace = hash_workspace(n, d, nbits, emb.device)
     ws_bytes = workspace.numel() * workspace.element_size()
-    st = load().semshare_hash(_ptr(emb), dt, n, d, emb.stride(0), _ptr(positions), _ptr(rope_table),
-                              _ptr(hyperplanes), nbits, _ptr(codes), _ptr(proj_out), _ptr(workspace), ws_bytes,
-                              _ptr(err_flag), _stream(stream))
+    if rope_layout not in ROPE_LAYOUTS:
+        raise ValueError(f"rope_layout must be one of {sorted(ROPE_LAYOUTS)}")
+    st = load().semshare_hash_ex(_ptr(emb), dt, n, d, emb.stride(0), _ptr(positions), _ptr(rope_table),
+                                 _ptr(hyperplanes), nbits, ROPE_LAYOUTS[rope_layout], _ptr(codes), _ptr(proj_out),
+                                 _ptr(workspace), ws_bytes, _ptr(err_flag), _stream(stream))
     _check(st, "semshare_hash")
     return codes
 

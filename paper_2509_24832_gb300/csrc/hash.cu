@@ -32,6 +32,12 @@
 //                 32-bit words, or the partial-sum hand-off of a shared tile
 // Every pipeline wait is bounded; on timeout the CTA raises SEMSHARE_FLAG_TIMEOUT, lets its
 // copies and MMAs in flight finish, frees TMEM and returns.
+//
+// Rotate-half pairing (semshare_hash_ex, SEMSHARE_ROPE_HALF): pair k is (k, k + d/2).  A stage
+// then also loads the partner block (columns kb*64 +- d/2, the same 128-byte swizzled box) into
+// its staging slot, and the RoPE warps write each of the stage's own 64 columns from its own
+// value and its partner's: y = x*c - x_partner*s in the first half, x*c + x_partner*s in the
+// second, at angle index (column mod d/2).  The hyperplane tiles and the MMA are unchanged.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -111,6 +117,15 @@ __device__ __forceinline__ uint32_t rotate_to_bf16(float x0, float x1, float c, 
     return *reinterpret_cast<uint32_t*>(&r);
 }
 
+// The K block holding the rotate-half partners of block kb's columns (d/2 = nkb/2 blocks away).
+__device__ __forceinline__ int partner_kb(int kb, int nkb) { return kb < nkb / 2 ? kb + nkb / 2 : kb - nkb / 2; }
+
+// Rotate-half outputs of one column from its own value and its partner's (the two lines of the
+// pair rotation, with the operands in the order the column takes in the pair).
+__device__ __forceinline__ float rotate_half_col(float own, float partner, float c, float s, bool first_half) {
+    return first_half ? fmaf(own, c, -partner * s) : fmaf(partner, s, own * c);
+}
+
 __device__ __forceinline__ bool drain_wait(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = global_timer_ns();
@@ -136,6 +151,25 @@ __device__ __forceinline__ bool epilogue_all(bool v) {
         : "r"(static_cast<uint32_t>(v)), "n"(kEpiBarrier), "n"(kEpiWarps * 32)
         : "memory");
     return r != 0;
+}
+
+// Table entries of 8 consecutive angle indices j0 .. j0+7 (rotate-half pairing).
+struct Pairs8 {
+    uint64_t turns[8];
+    uint64_t cis32[8];
+};
+
+__device__ __forceinline__ void load_pairs8(const uint64_t* table, int half, int j0, Pairs8& t) {
+    const ulonglong2* tp = reinterpret_cast<const ulonglong2*>(table + j0);
+    const ulonglong2* cp = reinterpret_cast<const ulonglong2*>(table + half + j0);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const ulonglong2 a = __ldg(tp + i), b = __ldg(cp + i);
+        t.turns[2 * i] = a.x;
+        t.turns[2 * i + 1] = a.y;
+        t.cis32[2 * i] = b.x;
+        t.cis32[2 * i + 1] = b.y;
+    }
 }
 
 // Table entries of the 4 pairs (kb*32 + 4c .. +3): turn fractions, and the rotation between
@@ -182,6 +216,7 @@ __device__ __forceinline__ void store_codes(uint32_t* codes, int64_t row, int W,
     }
 }
 
+template <bool kHalf>
 __global__ void __launch_bounds__(kThreads, 1)
     lsh_hash_kernel(const __grid_constant__ CUtensorMap tmap_emb, const __grid_constant__ CUtensorMap tmap_hyp,
                     const HashArgs a) {
@@ -254,6 +289,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (pf_it >= i1) return;
                 tma_prefetch_l2_2d(&tmap_emb, pf_kb * kBK, pf_tile * kBM);
                 if (a.is_f32) tma_prefetch_l2_2d(&tmap_emb, pf_kb * kBK + 32, pf_tile * kBM);
+                if (kHalf) tma_prefetch_l2_2d(&tmap_emb, partner_kb(pf_kb, nkb) * kBK, pf_tile * kBM);
                 ++pf_it;
                 if (++pf_kb == nkb) {
                     pf_kb = 0;
@@ -277,6 +313,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tma_load_2d(stg + kF32Bytes / 2, &tmap_emb, full, kb * kBK + 32, tile * kBM);
                 } else {
                     tma_load_2d(st, &tmap_emb, full, kb * kBK, tile * kBM);
+                    if (kHalf) tma_load_2d(st + kABytes + a.b_bytes, &tmap_emb, full, partner_kb(kb, nkb) * kBK,
+                                           tile * kBM);
                 }
                 tma_load_2d(st + kABytes, &tmap_hyp, full, kb * kBK, 0);
                 prefetch_next();
@@ -334,7 +372,90 @@ __global__ void __launch_bounds__(kThreads, 1)
             drain_wait(bar_mma_done, 0, kWaitLimitNs);
         }
         __syncwarp();
-    } else if (warp >= kRopeWarp0 && warp < kRopeWarp0 + kRopeWarps) {
+    } else if (kHalf && warp >= kRopeWarp0 && warp < kRopeWarp0 + kRopeWarps) {
+        // ---------------- RoPE, rotate-half pairing ----------------
+        // A thread owns the 8 columns of one 16-byte chunk (c) of 4 rows 32 apart; their partners
+        // sit at the same place in the staged partner block.
+        const int rt = threadIdx.x - kRopeWarp0 * 32;
+        const int c = rt & 7;
+        const int rg = rt >> 3;
+        const uint32_t chunk_off = (static_cast<uint32_t>(c) ^ static_cast<uint32_t>(rg & 7)) << 4;
+        const int hk = nkb / 2;
+        const int half = nkb * (kBK / 2);
+        uint32_t q = 0;
+        int tile = static_cast<int>(i0 / nkb), kb = static_cast<int>(i0 % nkb), cur_tile = -1;
+        uint32_t m[4] = {0u, 0u, 0u, 0u};
+        bool steps32 = false;
+        Pairs8 tn;
+        load_pairs8(a.rope_table, half, (kb % hk) * kBK + 8 * c, tn);
+        for (int64_t it = i0; it < i1; ++it, ++q) {
+            if (tile != cur_tile) {
+                cur_tile = tile;
+                const int64_t r0 = static_cast<int64_t>(tile) * kBM + rg;
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int64_t row = r0 + 32 * i;
+                    m[i] = row < a.n ? (a.positions ? static_cast<uint32_t>(__ldg(a.positions + row))
+                                                    : static_cast<uint32_t>(row))
+                                     : m[0] + 32u * i;
+                }
+                steps32 = m[1] == m[0] + 32u && m[2] == m[0] + 64u && m[3] == m[0] + 96u;
+            }
+            const Pairs8 tc = tn;
+            const bool first_half = kb < hk;
+            const int kb_next = kb + 1 == nkb ? 0 : kb + 1;
+            if (it + 1 < i1) load_pairs8(a.rope_table, half, (kb_next % hk) * kBK + 8 * c, tn);
+
+            const uint32_t s = q % S, ph = (q / S) & 1u;
+            const bool got = mbar_wait_bounded(bar_full + 8u * s, ph, abort_flag, a.err_flag, SEMSHARE_FLAG_TIMEOUT,
+                                               a.wait_limit_ns);
+            if (!__all_sync(0xFFFFFFFFu, got)) break;
+            uint8_t* const st = gbase + s * a.stage_bytes;
+            const uint8_t* const pt = st + kABytes + a.b_bytes;  // partner block
+            float cs[8], sn[8];
+            if (steps32) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) rotation(m[0], tc.turns[e], cs[e], sn[e]);
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const uint32_t off = (rg + 32 * i) * 128 + chunk_off;
+                const uint4 vo = *reinterpret_cast<const uint4*>(st + off);
+                const uint4 vp = *reinterpret_cast<const uint4*>(pt + off);
+                const uint32_t wo[4] = {vo.x, vo.y, vo.z, vo.w}, wp[4] = {vp.x, vp.y, vp.z, vp.w};
+                if (!steps32) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) rotation(m[i], tc.turns[e], cs[e], sn[e]);
+                }
+                uint32_t y[4];
+#pragma unroll
+                for (int w = 0; w < 4; ++w) {
+                    const float o0 = __uint_as_float(wo[w] << 16), o1 = __uint_as_float(wo[w] & 0xFFFF0000u);
+                    const float p0 = __uint_as_float(wp[w] << 16), p1 = __uint_as_float(wp[w] & 0xFFFF0000u);
+                    const float y0 = rotate_half_col(o0, p0, cs[2 * w], sn[2 * w], first_half);
+                    const float y1 = rotate_half_col(o1, p1, cs[2 * w + 1], sn[2 * w + 1], first_half);
+                    __nv_bfloat162 r = __floats2bfloat162_rn(y0, y1);
+                    y[w] = *reinterpret_cast<uint32_t*>(&r);
+                }
+                *reinterpret_cast<uint4*>(st + off) = make_uint4(y[0], y[1], y[2], y[3]);
+                if (steps32 && i < 3) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const float c32 = __uint_as_float(static_cast<uint32_t>(tc.cis32[e]));
+                        const float s32 = __uint_as_float(static_cast<uint32_t>(tc.cis32[e] >> 32));
+                        const float nc = fmaf(cs[e], c32, -sn[e] * s32);
+                        sn[e] = fmaf(cs[e], s32, sn[e] * c32);
+                        cs[e] = nc;
+                    }
+                }
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_ready + 8u * s);
+            kb = kb_next;
+            if (kb == 0) ++tile;
+        }
+    } else if (!kHalf && warp >= kRopeWarp0 && warp < kRopeWarp0 + kRopeWarps) {
         // ---------------- RoPE (Eq. 1) on the staged tile ----------------
         const int rt = threadIdx.x - kRopeWarp0 * 32;  // 0..255
         const int c = rt & 7;                          // 16-byte chunk of the 128-byte row: pairs 4c..4c+3
@@ -659,13 +780,16 @@ extern "C" size_t semshare_hash_workspace_size(int64_t n, int32_t d, int32_t nbi
     return p.partial_bytes + p.count_bytes;
 }
 
-extern "C" semshare_status semshare_hash(const void* emb, semshare_dtype dtype, int64_t n, int32_t d,
-                                         int64_t row_stride, const int32_t* positions, const uint64_t* rope_table,
-                                         const uint16_t* hyperplanes, int32_t nbits, uint32_t* codes,
-                                         float* proj_out, void* workspace, size_t workspace_bytes,
-                                         uint32_t* err_flag, void* stream) {
+extern "C" semshare_status semshare_hash_ex(const void* emb, semshare_dtype dtype, int64_t n, int32_t d,
+                                            int64_t row_stride, const int32_t* positions, const uint64_t* rope_table,
+                                            const uint16_t* hyperplanes, int32_t nbits, uint32_t rope_layout,
+                                            uint32_t* codes, float* proj_out, void* workspace,
+                                            size_t workspace_bytes, uint32_t* err_flag, void* stream) {
     using namespace semshare;
     if (dtype != SEMSHARE_BF16 && dtype != SEMSHARE_F32) return SEMSHARE_EINVAL;
+    if (rope_layout != SEMSHARE_ROPE_INTERLEAVED && rope_layout != SEMSHARE_ROPE_HALF) return SEMSHARE_EINVAL;
+    const bool half = rope_layout == SEMSHARE_ROPE_HALF;
+    if (half && (dtype != SEMSHARE_BF16 || d % (2 * kBK) != 0)) return SEMSHARE_EUNSUPPORTED;
     if (n < 0 || d <= 0 || (d & 1) || row_stride < d) return SEMSHARE_EINVAL;
     if (d % kBK != 0 || d > 65536) return SEMSHARE_EUNSUPPORTED;
     if (nbits < 32 || nbits > 256 || nbits % 32 != 0) return SEMSHARE_EUNSUPPORTED;
@@ -697,8 +821,9 @@ extern "C" semshare_status semshare_hash(const void* emb, semshare_dtype dtype, 
     a.n_tiles = static_cast<int32_t>(plan.n_tiles);
     a.is_f32 = dtype == SEMSHARE_F32;
     a.b_bytes = static_cast<uint32_t>(nbits) * kBK * 2;
-    a.stage_bytes = kABytes + a.b_bytes + (a.is_f32 ? kF32Bytes : 0u);
-    a.tx_bytes = (a.is_f32 ? kF32Bytes : kABytes) + a.b_bytes;
+    // the staging slot after the hyperplane block: fp32 rows, or the rotate-half partner block
+    a.stage_bytes = kABytes + a.b_bytes + (a.is_f32 ? kF32Bytes : (half ? kABytes : 0u));
+    a.tx_bytes = (a.is_f32 ? kF32Bytes : kABytes) + a.b_bytes + (half ? kABytes : 0u);
     uint32_t cols = 32;
     while (cols < 2u * static_cast<uint32_t>(nbits)) cols <<= 1;
     a.tmem_cols = cols;
@@ -728,9 +853,18 @@ extern "C" semshare_status semshare_hash(const void* emb, semshare_dtype dtype, 
                    static_cast<uint64_t>(nbits), static_cast<uint64_t>(d) * 2, 64u, static_cast<uint32_t>(nbits)))
         return SEMSHARE_ECUDA;
 
-    if (cudaFuncSetAttribute(lsh_hash_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
-        cudaSuccess)
+    auto kernel = half ? lsh_hash_kernel<true> : lsh_hash_kernel<false>;
+    if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) != cudaSuccess)
         return SEMSHARE_ECUDA;
-    lsh_hash_kernel<<<plan.grid, kThreads, smem, as_stream(stream)>>>(tm_emb, tm_hyp, a);
+    kernel<<<plan.grid, kThreads, smem, as_stream(stream)>>>(tm_emb, tm_hyp, a);
     return launch_status();
+}
+
+extern "C" semshare_status semshare_hash(const void* emb, semshare_dtype dtype, int64_t n, int32_t d,
+                                         int64_t row_stride, const int32_t* positions, const uint64_t* rope_table,
+                                         const uint16_t* hyperplanes, int32_t nbits, uint32_t* codes,
+                                         float* proj_out, void* workspace, size_t workspace_bytes,
+                                         uint32_t* err_flag, void* stream) {
+    return semshare_hash_ex(emb, dtype, n, d, row_stride, positions, rope_table, hyperplanes, nbits,
+                            SEMSHARE_ROPE_INTERLEAVED, codes, proj_out, workspace, workspace_bytes, err_flag, stream);
 }

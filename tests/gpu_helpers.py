@@ -39,15 +39,20 @@ def unpack_bits(codes: np.ndarray) -> np.ndarray:
 GPU_ROPE_REL_ERR = 3e-6
 
 
-def operand_flip_allowance(orc, emb, pos, R):
+def operand_flip_allowance(orc, emb, pos, R, layout="interleaved"):
     """Per projection, the largest change bf16 operand rounding can make when the GPU's y
     differs from the exact y by up to GPU_ROPE_REL_ERR of its pair norm: only elements that
     close to a bf16 rounding midpoint can round the other way, each by one bf16 ulp.
     Returns [n][nbits] float64 (added to the projection tolerance and the code band)."""
     x = emb.astype(np.float64) if emb.dtype == np.float32 else \
         (emb.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
-    y = orc.rope(x, np.arange(len(x)) if pos is None else pos)
-    pair = np.repeat(np.hypot(y[:, 0::2], y[:, 1::2]), 2, axis=1)
+    y = orc.rope(x, np.arange(len(x)) if pos is None else pos, layout=layout)
+    if layout == "half":
+        h = y.shape[1] // 2
+        pn = np.hypot(y[:, :h], y[:, h:])
+        pair = np.concatenate([pn, pn], axis=1)
+    else:
+        pair = np.repeat(np.hypot(y[:, 0::2], y[:, 1::2]), 2, axis=1)
     ay = np.abs(y)
     e = np.floor(np.log2(np.maximum(ay, 1e-300)))
     ulp = np.exp2(e - 7)                      # bf16: 8 significant bits

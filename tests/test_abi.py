@@ -75,6 +75,17 @@ def test_hash_argument_errors(lib):
     assert _hash(lib, n=0, emb=None, codes=None) == 0    # empty: nothing to do
 
 
+def test_hash_ex_argument_errors(lib):
+    def hx(layout, dtype=0, d=128):
+        return lib.semshare_hash_ex(FAKE, dtype, 10, d, d, None, FAKE, FAKE, 64, layout, FAKE, None, FAKE, 1 << 30,
+                                    None, None)
+    assert hx(2) == 1                    # unknown pairing
+    assert hx(1, dtype=1) == 2           # rotate-half takes bf16 rows
+    assert hx(1, d=192) == 2             # and d a multiple of 128
+    assert lib.semshare_hash_ex(None, 0, 0, 128, 128, None, None, None, 64, 1, None, None, None, 0, None,
+                                None) == 0  # empty
+
+
 def test_match_argument_errors(lib):
     m = lib.semshare_match
     assert m(FAKE, 10, FAKE, 0, 64, FAKE, None, FAKE, 80, None) == 1   # n_ref = 0
