@@ -11,6 +11,7 @@ namespace {
 //   table[d/2 + k]     cos(32*theta_k) and sin(32*theta_k) as two floats (low word: cos): the
 //                      rotation between positions 32 apart, for stepping from one row to another
 __global__ void rope_table_kernel(int32_t d, double base, uint64_t* __restrict__ table) {
+    pdl_prologue();
     const int32_t k = blockIdx.x * blockDim.x + threadIdx.x;
     if (k >= d / 2) return;
     const double theta = pow(base, -2.0 * static_cast<double>(k) / static_cast<double>(d));
@@ -53,6 +54,8 @@ extern "C" semshare_status semshare_rope_table(int32_t d, double rope_base, uint
     if (!(rope_base > 0.0) || !(rope_base < 1e300)) return SEMSHARE_EINVAL;
     if (table == nullptr || !aligned(table, 16)) return SEMSHARE_EINVAL;
     const int32_t pairs = d / 2;
-    rope_table_kernel<<<(pairs + 255) / 256, 256, 0, as_stream(stream)>>>(d, rope_base, table);
+    if (launch_pdl(rope_table_kernel, dim3(static_cast<unsigned>((pairs + 255) / 256)), dim3(256), 0, as_stream(stream),
+                   d, rope_base, table) != cudaSuccess)
+        return SEMSHARE_ECUDA;
     return launch_status();
 }

@@ -5,6 +5,7 @@
 
 #include <cstdint>
 #include <cstdlib>
+#include <utility>
 
 #include "semshare.h"
 
@@ -23,6 +24,39 @@ inline semshare_status current_sm_count(int* sms, int* device) {
     *sms = n;
     if (device) *device = dev;
     return SEMSHARE_OK;
+}
+
+// Programmatic dependent launch.  grid_dependency_wait: returns once every grid this one depends
+// on has completed and its memory is visible (immediately when launched without the programmatic
+// attribute).  grid_dependents_launch: lets the next grid in the stream be scheduled once every
+// CTA of this grid has executed it (or exited); that grid still waits for this one to complete
+// before touching memory.
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dependents_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// Every kernel of the library starts with this pair: nothing before it touches global memory.
+__device__ __forceinline__ void pdl_prologue() {
+    grid_dependency_wait();
+    grid_dependents_launch();
+}
+
+// Launches kernel<<<grid, block, smem, s>>>(args...) as a programmatic dependent of the work
+// before it in the stream: its CTAs may be scheduled while the previous kernel drains, and they
+// wait (griddepcontrol.wait, first thing in every kernel of the library) until it has completed.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                              Args&&... args) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
 inline semshare_status launch_status() {

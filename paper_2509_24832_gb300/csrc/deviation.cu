@@ -117,6 +117,7 @@ __device__ __forceinline__ void deviation_of_token(const DevArgs& a, int64_t w, 
 
 // Grid-stride over (layer, token) items, one warp each; the grid is the resident CTAs.
 __global__ void __launch_bounds__(kDevThreads) kv_deviation_kernel(const DevArgs a) {
+    pdl_prologue();
     const int lane = threadIdx.x & 31;
     const int64_t n_items = static_cast<int64_t>(a.n_layers) * a.n_tok;
     const int64_t n_warps = static_cast<int64_t>(gridDim.x) * (kDevThreads / 32);
@@ -163,6 +164,7 @@ template <bool kStaged>
 __global__ void __launch_bounds__(kSelThreads)
     hd_select_kernel(const float* __restrict__ sigma, int64_t n_tok, int64_t k, int32_t* __restrict__ hd_idx,
                      uint8_t* __restrict__ hd_mask) {
+    pdl_prologue();
     extern __shared__ uint32_t staged[];
     __shared__ unsigned int hist[256];
     __shared__ int warp_tot[kSelThreads / 32];
@@ -333,7 +335,9 @@ extern "C" semshare_status semshare_kv_deviation(const void* k_reused, const voi
     const int64_t need = (warps * 32 + kDevThreads - 1) / kDevThreads;
     const int64_t resident = static_cast<int64_t>(sms) * (per_sm > 0 ? per_sm : 1);
     const int64_t grid = need < resident ? need : resident;
-    kv_deviation_kernel<<<static_cast<unsigned>(grid), kDevThreads, 0, as_stream(stream)>>>(a);
+    if (launch_pdl(kv_deviation_kernel, dim3(static_cast<unsigned>(grid)), dim3(kDevThreads), 0, as_stream(stream), a) !=
+        cudaSuccess)
+        return SEMSHARE_ECUDA;
     return launch_status();
 }
 
@@ -356,9 +360,13 @@ extern "C" semshare_status semshare_select_hd(const float* sigma, int32_t n_laye
         if (stage > 48 * 1024 && cudaFuncSetAttribute(hd_select_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                       static_cast<int>(stage)) != cudaSuccess)
             return SEMSHARE_ECUDA;
-        hd_select_kernel<true><<<n_layers, kSelThreads, stage, s>>>(sigma, n_tok, k, hd_idx, hd_mask);
+        if (launch_pdl(hd_select_kernel<true>, dim3(n_layers), dim3(kSelThreads), stage, s, sigma, n_tok, k, hd_idx,
+                       hd_mask) != cudaSuccess)
+            return SEMSHARE_ECUDA;
     } else {
-        hd_select_kernel<false><<<n_layers, kSelThreads, 0, s>>>(sigma, n_tok, k, hd_idx, hd_mask);
+        if (launch_pdl(hd_select_kernel<false>, dim3(n_layers), dim3(kSelThreads), 0, s, sigma, n_tok, k, hd_idx,
+                       hd_mask) != cudaSuccess)
+            return SEMSHARE_ECUDA;
     }
     return launch_status();
 }

@@ -108,6 +108,7 @@ __device__ __forceinline__ bool resolve_rows(const GatherArgs& a, const RT& rt, 
 template <int C, bool kRetain, typename RT>
 __global__ void __launch_bounds__(kThreads)
     kv_gather_kernel(const __grid_constant__ GatherArgs a, const __grid_constant__ RT rt) {
+    pdl_prologue();
     constexpr int kRowsPerPass = kThreads / C;
     constexpr int kPasses = 2 * kTokens / kRowsPerPass;  // K rows then V rows
     static_assert(kThreads % C == 0 && (2 * kTokens) % kRowsPerPass == 0, "row split");
@@ -152,6 +153,7 @@ __global__ void __launch_bounds__(kThreads)
 template <bool kRetain, typename RT>
 __global__ void __launch_bounds__(kThreads)
     kv_gather_generic_kernel(const __grid_constant__ GatherArgs a, const __grid_constant__ RT rt, int chunks) {
+    pdl_prologue();
     __shared__ int64_t s_src_off[kTokens];
     __shared__ int32_t s_seg[kTokens];
     const int64_t plane = blockIdx.y + static_cast<int64_t>(gridDim.y) * blockIdx.z;
@@ -233,13 +235,15 @@ semshare_status launch_gather(const GatherArgs& a, const RT& rt, int64_t planes,
     if (planes / gy > 65535) return SEMSHARE_EUNSUPPORTED;
     const dim3 grid(static_cast<unsigned>(tblocks), static_cast<unsigned>(gy), static_cast<unsigned>(planes / gy));
     const int chunks = static_cast<int>(row_bytes / 16);
+    cudaError_t e;
     switch (chunks) {
-        case 4: kv_gather_kernel<4, kRetain><<<grid, kThreads, 0, s>>>(a, rt); break;
-        case 8: kv_gather_kernel<8, kRetain><<<grid, kThreads, 0, s>>>(a, rt); break;
-        case 16: kv_gather_kernel<16, kRetain><<<grid, kThreads, 0, s>>>(a, rt); break;
-        case 32: kv_gather_kernel<32, kRetain><<<grid, kThreads, 0, s>>>(a, rt); break;
-        default: kv_gather_generic_kernel<kRetain><<<grid, kThreads, 0, s>>>(a, rt, chunks); break;
+        case 4: e = launch_pdl(kv_gather_kernel<4, kRetain, RT>, grid, dim3(kThreads), 0, s, a, rt); break;
+        case 8: e = launch_pdl(kv_gather_kernel<8, kRetain, RT>, grid, dim3(kThreads), 0, s, a, rt); break;
+        case 16: e = launch_pdl(kv_gather_kernel<16, kRetain, RT>, grid, dim3(kThreads), 0, s, a, rt); break;
+        case 32: e = launch_pdl(kv_gather_kernel<32, kRetain, RT>, grid, dim3(kThreads), 0, s, a, rt); break;
+        default: e = launch_pdl(kv_gather_generic_kernel<kRetain, RT>, grid, dim3(kThreads), 0, s, a, rt, chunks); break;
     }
+    if (e != cudaSuccess) return SEMSHARE_ECUDA;
     return launch_status();
 }
 

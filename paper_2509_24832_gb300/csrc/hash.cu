@@ -220,6 +220,7 @@ template <bool kHalf>
 __global__ void __launch_bounds__(kThreads, 1)
     lsh_hash_kernel(const __grid_constant__ CUtensorMap tmap_emb, const __grid_constant__ CUtensorMap tmap_hyp,
                     const HashArgs a) {
+    pdl_prologue();
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_addr(smem_raw);
     const uint32_t sbase = (raw + 1023u) & ~1023u;  // stage tiles on the swizzle-atom boundary
@@ -856,7 +857,8 @@ extern "C" semshare_status semshare_hash_ex(const void* emb, semshare_dtype dtyp
     auto kernel = half ? lsh_hash_kernel<true> : lsh_hash_kernel<false>;
     if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) != cudaSuccess)
         return SEMSHARE_ECUDA;
-    kernel<<<plan.grid, kThreads, smem, as_stream(stream)>>>(tm_emb, tm_hyp, a);
+    if (launch_pdl(kernel, dim3(plan.grid), dim3(kThreads), smem, as_stream(stream), tm_emb, tm_hyp, a) != cudaSuccess)
+        return SEMSHARE_ECUDA;
     return launch_status();
 }
 

@@ -28,6 +28,7 @@ constexpr int kRC = 256;                    // reference codes per staging round
 constexpr unsigned long long kNoKey = ~0ull;
 
 __global__ void keys_init_kernel(unsigned long long* __restrict__ keys, int64_t n) {
+    pdl_prologue();
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x)
         keys[i] = kNoKey;
@@ -35,6 +36,7 @@ __global__ void keys_init_kernel(unsigned long long* __restrict__ keys, int64_t 
 
 __global__ void keys_split_kernel(const unsigned long long* __restrict__ keys, int64_t n, int32_t* __restrict__ idx,
                                   int32_t* __restrict__ dist) {
+    pdl_prologue();
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const unsigned long long k = keys[i];
@@ -61,6 +63,7 @@ template <int W>
 __global__ void __launch_bounds__(kThreads)
     hamming_nn_kernel(const uint32_t* __restrict__ tgt, int64_t n_tgt, const uint32_t* __restrict__ ref, int64_t n_ref,
                       unsigned long long* __restrict__ keys, int64_t n_tblocks) {
+    pdl_prologue();
     __shared__ __align__(16) uint32_t sref[kRC * W];
 
     // this CTA's share of the n_tblocks * n_ref (target block, reference row) pairs
@@ -157,7 +160,9 @@ semshare_status launch_search(const uint32_t* tgt, int64_t n_tgt, const uint32_t
     const int64_t total = n_tblocks * n_ref;
     int64_t grid = static_cast<int64_t>(sms) * per_sm;
     if (grid > total) grid = total;
-    hamming_nn_kernel<W><<<static_cast<unsigned>(grid), kThreads, 0, s>>>(tgt, n_tgt, ref, n_ref, keys, n_tblocks);
+    if (launch_pdl(hamming_nn_kernel<W>, dim3(static_cast<unsigned>(grid)), dim3(kThreads), 0, s, tgt, n_tgt, ref, n_ref,
+                   keys, n_tblocks) != cudaSuccess)
+        return SEMSHARE_ECUDA;
     return launch_status();
 }
 
@@ -188,7 +193,7 @@ extern "C" semshare_status semshare_match(const uint32_t* tgt_codes, int64_t n_t
     auto* keys = static_cast<unsigned long long*>(workspace);
     const int small_grid = static_cast<int>((n_tgt + 255) / 256 < sms * 4 ? (n_tgt + 255) / 256 : sms * 4);
 
-    keys_init_kernel<<<small_grid, 256, 0, s>>>(keys, n_tgt);
+    if (launch_pdl(keys_init_kernel, dim3(small_grid), dim3(256), 0, s, keys, n_tgt) != cudaSuccess) return SEMSHARE_ECUDA;
     if (launch_status() != SEMSHARE_OK) return SEMSHARE_ECUDA;
     semshare_status st = SEMSHARE_EUNSUPPORTED;
     switch (nbits / 32) {
@@ -202,7 +207,8 @@ extern "C" semshare_status semshare_match(const uint32_t* tgt_codes, int64_t n_t
         case 8: st = launch_search<8>(tgt_codes, n_tgt, ref_codes, n_ref, keys, sms, s); break;
     }
     if (st != SEMSHARE_OK) return st;
-    keys_split_kernel<<<small_grid, 256, 0, s>>>(keys, n_tgt, idx, dist);
+    if (launch_pdl(keys_split_kernel, dim3(small_grid), dim3(256), 0, s, keys, n_tgt, idx, dist) != cudaSuccess)
+        return SEMSHARE_ECUDA;
     return launch_status();
 }
 
@@ -265,7 +271,7 @@ extern "C" semshare_status semshare_match_static(const uint32_t* tgt_codes, int6
     const int small_grid = static_cast<int>((n_tgt + 255) / 256 < sms * 4 ? (n_tgt + 255) / 256 : sms * 4);
 
     // the array keeps the previous call's keys: reset the ones this call uses
-    keys_init_kernel<<<small_grid, 256, 0, s>>>(keys, n_tgt);
+    if (launch_pdl(keys_init_kernel, dim3(small_grid), dim3(256), 0, s, keys, n_tgt) != cudaSuccess) return SEMSHARE_ECUDA;
     if (launch_status() != SEMSHARE_OK) return SEMSHARE_ECUDA;
     st = SEMSHARE_EUNSUPPORTED;
     switch (nbits / 32) {
@@ -279,6 +285,7 @@ extern "C" semshare_status semshare_match_static(const uint32_t* tgt_codes, int6
         case 8: st = launch_search<8>(tgt_codes, n_tgt, ref_codes, n_ref, keys, sms, s); break;
     }
     if (st != SEMSHARE_OK) return st;
-    keys_split_kernel<<<small_grid, 256, 0, s>>>(keys, n_tgt, idx, dist);
+    if (launch_pdl(keys_split_kernel, dim3(small_grid), dim3(256), 0, s, keys, n_tgt, idx, dist) != cudaSuccess)
+        return SEMSHARE_ECUDA;
     return launch_status();
 }

@@ -73,6 +73,7 @@ __global__ void expand_codes_kernel(const uint32_t* __restrict__ tgt, int64_t n_
                                     int64_t n_ref, int32_t nbits, int32_t kpad, uint8_t* __restrict__ tpm,
                                     uint8_t* __restrict__ rpm, unsigned long long* __restrict__ keys, int64_t n_keys,
                                     unsigned int* __restrict__ counter) {
+    pdl_prologue();
     const int W = nbits >> 5;
     const int per_row = kpad >> 4;  // 16-byte pieces per row
     const int64_t total = (n_tgt + n_ref) * per_row;
@@ -104,6 +105,7 @@ __global__ void expand_codes_kernel(const uint32_t* __restrict__ tgt, int64_t n_
 
 __global__ void tc_keys_split_kernel(const unsigned long long* __restrict__ keys, int64_t n, int32_t* __restrict__ idx,
                                      int32_t* __restrict__ dist) {
+    pdl_prologue();
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const unsigned long long k = keys[i];
@@ -124,6 +126,7 @@ template <int kMaxSeg>
 __global__ void __launch_bounds__(kThreads, 1)
     hamming_tc_kernel(const __grid_constant__ CUtensorMap tm_t, const __grid_constant__ CUtensorMap tm_r,
                       const TcArgs a, const __grid_constant__ SegTable<kMaxSeg> seg) {
+    pdl_prologue();
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_addr(smem_raw);
     const uint32_t sbase = (raw + 1023u) & ~1023u;
@@ -394,6 +397,7 @@ __global__ void __launch_bounds__(256)
                              double max_dist, double threshold, long long* sums, unsigned int* counter,
                              double* __restrict__ mean_dist, double* __restrict__ similarity,
                              int32_t* __restrict__ best, int32_t* __restrict__ applies) {
+    pdl_prologue();
     __shared__ long long warp_sum[8];
     __shared__ bool last;
     const int s = blockIdx.x;
@@ -453,6 +457,7 @@ __global__ void __launch_bounds__(256)
 __global__ void retrieve_select_kernel(const unsigned long long* __restrict__ keys, int64_t n_tgt,
                                        const int32_t* __restrict__ best, int32_t* __restrict__ idx,
                                        int32_t* __restrict__ dist) {
+    pdl_prologue();
     const unsigned long long* k = keys + static_cast<int64_t>(*best) * n_tgt;
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n_tgt;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -504,11 +509,14 @@ semshare_status launch_search(const uint32_t* tgt_codes, int64_t n_tgt, const ui
 
     const int64_t pieces = (n_tgt + n_ref) * (plan.kpad / 16);
     const int64_t eg = (pieces + 255) / 256;
-    expand_codes_kernel<<<static_cast<unsigned>(eg < sms * 8 ? eg : sms * 8), 256, 0, s>>>(
-        tgt_codes, n_tgt, ref_codes, n_ref, nbits, plan.kpad, tpm, rpm, keys, n_tgt * seg.n_seg, counter);
-    if (launch_status() != SEMSHARE_OK) return SEMSHARE_ECUDA;
+    if (launch_pdl(expand_codes_kernel, dim3(static_cast<unsigned>(eg < sms * 8 ? eg : sms * 8)), dim3(256), 0, s,
+                   tgt_codes, n_tgt, ref_codes, n_ref, nbits, plan.kpad, tpm, rpm, keys, n_tgt * seg.n_seg,
+                   counter) != cudaSuccess)
+        return SEMSHARE_ECUDA;
     const int64_t grid = a.total < sms ? a.total : sms;
-    hamming_tc_kernel<kMaxSeg><<<static_cast<unsigned>(grid), kThreads, smem, s>>>(tm_t, tm_r, a, seg);
+    if (launch_pdl(hamming_tc_kernel<kMaxSeg>, dim3(static_cast<unsigned>(grid)), dim3(kThreads), smem, s, tm_t, tm_r, a,
+                   seg) != cudaSuccess)
+        return SEMSHARE_ECUDA;
     return launch_status();
 }
 
@@ -551,7 +559,9 @@ extern "C" semshare_status semshare_match_tc(const uint32_t* tgt_codes, int64_t 
                                              err_flag, s, sms, dev);
     if (st != SEMSHARE_OK) return st;
     const int small = static_cast<int>((n_tgt + 255) / 256 < sms * 4 ? (n_tgt + 255) / 256 : sms * 4);
-    tc_keys_split_kernel<<<small, 256, 0, s>>>(static_cast<const unsigned long long*>(workspace), n_tgt, idx, dist);
+    if (launch_pdl(tc_keys_split_kernel, dim3(small), dim3(256), 0, s, static_cast<const unsigned long long*>(workspace),
+                   n_tgt, idx, dist) != cudaSuccess)
+        return SEMSHARE_ECUDA;
     return launch_status();
 }
 
@@ -604,12 +614,15 @@ extern "C" semshare_status semshare_retrieve(const uint32_t* tgt_codes, int64_t 
     auto* sums = reinterpret_cast<long long*>(static_cast<uint8_t*>(workspace) + plan.keys_bytes + plan.t_bytes +
                                               plan.r_bytes);
     auto* counter = reinterpret_cast<unsigned int*>(sums + n_cand);
-    retrieve_finalize_kernel<<<n_cand, 256, 0, s>>>(keys, n_tgt, n_cand, max_dist, threshold, sums, counter,
-                                                    mean_dist, similarity, best, applies);
+    if (launch_pdl(retrieve_finalize_kernel, dim3(n_cand), dim3(256), 0, s, keys, n_tgt, n_cand, max_dist, threshold, sums,
+                   counter, mean_dist, similarity, best, applies) != cudaSuccess)
+        return SEMSHARE_ECUDA;
     if (launch_status() != SEMSHARE_OK) return SEMSHARE_ECUDA;
     if (idx || dist) {
         const int small = static_cast<int>((n_tgt + 255) / 256 < sms * 4 ? (n_tgt + 255) / 256 : sms * 4);
-        retrieve_select_kernel<<<small, 256, 0, s>>>(keys, n_tgt, best, idx, dist);
+        if (launch_pdl(retrieve_select_kernel, dim3(small), dim3(256), 0, s, keys, n_tgt, best, idx, dist) !=
+            cudaSuccess)
+            return SEMSHARE_ECUDA;
         st = launch_status();
     }
     return st;
