@@ -51,12 +51,12 @@ L2_FLUSH_BYTES = 512 << 20
 # workload, valid only for that workload and while the kernel source has the recorded sha256
 # prefix (the traffic depends on the index pattern, e.g. how often a gathered row repeats).
 NCU_TRAFFIC = {
-    ("gather", "llama8b-5k"): {"file": "gather.cu", "sha": "7d05bda6e8a70170", "bytes_per_launch": 1092.7e6},
-    ("gather_retained", "llama8b-5k"): {"file": "gather.cu", "sha": "7d05bda6e8a70170", "bytes_per_launch": 663.2e6},
-    ("hash", "llama8b-5k"): {"file": "hash.cu", "sha": "c9f57175642e48ea", "bytes_per_launch": 90.85e6},
-    ("match", "llama8b-5k"): {"file": "match.cu", "sha": "69ac4b7ce5b193e4", "bytes_per_launch": 0.3845e6},
-    ("match_tc", "llama8b-5k"): {"file": "match_tc.cu", "sha": "c494ec8dce435f1b", "bytes_per_launch": 2.736e6},
-    ("retrieve", "retrieve-16x4096"): {"file": "match_tc.cu", "sha": "c494ec8dce435f1b", "bytes_per_launch": 18.42e6},
+    ("gather", "llama8b-5k"): {"file": "gather.cu", "sha": "05f4f810661f80c0", "bytes_per_launch": 1093.5e6},
+    ("gather_retained", "llama8b-5k"): {"file": "gather.cu", "sha": "05f4f810661f80c0", "bytes_per_launch": 663.0e6},
+    ("gather", "retrieve-16x4096"): {"file": "gather.cu", "sha": "05f4f810661f80c0", "bytes_per_launch": 1001.6e6},
+    ("hash", "llama8b-5k"): {"file": "hash.cu", "sha": "44b3ff223d9e1bd0", "bytes_per_launch": 90.96e6},
+    ("match_tc", "llama8b-5k"): {"file": "match_tc.cu", "sha": "2da41b19612a09a3", "bytes_per_launch": 2.737e6},
+    ("retrieve", "retrieve-16x4096"): {"file": "match_tc.cu", "sha": "2da41b19612a09a3", "bytes_per_launch": 18.42e6},
 }
 
 
