@@ -287,7 +287,9 @@ typedef struct {
  * KV head h and target token t < n_tgt:
  *     out_k[b][l][h][t][:] = ref_k[l][h][idx[b*n_tgt + t]][:]      (same for V)
  *
- *   ref_k, ref_v   host arrays of n_seg device base pointers, one reference prompt each.
+ *   ref_k, ref_v   host arrays of n_seg base pointers, one reference prompt each: device memory,
+ *                  or page-locked host memory the device can address (the kernel then reads the
+ *                  selected rows across the host link, and only those rows cross it).
  *                  Global reference row r belongs to the segment s with
  *                  seg_offsets[s] <= r < seg_offsets[s+1] and is its local row
  *                  r - seg_offsets[s].  Every segment uses the strides of `src`.

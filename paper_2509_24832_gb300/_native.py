@@ -117,6 +117,13 @@ def _need_cuda(t: torch.Tensor, name: str):
         raise ValueError(f"{name} must be a CUDA tensor")
 
 
+def _need_device_accessible(t: torch.Tensor, name: str):
+    """A CUDA tensor, or a pinned (page-locked) host tensor: the GPU reads it in place over the
+    host link (its address is valid on the device)."""
+    if not isinstance(t, torch.Tensor) or not (t.is_cuda or t.is_pinned()):
+        raise ValueError(f"{name} must be a CUDA tensor or a pinned host tensor")
+
+
 def new_err_flag(device=None) -> torch.Tensor:
     """A zeroed device word for the kernels' error bits."""
     return torch.zeros(1, dtype=torch.int32, device=device or "cuda")
@@ -387,7 +394,7 @@ def semshare_gather_kv(ref_k, ref_v, idx: torch.Tensor, out_k: torch.Tensor | No
                        out_v: torch.Tensor | None = None, err_flag: torch.Tensor | None = None, stream=None):
     """Reordered K/V cache: out[b][l][h][t] = ref[l][h][idx[b][t]].
 
-    ref_k/ref_v: a [L][H][N][hd] CUDA tensor, or a list of them (a pool of reference prompts
+    ref_k/ref_v: a [L][H][N][hd] CUDA or pinned host tensor, or a list of them (a pool of reference prompts
     with identical strides; global row r = running offset of its segment + local row).
     idx: [n_batch][n_tgt] or [n_tgt] int32.  Returns (out_k, out_v), [n_batch][L][H][n_tgt][hd]."""
     seg_k = list(ref_k) if isinstance(ref_k, (list, tuple)) else [ref_k]
@@ -395,7 +402,7 @@ def semshare_gather_kv(ref_k, ref_v, idx: torch.Tensor, out_k: torch.Tensor | No
     if len(seg_k) != len(seg_v) or not seg_k:
         raise ValueError("ref_k and ref_v must have the same number of segments")
     for t in seg_k + seg_v:
-        _need_cuda(t, "ref")
+        _need_device_accessible(t, "ref")
     src = kv_layout(seg_k[0], batched=False)
     for t in seg_k[1:] + seg_v:
         o = kv_layout(t, batched=False)
@@ -409,9 +416,11 @@ def semshare_gather_kv(ref_k, ref_v, idx: torch.Tensor, out_k: torch.Tensor | No
     n_batch, n_tgt = idx2.shape
     L, H, hd = src.n_layers, src.n_heads, src.head_dim
     if out_k is None:
-        out_k = torch.empty((n_batch, L, H, n_tgt, hd), dtype=seg_k[0].dtype, device=seg_k[0].device)
+        out_k = torch.empty((n_batch, L, H, n_tgt, hd), dtype=seg_k[0].dtype, device=idx.device)
     if out_v is None:
-        out_v = torch.empty((n_batch, L, H, n_tgt, hd), dtype=seg_v[0].dtype, device=seg_v[0].device)
+        out_v = torch.empty((n_batch, L, H, n_tgt, hd), dtype=seg_v[0].dtype, device=idx.device)
+    _need_cuda(out_k, "out_k")
+    _need_cuda(out_v, "out_v")
     dst = kv_layout(out_k, batched=True)
     dv = kv_layout(out_v, batched=True)
     if (dst.stride_batch, dst.stride_layer, dst.stride_head, dst.stride_token) != \
@@ -510,7 +519,7 @@ def semshare_gather_kv_retained(ref_k, ref_v, idx: torch.Tensor, retained, ret_o
                                 err_flag: torch.Tensor | None = None, stream=None):
     """Retention-aware rearrangement (Sec. 3.3.4): out[l][h][r] = ref[l][h][idx[retained_l[r]]].
 
-    ref_k/ref_v: a [L][H][N][hd] CUDA tensor or a list of them (a pool, as semshare_gather_kv).
+    ref_k/ref_v: a [L][H][N][hd] CUDA or pinned host tensor, or a list of them (as semshare_gather_kv).
     idx: int32 [n_tgt].  retained: int32 CUDA tensor, the layers' lists back to back;
     ret_offsets: host sequence of L + 1 ints.  Returns (out_k, out_v), [L][H][longest][hd]."""
     seg_k = list(ref_k) if isinstance(ref_k, (list, tuple)) else [ref_k]
@@ -518,7 +527,7 @@ def semshare_gather_kv_retained(ref_k, ref_v, idx: torch.Tensor, retained, ret_o
     if len(seg_k) != len(seg_v) or not seg_k:
         raise ValueError("ref_k and ref_v must have the same number of segments")
     for t in seg_k + seg_v:
-        _need_cuda(t, "ref")
+        _need_device_accessible(t, "ref")
     src = kv_layout(seg_k[0], batched=False)
     for t in seg_k[1:] + seg_v:
         o = kv_layout(t, batched=False)
@@ -535,9 +544,11 @@ def semshare_gather_kv_retained(ref_k, ref_v, idx: torch.Tensor, retained, ret_o
         raise ValueError("ret_offsets needs n_layers + 1 entries")
     longest = max(int(ret_offsets[l + 1]) - int(ret_offsets[l]) for l in range(L))
     if out_k is None:
-        out_k = torch.empty((L, H, max(longest, 0), hd), dtype=seg_k[0].dtype, device=seg_k[0].device)
+        out_k = torch.empty((L, H, max(longest, 0), hd), dtype=seg_k[0].dtype, device=idx.device)
     if out_v is None:
-        out_v = torch.empty((L, H, max(longest, 0), hd), dtype=seg_v[0].dtype, device=seg_v[0].device)
+        out_v = torch.empty((L, H, max(longest, 0), hd), dtype=seg_v[0].dtype, device=idx.device)
+    _need_cuda(out_k, "out_k")
+    _need_cuda(out_v, "out_v")
     dst = kv_layout(out_k, batched=False)
     if kv_layout(out_v, batched=False).stride_token != dst.stride_token or out_v.stride() != out_k.stride():
         raise ValueError("out_k and out_v must share one layout")

@@ -361,3 +361,18 @@ def test_wait_timeout_reports_status_and_context_survives(ss, orc, monkeypatch):
     gc = codes_host(codes)
     oi, od = orc.match(gc[wl.n_ref:], gc[: wl.n_ref])
     np.testing.assert_array_equal(idx.cpu().numpy(), oi)
+
+
+def test_gather_from_pinned_host_cache(ss):
+    """Reference segments in page-locked host memory: the kernel reads the selected rows across the
+    host link in place; the result equals the gather from device copies bit for bit."""
+    g = torch.Generator().manual_seed(5)
+    segs = [(torch.randn((3, 2, n, 128), generator=g).to(torch.bfloat16).pin_memory(),
+             torch.randn((3, 2, n, 128), generator=g).to(torch.bfloat16).pin_memory()) for n in (300, 300)]
+    idx = torch.randint(0, 600, (2, 257), generator=g, dtype=torch.int32).cuda()
+    flag = ss.new_err_flag()
+    hk, hv = ss.semshare_gather_kv([s[0] for s in segs], [s[1] for s in segs], idx, err_flag=flag)
+    dk, dv = ss.semshare_gather_kv([s[0].cuda() for s in segs], [s[1].cuda() for s in segs], idx)
+    torch.cuda.synchronize()
+    assert hk.is_cuda and int(flag.item()) == 0
+    assert torch.equal(hk.view(torch.int16), dk.view(torch.int16)) and torch.equal(hv.view(torch.int16), dv.view(torch.int16))
