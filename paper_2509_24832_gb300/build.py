@@ -18,7 +18,12 @@ LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "libsemshare.so")
 SOURCES = ["api.cu", "hash.cu", "match.cu", "match_tc.cu", "gather.cu", "deviation.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-NVCC_FLAGS = ARCH + ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2", "-I", INCLUDE, "-I", CSRC]
+# -warn-spills: a register spill in a file with tensor-memory loads is a build error (below).  Those
+# kernels hand tcgen05.ld destination registers to later code before the load's wait; a spill placed
+# in between would store them before the data arrives.
+NO_SPILL = {"hash.cu", "match_tc.cu"}
+NVCC_FLAGS = ARCH + ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2", "-Xptxas", "-warn-spills",
+                     "-I", INCLUDE, "-I", CSRC]
 
 
 def nvcc() -> str:
@@ -59,12 +64,13 @@ def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | N
     failed = []
     for src, p in procs:
         out, _ = p.communicate()
-        if out and (verbose or p.returncode):
+        spilled = src in NO_SPILL and "spill" in (out or "").lower()
+        if out and (verbose or p.returncode or spilled):
             print(out, file=sys.stderr)
-        if p.returncode:
+        if p.returncode or spilled:
             failed.append(src)
     if failed:
-        raise RuntimeError(f"nvcc failed on {failed}")
+        raise RuntimeError(f"nvcc failed (or spilled registers) on {failed}")
     tmp = LIB + f".tmp{os.getpid()}"
     subprocess.run([cc, *ARCH, "-shared", "-Xcompiler", "-fPIC", *objs, "-o", tmp], check=True)
     os.replace(tmp, LIB)

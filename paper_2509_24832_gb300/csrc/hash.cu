@@ -52,11 +52,15 @@ namespace {
 constexpr int kBM = 128;                       // rows per tile (MMA M, one TMEM lane per row)
 constexpr int kBK = 64;                        // K elements per stage: one 128-byte row of bf16
 constexpr int kUmmaK = 16;                     // K of one tcgen05.mma kind::f16
-constexpr int kThreads = 512;
 constexpr int kRopeWarp0 = 4;
 constexpr int kRopeWarps = 8;
-constexpr int kEpiWarp0 = 12;                  // 12 % 4 == 0: epilogue warp w reads TMEM lanes 32*(w%4)
+// (row, 16-byte chunk) items of a stage per RoPE thread: rows rbase + 32*i, i < kRopeRows
+constexpr int kRopeRows = kBM * (kBK * 2 / 16) / (kRopeWarps * 32);
+static_assert(kRopeRows >= 1 && kRopeRows <= 4 && kRopeRows * kRopeWarps * 32 == kBM * (kBK * 2 / 16), "RoPE split");
+constexpr int kEpiWarp0 = kRopeWarp0 + kRopeWarps;  // a multiple of 4: epilogue warp w reads TMEM lanes 32*(w%4)
 constexpr int kEpiWarps = 4;
+constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
+static_assert(kEpiWarp0 % 4 == 0, "epilogue warps must start on a warpgroup");
 constexpr uint32_t kABytes = kBM * kBK * 2;    // bf16 operand tile, 16 KB
 constexpr uint32_t kF32Bytes = kBM * kBK * 4;  // fp32 staging: two 128-byte-wide boxes, 32 KB
 constexpr int kEpiBarrier = 1;                 // named barrier of the epilogue warps
@@ -379,28 +383,30 @@ __global__ void __launch_bounds__(kThreads, 1)
         // sit at the same place in the staged partner block.
         const int rt = threadIdx.x - kRopeWarp0 * 32;
         const int c = rt & 7;
-        const int rg = rt >> 3;
+        const int rg = (rt >> 3) & 31;
+        const int rbase = rg + 32 * kRopeRows * (rt >> 8);  // rows rbase + 32*i, i < kRopeRows
         const uint32_t chunk_off = (static_cast<uint32_t>(c) ^ static_cast<uint32_t>(rg & 7)) << 4;
         const int hk = nkb / 2;
         const int half = nkb * (kBK / 2);
         uint32_t q = 0;
         int tile = static_cast<int>(i0 / nkb), kb = static_cast<int>(i0 % nkb), cur_tile = -1;
-        uint32_t m[4] = {0u, 0u, 0u, 0u};
+        uint32_t m[kRopeRows];
         bool steps32 = false;
         Pairs8 tn;
         load_pairs8(a.rope_table, half, (kb % hk) * kBK + 8 * c, tn);
         for (int64_t it = i0; it < i1; ++it, ++q) {
             if (tile != cur_tile) {
                 cur_tile = tile;
-                const int64_t r0 = static_cast<int64_t>(tile) * kBM + rg;
+                const int64_t r0 = static_cast<int64_t>(tile) * kBM + rbase;
+                steps32 = true;
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
+                for (int i = 0; i < kRopeRows; ++i) {
                     const int64_t row = r0 + 32 * i;
                     m[i] = row < a.n ? (a.positions ? static_cast<uint32_t>(__ldg(a.positions + row))
                                                     : static_cast<uint32_t>(row))
-                                     : m[0] + 32u * i;
+                                     : (i == 0 ? 0u : m[0] + 32u * i);
+                    steps32 = steps32 && m[i] == m[0] + 32u * i;
                 }
-                steps32 = m[1] == m[0] + 32u && m[2] == m[0] + 64u && m[3] == m[0] + 96u;
             }
             const Pairs8 tc = tn;
             const bool first_half = kb < hk;
@@ -419,8 +425,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int e = 0; e < 8; ++e) rotation(m[0], tc.turns[e], cs[e], sn[e]);
             }
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const uint32_t off = (rg + 32 * i) * 128 + chunk_off;
+            for (int i = 0; i < kRopeRows; ++i) {
+                const uint32_t off = (rbase + 32 * i) * 128 + chunk_off;
                 const uint4 vo = *reinterpret_cast<const uint4*>(st + off);
                 const uint4 vp = *reinterpret_cast<const uint4*>(pt + off);
                 const uint32_t wo[4] = {vo.x, vo.y, vo.z, vo.w}, wp[4] = {vp.x, vp.y, vp.z, vp.w};
@@ -439,7 +445,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     y[w] = *reinterpret_cast<uint32_t*>(&r);
                 }
                 *reinterpret_cast<uint4*>(st + off) = make_uint4(y[0], y[1], y[2], y[3]);
-                if (steps32 && i < 3) {
+                if (steps32 && i < kRopeRows - 1) {
 #pragma unroll
                     for (int e = 0; e < 8; ++e) {
                         const float c32 = __uint_as_float(static_cast<uint32_t>(tc.cis32[e]));
@@ -458,15 +464,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if (!kHalf && warp >= kRopeWarp0 && warp < kRopeWarp0 + kRopeWarps) {
         // ---------------- RoPE (Eq. 1) on the staged tile ----------------
-        const int rt = threadIdx.x - kRopeWarp0 * 32;  // 0..255
+        const int rt = threadIdx.x - kRopeWarp0 * 32;
         const int c = rt & 7;                          // 16-byte chunk of the 128-byte row: pairs 4c..4c+3
-        const int rg = rt >> 3;                        // rows rg + 32*i, i < 4 (all with row & 7 == rg & 7)
+        const int rg = (rt >> 3) & 31;
+        const int rbase = rg + 32 * kRopeRows * (rt >> 8);  // rows rbase + 32*i, i < kRopeRows (row & 7 == rg & 7)
         const uint32_t swz = static_cast<uint32_t>(rg & 7);
         const uint32_t chunk_off = (static_cast<uint32_t>(c) ^ swz) << 4;
         uint32_t q = 0;
         int tile = static_cast<int>(i0 / nkb), kb = static_cast<int>(i0 % nkb), cur_tile = -1;
         const int half = nkb * (kBK / 2);  // d/2: start of the 32-position rotations in the table
-        uint32_t m[4] = {0u, 0u, 0u, 0u};
+        uint32_t m[kRopeRows];
         bool steps32 = false;
         Pairs4 tn;
         load_pairs4(a.rope_table, half, kb, c, tn);
@@ -474,18 +481,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (tile != cur_tile) {
                 cur_tile = tile;
                 const int64_t row0 = static_cast<int64_t>(tile) * kBM;
-                const int64_t r0 = row0 + rg;
+                const int64_t r0 = row0 + rbase;
                 m[0] = r0 < a.n ? (a.positions ? static_cast<uint32_t>(__ldg(a.positions + r0)) : static_cast<uint32_t>(r0))
                                 : 0u;
+                steps32 = true;
 #pragma unroll
-                for (int i = 1; i < 4; ++i) {
+                for (int i = 1; i < kRopeRows; ++i) {
                     // rows past n are zero-filled by TMA: any angle will do, keep the 32-step pattern
                     const int64_t row = r0 + 32 * i;
                     m[i] = row < a.n ? (a.positions ? static_cast<uint32_t>(__ldg(a.positions + row))
                                                     : static_cast<uint32_t>(row))
                                      : m[0] + 32u * i;
+                    steps32 = steps32 && m[i] == m[0] + 32u * i;
                 }
-                steps32 = m[1] == m[0] + 32u && m[2] == m[0] + 64u && m[3] == m[0] + 96u;
             }
             const Pairs4 tc = tn;
             const int kb_next = kb + 1 == nkb ? 0 : kb + 1;
@@ -496,12 +504,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                                                a.wait_limit_ns);
             if (!__all_sync(0xFFFFFFFFu, got)) break;
             uint8_t* const st = gbase + s * a.stage_bytes;
-            float x[4][8];
+            float x[kRopeRows][8];
             if (a.is_f32) {
                 const uint32_t c0 = static_cast<uint32_t>((c & 3) * 2);
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const uint8_t* stg = st + kABytes + a.b_bytes + (c >> 2) * (kF32Bytes / 2) + (rg + 32 * i) * 128;
+                for (int i = 0; i < kRopeRows; ++i) {
+                    const uint8_t* stg = st + kABytes + a.b_bytes + (c >> 2) * (kF32Bytes / 2) + (rbase + 32 * i) * 128;
                     const float4 f0 = *reinterpret_cast<const float4*>(stg + ((c0 ^ swz) << 4));
                     const float4 f1 = *reinterpret_cast<const float4*>(stg + (((c0 + 1u) ^ swz) << 4));
                     x[i][0] = f0.x; x[i][1] = f0.y; x[i][2] = f0.z; x[i][3] = f0.w;
@@ -509,8 +517,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             } else {
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const uint4 v = *reinterpret_cast<const uint4*>(st + (rg + 32 * i) * 128 + chunk_off);
+                for (int i = 0; i < kRopeRows; ++i) {
+                    const uint4 v = *reinterpret_cast<const uint4*>(st + (rbase + 32 * i) * 128 + chunk_off);
                     const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
                     for (int p = 0; p < 4; ++p) {
@@ -519,18 +527,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
             }
-            uint32_t y[4][4];
+            uint32_t y[kRopeRows][4];
             if (steps32) {
                 // row i+1 sits 32 positions after row i: turn the angle on by the 32-step rotation
                 float cs[4], sn[4];
 #pragma unroll
                 for (int p = 0; p < 4; ++p) rotation(m[0], tc.turns[p], cs[p], sn[p]);
 #pragma unroll
-                for (int i = 0; i < 4; ++i)
+                for (int i = 0; i < kRopeRows; ++i)
 #pragma unroll
                     for (int p = 0; p < 4; ++p) {
                         y[i][p] = rotate_to_bf16(x[i][2 * p], x[i][2 * p + 1], cs[p], sn[p]);
-                        if (i < 3) {
+                        if (i < kRopeRows - 1) {
                             const float c32 = __uint_as_float(static_cast<uint32_t>(tc.cis32[p]));
                             const float s32 = __uint_as_float(static_cast<uint32_t>(tc.cis32[p] >> 32));
                             const float nc = fmaf(cs[p], c32, -sn[p] * s32);
@@ -540,7 +548,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
             } else {
 #pragma unroll
-                for (int i = 0; i < 4; ++i)
+                for (int i = 0; i < kRopeRows; ++i)
 #pragma unroll
                     for (int p = 0; p < 4; ++p) {
                         float cs, sn;
@@ -549,8 +557,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
             }
 #pragma unroll
-            for (int i = 0; i < 4; ++i)
-                *reinterpret_cast<uint4*>(st + (rg + 32 * i) * 128 + chunk_off) =
+            for (int i = 0; i < kRopeRows; ++i)
+                *reinterpret_cast<uint4*>(st + (rbase + 32 * i) * 128 + chunk_off) =
                     make_uint4(y[i][0], y[i][1], y[i][2], y[i][3]);
             fence_proxy_async_smem();
             __syncwarp();
@@ -590,8 +598,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     words[qq] = 0u;
                     if (qq < W) {
                         uint32_t v[32];
-                        tmem_load_32cols(taddr + qq * 32, v);
-                        tmem_load_wait_fence(v);
+                        tmem_load_32cols_sync(taddr + qq * 32, v);
                         words[qq] = sign_word(v);
                         if (a.proj != nullptr && row < a.n) store_proj(a.proj, row, a.nbits, qq, v);
                     }
@@ -609,8 +616,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int qq = 0; qq < 8; ++qq) {
                     if (qq < W) {
                         uint32_t v[32];
-                        tmem_load_32cols(taddr + qq * 32, v);
-                        tmem_load_wait_fence(v);
+                        tmem_load_32cols_sync(taddr + qq * 32, v);
 #pragma unroll
                         for (int j = 0; j < 8; ++j)
                             dst[(qq * 8 + j) * kBM + r] =
