@@ -14,10 +14,11 @@
 // (distance << 32 | index) of a target over the tiles a CTA visits goes to a 64-bit atomicMin,
 // which is "smallest distance, then lowest index" whatever the split.
 //
-// Roles (256 threads): warp 0 TMA producer (the 128-target A tile, reloaded only when the
+// Roles (384 threads): warp 0 TMA producer (the 128-target A tile, reloaded only when the
 // target block changes, and the 256-reference B tile, double-buffered); warp 1 TMEM allocator
-// and MMA issuer (tcgen05.mma kind::f8f6f4, M=128, N=256, K=32); warps 4-7 epilogue
-// (tcgen05.ld, lane = target, running arg-max).  The (target block, reference block) tiles are
+// and MMA issuer (tcgen05.mma kind::f8f6f4, M=128, N=256, K=32); warps 4-11 epilogue
+// (tcgen05.ld, lane = target, running arg-max), two warps per TMEM lane quadrant, each reducing
+// one 128-column half of every tile.  The (target block, reference block) tiles are
 // split into one equal contiguous range per CTA, target blocks outermost.  Every pipeline wait
 // is bounded (SEMSHARE_FLAG_TIMEOUT), nothing traps.
 //
@@ -40,8 +41,10 @@ namespace {
 constexpr int kTM = 128;        // targets per tile (TMEM lanes)
 constexpr int kTN = 256;        // references per tile (MMA N)
 constexpr int kChunk = 128;     // bytes per 128-byte swizzle chunk along the code
-constexpr int kThreads = 256;
-constexpr int kEpiWarp0 = 4;
+constexpr int kEpiWarp0 = 4;   // a multiple of 4: epilogue warp w reads TMEM lanes 32*(w%4)
+constexpr int kEpiWarps = 8;   // two per lane quadrant, one per 128-column half of every tile
+constexpr int kHalfCols = kTN / 2;
+constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
 constexpr unsigned long long kNoKey = ~0ull;
 constexpr size_t kFixedSmem = 1024 + 256;
 
@@ -151,7 +154,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(bar_bfull + 8 * i, 1);
             mbar_init(bar_bempty + 8 * i, 1);
             mbar_init(bar_accfull + 8 * i, 1);
-            mbar_init(bar_accempty + 8 * i, 4);
+            mbar_init(bar_accempty + 8 * i, kEpiWarps);
         }
         mbar_init(bar_done, 1);
         *abort_flag = 0;
@@ -257,21 +260,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
     } else if (warp >= kEpiWarp0) {
         // ---------------- epilogue: best reference of every target row ----------------
-        // (per candidate in segmented mode; candidate cs covers columns [off[cs], next_b))
+        // (per candidate in segmented mode; candidate cs covers columns [off[cs], next_b)).  This
+        // warp reduces lanes 32*quad.. of columns [half*128, half*128 + 128) of every tile.
         const int ew = warp - kEpiWarp0;
-        const int r = ew * 32 + lane;
+        const int quad = ew & 3;
+        const int half = ew >> 2;
+        const int r = quad * 32 + lane;
         uint32_t acc = 0;
         int64_t cur_tb = -1, col0 = 0, next_b = 0;
         int32_t cs = 0;
         unsigned long long best = kNoKey;
-        // fold the tile's best key 256*dot - j (j = column within the tile) into `best`
+        // fold the best key 256*dot - j (j = column within this warp's half of the tile) into `best`
         auto fold = [&](float bk) {
             if (bk > -1.0e38f) {
                 const int ik = __float2int_rn(bk);
                 const int dot = -((-ik) >> 8);  // ceil(ik / 256)
-                const int j = 256 * dot - ik;    // 0..255
+                const int j = 256 * dot - ik;    // 0..127
                 const unsigned long long dist = static_cast<unsigned long long>((a.nbits - dot) >> 1);
-                const unsigned long long cand = (dist << 32) | static_cast<unsigned long long>(col0 + j);
+                const unsigned long long cand =
+                    (dist << 32) | static_cast<unsigned long long>(col0 + half * kHalfCols + j);
                 best = cand < best ? cand : best;
             }
         };
@@ -281,21 +288,32 @@ __global__ void __launch_bounds__(kThreads, 1)
                 atomicMin(a.keys + static_cast<int64_t>(cs) * a.n_tgt + g, best);
             best = kNoKey;
         };
+        auto advance = [&]() {
+            ++cs;
+            next_b = cs + 1 <= seg.n_seg ? seg.off[cs + 1] : a.n_ref;
+        };
         for (int64_t u = u0; u < u1; ++u, ++acc) {
             const int64_t tb = u / a.n_rb, rb = u - tb * a.n_rb;
             col0 = rb * kTN;
+            const int64_t h0 = col0 + half * kHalfCols;  // this warp's first column of the tile
             if (tb != cur_tb) {
                 if (cur_tb >= 0) flush();
                 cur_tb = tb;
                 best = kNoKey;
-                // candidate holding column col0: the largest cs with off[cs] <= col0
+                // candidate holding column h0: the largest cs with off[cs] <= h0
                 int lo = 0, hi = seg.n_seg - 1;
                 while (lo < hi) {
                     const int mid = (lo + hi + 1) >> 1;
-                    if (seg.off[mid] <= col0) lo = mid; else hi = mid - 1;
+                    if (seg.off[mid] <= h0) lo = mid; else hi = mid - 1;
                 }
                 cs = lo;
                 next_b = seg.off[lo + 1];
+            } else {
+                // the other half's columns lie in between: leave every candidate that ended there
+                while (next_b <= h0 && cs + 1 < seg.n_seg) {
+                    flush();
+                    advance();
+                }
             }
             const uint32_t buf = acc & 1u;
             const bool got = mbar_wait_bounded(bar_accfull + 8 * buf, (acc >> 1) & 1u, abort_flag, err,
@@ -307,52 +325,56 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after_sync();
             const int64_t rem = a.n_ref - col0;
             const int valid = rem < kTN ? static_cast<int>(rem) : kTN;
-            const uint32_t taddr = tmem_base + (static_cast<uint32_t>(ew * 32) << 16) + buf * kTN;
-            float bk = -3.0e38f;  // best key 256*dot - j of this tile (current candidate)
-            // 32-column chunks, double-buffered: the load of chunk q+1 is in flight while chunk
-            // q is reduced
-            uint32_t va[32], vb[32];
-            tmem_load_32cols(taddr, va);
-            tmem_load_wait_fence(va);
+            const int hv = valid - half * kHalfCols;  // valid columns of this half (may be <= 0)
+            const uint32_t taddr =
+                tmem_base + (static_cast<uint32_t>(quad * 32) << 16) + buf * kTN + half * kHalfCols;
+            float bk = -3.0e38f;  // best key 256*dot - j of this tile's half (current candidate)
+            if (hv > 0) {
+                // 32-column chunks, double-buffered: the load of chunk q+1 is in flight while
+                // chunk q is reduced
+                uint32_t va[32], vb[32];
+                tmem_load_32cols(taddr, va);
+                tmem_load_wait_fence(va);
 #pragma unroll
-            for (int q = 0; q < kTN / 32; ++q) {
-                uint32_t(&v)[32] = (q & 1) ? vb : va;
-                uint32_t(&vn)[32] = (q & 1) ? va : vb;
-                if (q + 1 < kTN / 32) tmem_load_32cols(taddr + (q + 1) * 32, vn);
-                const int64_t c0 = col0 + q * 32;
-                if (q * 32 + 32 <= valid && c0 + 32 <= next_b) {
-                    // four independent max chains (the keys are distinct: order does not matter)
-                    float m0 = -3.0e38f, m1 = -3.0e38f, m2 = -3.0e38f, m3 = -3.0e38f;
+                for (int q = 0; q < kHalfCols / 32; ++q) {
+                    uint32_t(&v)[32] = (q & 1) ? vb : va;
+                    uint32_t(&vn)[32] = (q & 1) ? va : vb;
+                    if (q + 1 < kHalfCols / 32) tmem_load_32cols(taddr + (q + 1) * 32, vn);
+                    const int tq = half * (kHalfCols / 32) + q;  // chunk index within the tile
+                    const int64_t c0 = col0 + tq * 32;
+                    if (q * 32 + 32 <= hv && c0 + 32 <= next_b) {
+                        // four independent max chains (the keys are distinct: order does not matter)
+                        float m0 = -3.0e38f, m1 = -3.0e38f, m2 = -3.0e38f, m3 = -3.0e38f;
 #pragma unroll
-                    for (int j = 0; j < 32; j += 4) {
-                        m0 = fmaxf(m0, fmaf(__uint_as_float(v[j]), 256.0f, -static_cast<float>(q * 32 + j)));
-                        m1 = fmaxf(m1, fmaf(__uint_as_float(v[j + 1]), 256.0f, -static_cast<float>(q * 32 + j + 1)));
-                        m2 = fmaxf(m2, fmaf(__uint_as_float(v[j + 2]), 256.0f, -static_cast<float>(q * 32 + j + 2)));
-                        m3 = fmaxf(m3, fmaf(__uint_as_float(v[j + 3]), 256.0f, -static_cast<float>(q * 32 + j + 3)));
+                        for (int j = 0; j < 32; j += 4) {
+                            m0 = fmaxf(m0, fmaf(__uint_as_float(v[j]), 256.0f, -static_cast<float>(q * 32 + j)));
+                            m1 = fmaxf(m1, fmaf(__uint_as_float(v[j + 1]), 256.0f, -static_cast<float>(q * 32 + j + 1)));
+                            m2 = fmaxf(m2, fmaf(__uint_as_float(v[j + 2]), 256.0f, -static_cast<float>(q * 32 + j + 2)));
+                            m3 = fmaxf(m3, fmaf(__uint_as_float(v[j + 3]), 256.0f, -static_cast<float>(q * 32 + j + 3)));
+                        }
+                        bk = fmaxf(bk, fmaxf(fmaxf(m0, m1), fmaxf(m2, m3)));
+                    } else if (q * 32 < hv) {
+                        // ragged end and/or candidate boundaries inside the chunk: runs [js, je)
+                        const int jend = hv - q * 32 < 32 ? hv - q * 32 : 32;
+                        int js = 0;
+                        for (;;) {
+                            const int64_t lim_b = next_b - c0;  // >= js: the boundary is not passed yet
+                            const int je = lim_b < jend ? static_cast<int>(lim_b) : jend;
+#pragma unroll
+                            for (int j = 0; j < 32; ++j)
+                                if (j >= js && j < je)
+                                    bk = fmaxf(bk, fmaf(__uint_as_float(v[j]), 256.0f, -static_cast<float>(q * 32 + j)));
+                            if (je == jend) break;
+                            // column c0 + je opens candidate cs + 1
+                            fold(bk);
+                            bk = -3.0e38f;
+                            flush();
+                            advance();
+                            js = je;
+                        }
                     }
-                    bk = fmaxf(bk, fmaxf(fmaxf(m0, m1), fmaxf(m2, m3)));
-                } else if (q * 32 < valid) {
-                    // ragged end and/or candidate boundaries inside the chunk: runs [js, je)
-                    const int jend = valid - q * 32 < 32 ? valid - q * 32 : 32;
-                    int js = 0;
-                    for (;;) {
-                        const int64_t lim_b = next_b - c0;  // >= js: the boundary is not passed yet
-                        const int je = lim_b < jend ? static_cast<int>(lim_b) : jend;
-#pragma unroll
-                        for (int j = 0; j < 32; ++j)
-                            if (j >= js && j < je)
-                                bk = fmaxf(bk, fmaf(__uint_as_float(v[j]), 256.0f, -static_cast<float>(q * 32 + j)));
-                        if (je == jend) break;
-                        // column c0 + je opens candidate cs + 1
-                        fold(bk);
-                        bk = -3.0e38f;
-                        flush();
-                        ++cs;
-                        next_b = cs + 1 <= seg.n_seg ? seg.off[cs + 1] : a.n_ref;
-                        js = je;
-                    }
+                    if (q + 1 < kHalfCols / 32) tmem_load_wait_fence(vn);
                 }
-                if (q + 1 < kTN / 32) tmem_load_wait_fence(vn);
             }
             tc_fence_before_sync();
             __syncwarp();
