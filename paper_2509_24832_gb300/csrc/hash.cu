@@ -240,7 +240,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem_slot = bar_mma_done + 8u;
     volatile uint32_t* const tmem_slot_ptr = reinterpret_cast<volatile uint32_t*>(gbase + (tmem_slot - sbase));
     volatile int* const abort_flag = reinterpret_cast<volatile int*>(gbase + (tmem_slot + 4u - sbase));
-    volatile uint32_t* const arrival = reinterpret_cast<volatile uint32_t*>(gbase + (tmem_slot + 8u - sbase));
     // hand-off bookkeeping shared with the end phase: [0] final partial staged (0/1), [1] its tile,
     // [2] its slot, [3] b_lo, [4] b_hi, [5] fix-ups pending, [6 + 3f ..] tile, b_lo, b_hi of fix-up f
     volatile int64_t* const ctl = reinterpret_cast<volatile int64_t*>(gbase + (tmem_slot + 16u - sbase));
