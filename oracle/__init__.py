@@ -15,6 +15,7 @@ it follows, is stated in `semshare_oracle.c`:
   kv_deviation  sigma_K + sigma_V per layer and token; App. A.4
   select_hd     the k highest-deviation tokens per layer; Insight 1, Sec. 3.2
   gather_kv_retained  the rearranged rows of each layer's retained tokens only; Sec. 3.3.4, App. A
+  fetch_rows    the reference rows the match selects, loaded once each; Sec. 3.2, Sec. 3.3
 
 Parity pins: every function here is pinned by `tests/test_oracle_*.py` against closed forms,
 invariants, hand-derived golden cases and brute force (none is "parity unpinned").
@@ -77,6 +78,8 @@ def _load():
         lib.oracle_select_hd.argtypes = [P, i32, i64, i64, P]
         lib.oracle_gather_kv_retained.argtypes = [P, P, i32, i32, i64, i64, P, i64, P, P, i64, P, P]
         lib.oracle_gather_kv_retained.restype = i64
+        lib.oracle_fetch_rows.argtypes = [P, P, P, P, P, i32, i32, i32, i64, P, i64]
+        lib.oracle_fetch_rows.restype = i64
         _lib = lib
         return lib
 
@@ -270,3 +273,35 @@ def gather_kv_retained(ref_k, ref_v, idx, retained, cap: int | None = None, out_
     bad = _load().oracle_gather_kv_retained(_ptr(ref_k), _ptr(ref_v), L, H, N, hd * ref_k.dtype.itemsize, _ptr(idx),
                                             len(idx), _ptr(flat), _ptr(off), cap, _ptr(out_k), _ptr(out_v))
     return out_k, out_v, int(bad)
+
+
+def fetch_rows(seg_k, seg_v, idx, dev_k=None, dev_v=None):
+    """Selected-row load (Sec. 3.2, Sec. 3.3): seg_k/seg_v one [L][H][n_s][hd] array per reference
+    segment (or a single array); dev_k/dev_v arrays of the same shapes (zeros when None) receive,
+    for every l, h, the rows named in idx (global rows, any order, repeats allowed); all other
+    rows stay as given.  Returns (dev_k, dev_v, n_bad), lists when seg_k is a list."""
+    as_list = not isinstance(seg_k, np.ndarray)
+    seg_k = [np.ascontiguousarray(a) for a in (seg_k if as_list else [seg_k])]
+    seg_v = [np.ascontiguousarray(a) for a in (seg_v if as_list else [seg_v])]
+    L, H, _, hd = seg_k[0].shape
+    dt = seg_k[0].dtype
+    if dev_k is None:
+        dev_k = [np.zeros_like(a) for a in seg_k]
+    if dev_v is None:
+        dev_v = [np.zeros_like(a) for a in seg_v]
+    dev_k = [dev_k] if isinstance(dev_k, np.ndarray) else list(dev_k)
+    dev_v = [dev_v] if isinstance(dev_v, np.ndarray) else list(dev_v)
+    offs = np.zeros(len(seg_k) + 1, dtype=np.int64)
+    for s, a in enumerate(seg_k):
+        if a.shape[:2] != (L, H) or a.shape[3] != hd or seg_v[s].shape != a.shape:
+            raise ValueError("segment shapes differ")
+        if dev_k[s].shape != a.shape or dev_v[s].shape != a.shape or not dev_k[s].flags.c_contiguous \
+                or not dev_v[s].flags.c_contiguous:
+            raise ValueError("dev arrays must be contiguous and shaped like the segments")
+        offs[s + 1] = offs[s] + a.shape[2]
+    idx = np.ascontiguousarray(np.asarray(idx, dtype=np.int32).ravel())
+    n = len(seg_k)
+    arr = lambda xs: (ctypes.c_void_p * n)(*[a.ctypes.data for a in xs])  # noqa: E731
+    bad = _load().oracle_fetch_rows(arr(seg_k), arr(seg_v), arr(dev_k), arr(dev_v), _ptr(offs), n, L, H,
+                                    hd * dt.itemsize, _ptr(idx), len(idx))
+    return (dev_k, dev_v, int(bad)) if as_list else (dev_k[0], dev_v[0], int(bad))

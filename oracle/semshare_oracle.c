@@ -358,3 +358,35 @@ int64_t oracle_gather_kv_retained(const uint8_t* ref_k, const uint8_t* ref_v, in
         }
     return bad;
 }
+
+/* ---- loading the selected reference rows ---------------------------------------------------- */
+
+/* Sec. 3.2 loads the retrieved reference prompt's KV cache onto the GPU before the rearrangement
+ * of Sec. 3.3, which reads only the rows the match selects.  This copies, for every layer l and
+ * head h, each reference row r named by some idx[i] (i < n_idx) from seg_k/seg_v to dev_k/dev_v
+ * (both laid out per segment as [L][H][n_s][row_bytes], as in oracle_gather_kv); every other row
+ * of dev_k/dev_v is left as it was.  An idx outside [0, seg_offsets[n_seg]) is skipped and
+ * counted; returns the count. */
+int64_t oracle_fetch_rows(const uint8_t* const* seg_k, const uint8_t* const* seg_v, uint8_t* const* dev_k,
+                          uint8_t* const* dev_v, const int64_t* seg_offsets, int32_t n_seg, int32_t L, int32_t H,
+                          int64_t row_bytes, const int32_t* idx, int64_t n_idx) {
+    const int64_t total = seg_offsets[n_seg];
+    int64_t bad = 0;
+    for (int64_t i = 0; i < n_idx; ++i) {
+        const int64_t r = idx[i];
+        if (r < 0 || r >= total) {
+            ++bad;
+            continue;
+        }
+        int32_t s = 0;
+        while (!(seg_offsets[s] <= r && r < seg_offsets[s + 1])) ++s;
+        const int64_t n_s = seg_offsets[s + 1] - seg_offsets[s];
+        for (int32_t l = 0; l < L; ++l)
+            for (int32_t h = 0; h < H; ++h) {
+                const int64_t off = (((int64_t)l * H + h) * n_s + (r - seg_offsets[s])) * row_bytes;
+                memcpy(dev_k[s] + off, seg_k[s] + off, (size_t)row_bytes);
+                memcpy(dev_v[s] + off, seg_v[s] + off, (size_t)row_bytes);
+            }
+    }
+    return bad;
+}
