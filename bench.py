@@ -354,12 +354,19 @@ class Problem:
             if ev:
                 ev[5].record()
 
-    def e2e_plan(self, copy_all: bool = False):
-        """(one, h2d, d2h, read): a step through the public API with host buffers.  The embedding
-        rows and positions are copied in from pinned host memory; the reference K/V cache stays in
-        pinned host memory and the gather reads the rows the match selects across the host link in
-        place (copy_all: the whole cache is copied in first, then gathered from HBM); the match
-        result (idx, dist) is copied back."""
+    def unique_rows(self) -> int:
+        """Distinct reference rows the current match selects (over every target prompt)."""
+        return int(np.unique(self.idx.cpu().numpy()).size)
+
+    def e2e_plan(self, mode: str = "fetch"):
+        """(one, h2d, d2h, read): a step through the public API with host buffers.  The
+        embedding rows and positions are copied in from pinned host memory; the reference K/V cache
+        stays in pinned host memory, and the gather's rows reach it one of three ways (`mode`):
+          fetch     semshare_fetch_rows copies each row the match selects into HBM once, then the
+                    gather runs on HBM;
+          inplace   the gather reads every selected row across the host link, repeats included;
+          copy_all  the whole cache is copied in first, then gathered from HBM.
+        The match result (idx, dist) is copied back."""
         import torch
 
         h_emb = self.emb.cpu().pin_memory()
@@ -368,22 +375,25 @@ class Problem:
         h_v = [t.cpu().pin_memory() for t in self.ref_v]
         h_idx = torch.empty_like(self.idx, device="cpu").pin_memory()
         h_dist = torch.empty_like(self.dist, device="cpu").pin_memory()
-        wl = self.wl
-        L, H, hd = wl.kv
-        rows = float(sum(self.counts)) * H if getattr(self, "retain", False) else float(wl.n_batch * wl.n_tgt) * L * H
-        kv_bytes = sum(t.numel() * t.element_size() for t in h_k + h_v) if copy_all else rows * hd * 2 * 2
+        kv_bytes = self.e2e_kv_bytes()[mode]
         h2d = h_emb.numel() * h_emb.element_size() + h_pos.numel() * 4 + kv_bytes
         d2h = (h_idx.numel() + h_dist.numel()) * 4
-        src_k, src_v = (self.ref_k, self.ref_v) if copy_all else (h_k, h_v)
+        ss = self.ss
+        fetch_ws = torch.empty(max(16, ss.semshare_fetch_workspace_size(self.wl.n_ref)), dtype=torch.uint8,
+                               device=self.dev)
+        src_k, src_v = (h_k, h_v) if mode == "inplace" else (self.ref_k, self.ref_v)
 
         def one():
             self.emb.copy_(h_emb, non_blocking=True)
             self.pos.copy_(h_pos, non_blocking=True)
-            if copy_all:
+            if mode == "copy_all":
                 for d, h in zip(self.ref_k + self.ref_v, h_k + h_v):
                     d.copy_(h, non_blocking=True)
             self.hash()
             self.match()
+            if mode == "fetch":
+                ss.semshare_fetch_rows(h_k, h_v, self.idx, dev_k=self.ref_k, dev_v=self.ref_v, workspace=fetch_ws,
+                                       err_flag=self.flag)
             self.gather(src_k, src_v)
             if self.hd:
                 self.deviation()
@@ -392,6 +402,15 @@ class Problem:
             h_dist.copy_(self.dist, non_blocking=True)
 
         return one, h2d, d2h, lambda: int(h_idx[0])
+
+    def e2e_kv_bytes(self) -> dict:
+        """K/V bytes crossing the host link per step in each e2e mode."""
+        wl = self.wl
+        L, H, hd = wl.kv
+        row = hd * 2 * 2  # a K and a V row, bf16
+        gathered = float(sum(self.counts)) * H if self.retain else float(wl.n_batch * wl.n_tgt) * L * H
+        return {"inplace": gathered * row, "fetch": float(self.unique_rows()) * L * H * row,
+                "copy_all": float(sum(t.numel() * t.element_size() for t in self.ref_k + self.ref_v))}
 
 
 class RetrieveProblem:
@@ -459,8 +478,8 @@ class RetrieveProblem:
         self.out_k = torch.empty((1, L, H, n_t, hd), dtype=torch.bfloat16, device=device)
         self.out_v = torch.empty_like(self.out_k)
         self.winner = -1
-        self.load_winner = None  # e2e (copy_all): copies the winner's K/V cache in from host memory
-        self.gather_src = None   # e2e: the stored caches in pinned host memory, read in place
+        self.load_winner = None  # e2e: brings the winner's K/V rows (or whole cache) in from host memory
+        self.gather_src = None   # e2e (inplace): the stored caches in pinned host memory, read in place
 
     def step(self, ev=None):
         ss, wl = self.ss, self.wl
@@ -499,12 +518,23 @@ class RetrieveProblem:
         if ev:
             ev[5].record()
 
-    def e2e_plan(self, copy_all: bool = False):
+    def unique_rows(self) -> int:
+        return int(np.unique(self.idx.cpu().numpy()).size)
+
+    def e2e_kv_bytes(self) -> dict:
+        L, H, hd = self.wl.kv
+        row = hd * 2 * 2
+        return {"inplace": float(self.wl.n_tgt) * L * H * row, "fetch": float(self.unique_rows()) * L * H * row,
+                "copy_all": float(self.ref_k[0].numel() * self.ref_k[0].element_size() * 2)}
+
+    def e2e_plan(self, mode: str = "fetch"):
         """(one, h2d, d2h, read): the target's embedding rows and positions copied in; the stored
-        prompts' K/V caches stay in pinned host memory and, once the winner is known, the gather
-        reads the rows it needs from the winner's cache in place (copy_all: the winner's whole
-        cache is copied in first -- Sec. 3.2 loads the retrieved prompt onto the GPU with its KV
-        cache); the winner and the match result (idx, dist) copied back."""
+        prompts' K/V caches stay in pinned host memory and, once the winner is known, the gather's
+        rows reach it one of three ways (`mode`): fetch -- semshare_fetch_rows copies each row the
+        match selects from the winner's cache into HBM once; inplace -- the gather reads them across
+        the host link, repeats included; copy_all -- the winner's whole cache is copied in first
+        (Sec. 3.2 loads the retrieved prompt onto the GPU with its KV cache).  The winner and the
+        match result (idx, dist) are copied back."""
         import torch
 
         h_emb = self.emb.cpu().pin_memory()
@@ -513,22 +543,28 @@ class RetrieveProblem:
         h_v = [t.cpu().pin_memory() for t in self.ref_v]
         h_idx = torch.empty_like(self.idx, device="cpu").pin_memory()
         h_dist = torch.empty_like(self.dist, device="cpu").pin_memory()
-        L, H, hd = self.wl.kv
-        kv_bytes = h_k[0].numel() * h_k[0].element_size() * 2 if copy_all else float(self.wl.n_tgt) * L * H * hd * 2 * 2
+        kv_bytes = self.e2e_kv_bytes()[mode]
         h2d = h_emb.numel() * h_emb.element_size() + h_pos.numel() * 4 + kv_bytes
         d2h = (h_idx.numel() + h_dist.numel()) * 4 + self.h_choice.numel() * 4
+        ss = self.ss
+        fetch_ws = torch.empty(max(16, ss.semshare_fetch_workspace_size(self.wl.seg_len)), dtype=torch.uint8,
+                               device=self.dev)
 
         def load(m):
-            self.ref_k[m].copy_(h_k[m], non_blocking=True)
-            self.ref_v[m].copy_(h_v[m], non_blocking=True)
+            if mode == "copy_all":
+                self.ref_k[m].copy_(h_k[m], non_blocking=True)
+                self.ref_v[m].copy_(h_v[m], non_blocking=True)
+            else:
+                ss.semshare_fetch_rows(h_k[m], h_v[m], self.idx, dev_k=self.ref_k[m], dev_v=self.ref_v[m],
+                                       workspace=fetch_ws, err_flag=self.flag)
 
         def one():
             self.emb.copy_(h_emb, non_blocking=True)
             self.pos.copy_(h_pos, non_blocking=True)
-            if copy_all:
-                self.load_winner = load
-            else:
+            if mode == "inplace":
                 self.gather_src = (h_k, h_v)
+            else:
+                self.load_winner = load
             try:
                 self.step()
             finally:
@@ -687,17 +723,15 @@ def run_gpu_arm(args, rank, world, local_rank):
     roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"
     roof["traffic"] = tr["bytes_per_launch"] if tr and tr.get("sha") == kernel_sha(tr["file"]) else None
 
-    # e2e: the reference K/V cache is read in place from pinned host memory when the rows the gather
-    # selects are no more than the cache holds (each crosses the host link once), and copied to HBM
-    # first when the cache is reused more than that (e.g. 64 target prompts against one reference);
-    # the other way is reported beside it
-    L, H, _ = wl.kv
-    gathered = (float(sum(prob.counts)) * H if getattr(prob, "retain", False)
-                else float(wl.n_batch * wl.n_tgt) * L * H)
-    cache = float(wl.seg_len if isinstance(prob, RetrieveProblem) else wl.n_ref) * L * H
-    in_place = gathered <= cache
-    e2e = run_e2e(args, prob, device, copy_all=not in_place)
-    e2e_alt = run_e2e(args, prob, device, copy_all=in_place)
+    # e2e: the reference K/V cache lives in pinned host memory and its rows reach the gather one of
+    # three ways (Problem.e2e_plan).  The headline mode is the one a cost model of the step's K/V
+    # movement picks: host-link bytes at HOST_LINK_GBS plus HBM bytes at the measured copy rate
+    # (fetch and copy_all write the rows to HBM and the gather then reads and writes them again;
+    # inplace only writes the gathered rows).  The other modes are measured and reported beside it.
+    kv_bytes = prob.e2e_kv_bytes()
+    mode = e2e_mode(kv_bytes, peaks["hbm_gbs"])
+    e2e = run_e2e(args, prob, device, mode)
+    e2e_alt = {m: run_e2e(args, prob, device, m) for m in E2E_KV if m != mode}
     ref_cached = run_ref_codes_cached(args, prob, device, flush) if isinstance(prob, Problem) else None
 
     cpu = None
@@ -797,13 +831,37 @@ class _Null:
         return False
 
 
-def run_e2e(args, prob, device, copy_all: bool = False):
+# Pinned host memory -> HBM on GB300, measured with the copy engines, with semshare_fetch_rows and with
+# the gather reading in place: all three move about 211 GB/s, for whole caches and for 30% of the rows.
+HOST_LINK_GBS = 211.0
+
+
+def e2e_mode(kv_bytes: dict, hbm_gbs: float) -> str:
+    """The e2e mode with the least estimated K/V movement time; ties go to the bulk copy."""
+    gathered = kv_bytes["inplace"]
+    hbm = {"inplace": gathered, "fetch": kv_bytes["fetch"] + 2 * gathered,
+           "copy_all": kv_bytes["copy_all"] + 2 * gathered}
+    order = ("copy_all", "fetch", "inplace")
+    cost = {m: kv_bytes[m] / (HOST_LINK_GBS * 1e9) + hbm[m] / (hbm_gbs * 1e9) for m in order}
+    return min(order, key=lambda m: (round(cost[m], 7), order.index(m)))
+
+
+E2E_KV = {
+    "fetch": "reference cache in pinned host memory; semshare_fetch_rows copies each selected row into HBM "
+             "once, then the gather runs on HBM",
+    "inplace": "reference cache in pinned host memory; the gather reads the selected rows in place "
+               "(h2d counts every selected row; repeats may be served by L2)",
+    "copy_all": "reference cache copied to HBM every step, then gathered",
+}
+
+
+def run_e2e(args, prob, device, mode: str = "fetch"):
     """Same metric through the public API with host buffers (the problem's e2e_plan says which
     inputs are copied in and which results are read back every step)."""
     import torch
 
     wl = prob.wl
-    one, h2d, d2h, read = prob.e2e_plan(copy_all=copy_all)
+    one, h2d, d2h, read = prob.e2e_plan(mode)
     for _ in range(3):
         one()
     torch.cuda.synchronize()
@@ -819,12 +877,8 @@ def run_e2e(args, prob, device, copy_all: bool = False):
         times.append(a.elapsed_time(b))
     ms = reduce_max(float(np.mean(times)), device)
     _, world, _ = dist_info()
-    out = {"value": world * wl.n_batch * wl.n_tgt / (ms * 1e-3), "unit": "tokens/s", "ms_per_step": ms,
-           "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
-    out["kv"] = ("reference cache copied to HBM every step, then gathered" if copy_all else
-                 "reference cache in pinned host memory; the gather reads the selected rows in place "
-                 "(h2d counts every selected row once; repeats may be served by L2)")
-    return out
+    return {"value": world * wl.n_batch * wl.n_tgt / (ms * 1e-3), "unit": "tokens/s", "ms_per_step": ms,
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "mode": mode, "kv": E2E_KV[mode]}
 
 
 # ---- CPU oracle (baseline leg and reference arm) -----------------------------------------------

@@ -342,6 +342,38 @@ semshare_status semshare_gather_kv_retained(const void* const* ref_k, const void
                                             semshare_kv_layout dst, uint32_t* err_flag, void* stream);
 
 /*
+ * semshare_fetch_rows -- bring the reference rows a match selects into device memory, each once.
+ *
+ * Sec. 3.2 loads the retrieved reference prompt onto the GPU with its KV cache before the
+ * rearrangement of Sec. 3.3, which reads only the rows the match selects -- and several target
+ * tokens often select the same row.  For every layer l, KV head h and global reference row r
+ * that some idx[i] (i < n_idx) names:
+ *     dev_k[s][l][h][r - seg_offsets[s]][:] = ref_k[s][l][h][r - seg_offsets[s]][:]  (same for V)
+ * with s the segment of r.  Rows that no idx names are neither read nor written, so a row
+ * selected by many targets crosses the host link once; semshare_gather_kv (or _retained) with
+ * ref_k/ref_v replaced by dev_k/dev_v and the same idx then gives the same result as on the
+ * original cache.  Copies are bitwise.
+ *
+ *   ref_k, ref_v     host arrays of n_seg source base pointers: device memory or page-locked
+ *                    host memory the device can address
+ *   dev_k, dev_v     host arrays of n_seg device base pointers, each segment laid out like its
+ *                    source (same strides, `layout`); may not overlap the sources
+ *   seg_offsets, n_seg, layout   as seg_offsets, n_seg and src of semshare_gather_kv
+ *   idx              device int32[n_idx]: global reference rows (any order, repeats allowed)
+ *   workspace        device scratch of at least semshare_fetch_workspace_size(n_rows) bytes,
+ *                    n_rows = seg_offsets[n_seg]; the call rewrites all of it
+ *   err_flag         device or NULL; an idx outside [0, n_rows) is skipped and sets
+ *                    SEMSHARE_FLAG_INDEX
+ * Alignment rules as for semshare_gather_kv.  n_idx = 0 or n_rows = 0 launches nothing.
+ * Returns EINVAL for bad arguments, EUNSUPPORTED for n_rows >= 2^31, ECUDA if a launch fails.
+ */
+size_t semshare_fetch_workspace_size(int64_t n_rows);
+semshare_status semshare_fetch_rows(const void* const* ref_k, const void* const* ref_v, void* const* dev_k,
+                                    void* const* dev_v, const int64_t* seg_offsets, int32_t n_seg,
+                                    semshare_kv_layout layout, const int32_t* idx, int64_t n_idx, void* workspace,
+                                    size_t workspace_bytes, uint32_t* err_flag, void* stream);
+
+/*
  * semshare_kv_deviation -- Key-Value deviation of the reused cache (App. A.4).
  *
  * sigma_K = ||K_reused - K_recomputed||_2, sigma_V likewise, sigma_KV = sigma_K + sigma_V

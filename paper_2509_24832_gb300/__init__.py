@@ -32,6 +32,8 @@ from ._native import (  # noqa: F401
     new_err_flag,
     retain_counts,
     semshare_abi_version,
+    semshare_fetch_rows,
+    semshare_fetch_workspace_size,
     semshare_gather_kv,
     semshare_gather_kv_retained,
     semshare_hash,

@@ -83,6 +83,10 @@ def load():
         lib.semshare_gather_kv.restype = ctypes.c_int
         lib.semshare_gather_kv_retained.argtypes = [P, P, P, i32, KVLayout, P, i64, P, P, P, P, KVLayout, P, P]
         lib.semshare_gather_kv_retained.restype = ctypes.c_int
+        lib.semshare_fetch_workspace_size.argtypes = [i64]
+        lib.semshare_fetch_workspace_size.restype = ctypes.c_size_t
+        lib.semshare_fetch_rows.argtypes = [P, P, P, P, P, i32, KVLayout, P, i64, P, ctypes.c_size_t, P, P]
+        lib.semshare_fetch_rows.restype = ctypes.c_int
         lib.semshare_kv_deviation.argtypes = [P, P, KVLayout, P, P, KVLayout, ctypes.c_int, i64, P, P, P, P]
         lib.semshare_kv_deviation.restype = ctypes.c_int
         lib.semshare_select_hd.argtypes = [P, i32, i64, i64, P, P, P]
@@ -437,6 +441,63 @@ def semshare_gather_kv(ref_k, ref_v, idx: torch.Tensor, out_k: torch.Tensor | No
                                    _ptr(err_flag), _stream(stream))
     _check(st, "semshare_gather_kv")
     return out_k, out_v
+
+
+def semshare_fetch_workspace_size(n_rows: int) -> int:
+    return int(load().semshare_fetch_workspace_size(int(n_rows)))
+
+
+def semshare_fetch_rows(ref_k, ref_v, idx: torch.Tensor, dev_k=None, dev_v=None, workspace: torch.Tensor | None = None,
+                        err_flag: torch.Tensor | None = None, stream=None):
+    """Copies the reference rows idx selects -- each once, whatever its count in idx -- from
+    ref_k/ref_v (CUDA or pinned host tensors [L][H][N][hd], or lists of them sharing one layout)
+    into device caches dev_k/dev_v of the same shapes and strides (allocated on idx.device when
+    None).  Rows no idx names are left as they were.  Returns (dev_k, dev_v), lists when the
+    sources are lists; semshare_gather_kv on them with the same idx gives the gather of the
+    sources."""
+    as_list = isinstance(ref_k, (list, tuple))
+    seg_k = list(ref_k) if as_list else [ref_k]
+    seg_v = list(ref_v) if isinstance(ref_v, (list, tuple)) else [ref_v]
+    if len(seg_k) != len(seg_v) or not seg_k:
+        raise ValueError("ref_k and ref_v must have the same number of segments")
+    for t in seg_k + seg_v:
+        _need_device_accessible(t, "ref")
+    lay = kv_layout(seg_k[0], batched=False)
+    for t in seg_k[1:] + seg_v:
+        o = kv_layout(t, batched=False)
+        if (o.stride_layer, o.stride_head, o.stride_token, o.head_dim, o.elem_bytes) != \
+                (lay.stride_layer, lay.stride_head, lay.stride_token, lay.head_dim, lay.elem_bytes):
+            raise ValueError("all segments must share one layout")
+    _need_cuda(idx, "idx")
+    if idx.dtype != torch.int32 or not idx.is_contiguous():
+        raise ValueError("idx must be contiguous int32")
+
+    def like(ts):
+        return [torch.empty_strided(t.shape, t.stride(), dtype=t.dtype, device=idx.device) for t in ts]
+
+    dk = like(seg_k) if dev_k is None else (list(dev_k) if isinstance(dev_k, (list, tuple)) else [dev_k])
+    dv = like(seg_v) if dev_v is None else (list(dev_v) if isinstance(dev_v, (list, tuple)) else [dev_v])
+    if len(dk) != len(seg_k) or len(dv) != len(seg_v):
+        raise ValueError("dev_k/dev_v need one tensor per segment")
+    for d, t in zip(dk + dv, seg_k + seg_v):
+        _need_cuda(d, "dev")
+        if d.shape != t.shape or d.stride() != t.stride() or d.dtype != t.dtype:
+            raise ValueError("dev_k/dev_v must have the shapes, strides and dtype of ref_k/ref_v")
+    n_seg = len(seg_k)
+    offs = [0]
+    for t in seg_k:
+        offs.append(offs[-1] + t.shape[2])
+    if workspace is None:
+        workspace = torch.empty(max(semshare_fetch_workspace_size(offs[-1]), 16), dtype=torch.uint8,
+                                device=idx.device)
+    _need_cuda(workspace, "workspace")
+    arr = lambda ts: (ctypes.c_void_p * n_seg)(*[t.data_ptr() for t in ts])  # noqa: E731
+    po = (ctypes.c_int64 * (n_seg + 1))(*offs)
+    st = load().semshare_fetch_rows(arr(seg_k), arr(seg_v), arr(dk), arr(dv), po, n_seg, lay, _ptr(idx), idx.numel(),
+                                    _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(err_flag),
+                                    _stream(stream))
+    _check(st, "semshare_fetch_rows")
+    return (dk, dv) if as_list else (dk[0], dv[0])
 
 
 HD_PERCENT = 40  # Insight 1: the 40% of tokens with the highest deviation are HD tokens

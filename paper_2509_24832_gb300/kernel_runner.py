@@ -65,7 +65,7 @@ def _retrieval(a, wl, e, pd, R, table, flag, dev):
 def main(argv=None):
     p = argparse.ArgumentParser()
     p.add_argument("--kernel", choices=["hash", "match", "match_tc", "gather", "gather_retained", "retrieve",
-                                        "deviation", "select"], required=True)
+                                        "deviation", "select", "fetch"], required=True)
     p.add_argument("--workload", default="llama8b-5k", choices=sorted(ALL))
     p.add_argument("--reps", type=int, default=3)
     a = p.parse_args(argv)
@@ -111,6 +111,16 @@ def main(argv=None):
                 out_v = torch.empty_like(out_k)
                 for _ in range(a.reps):
                     ss.semshare_gather_kv_retained(k, v, idx, flat, offs, out_k=out_k, out_v=out_v, err_flag=flag)
+            elif a.kernel == "fetch":
+                # the selected rows from a reference cache in pinned host memory into HBM
+                del e
+                segs = [workloads.kv_cache_device(wl, dev, segment=s) for s in range(wl.n_seg)]
+                hk = [s[0].cpu().pin_memory() for s in segs]
+                hv = [s[1].cpu().pin_memory() for s in segs]
+                dk = [s[0] for s in segs]
+                dv = [s[1] for s in segs]
+                for _ in range(a.reps):
+                    ss.semshare_fetch_rows(hk, hv, idx, dev_k=dk, dev_v=dv, err_flag=flag)
             elif a.kernel == "gather":
                 del e
                 segs = [workloads.kv_cache_device(wl, dev, segment=s) for s in range(wl.n_seg)]

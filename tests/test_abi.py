@@ -158,6 +158,33 @@ def test_gather_retained_argument_errors(lib):
     assert g(pk, pk, offs, 1, lay, None, 10, None, ro(0, 0, 0), None, None, out, None, None) == 0  # nothing kept
 
 
+def test_fetch_argument_errors(lib):
+    import paper_2509_24832_gb300 as ss
+
+    lay = ss.KVLayout(2, 4, 64, 2, 0, 4 * 100 * 64, 100 * 64, 64)
+    pk = (ctypes.c_void_p * 1)(1 << 20)
+    pd = (ctypes.c_void_p * 1)(1 << 21)
+    offs = (ctypes.c_int64 * 2)(0, 100)
+    f = lib.semshare_fetch_rows
+    ws = lib.semshare_fetch_workspace_size(100)
+    assert ws >= 100 and lib.semshare_fetch_workspace_size(0) == 0
+    assert f(pk, pk, pd, pd, offs, 0, lay, FAKE, 10, FAKE, ws, None, None) == 1            # n_seg
+    bad = ss.KVLayout(2, 4, 60, 2, 0, 4 * 100 * 60, 100 * 60, 60)                           # 120-byte rows
+    assert f(pk, pk, pd, pd, offs, 1, bad, FAKE, 10, FAKE, ws, None, None) == 1
+    odd = ss.KVLayout(2, 4, 64, 2, 0, 4 * 100 * 64 + 4, 100 * 64, 64)                       # stride not 16 B
+    assert f(pk, pk, pd, pd, offs, 1, odd, FAKE, 10, FAKE, ws, None, None) == 1
+    nul = (ctypes.c_void_p * 1)(None)
+    assert f(pk, pk, nul, pd, offs, 1, lay, FAKE, 10, FAKE, ws, None, None) == 1            # no destination
+    assert f(pk, pk, pd, pd, offs, 1, lay, None, 10, FAKE, ws, None, None) == 1             # no idx
+    assert f(pk, pk, pd, pd, offs, 1, lay, FAKE, 10, FAKE, ws - 1, None, None) == 1        # workspace too small
+    assert f(pk, pk, pd, pd, offs, 1, lay, FAKE, -1, FAKE, ws, None, None) == 1             # negative count
+    offs_bad = (ctypes.c_int64 * 2)(5, 100)
+    assert f(pk, pk, pd, pd, offs_bad, 1, lay, FAKE, 10, FAKE, ws, None, None) == 1
+    huge = (ctypes.c_int64 * 2)(0, 1 << 31)
+    assert f(pk, pk, pd, pd, huge, 1, lay, FAKE, 10, FAKE, ws, None, None) == 2
+    assert f(pk, pk, pd, pd, offs, 1, lay, None, 0, None, 0, None, None) == 0               # empty
+
+
 def test_deviation_and_select_argument_errors(lib):
     import paper_2509_24832_gb300 as ss
 
