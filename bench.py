@@ -11,8 +11,9 @@ value = target tokens of all ranks / max over ranks of the mean device time of a
 `--workload retrieve-16x4096` times the path with reference retrieval in front (Sec. 3.2):
 16 stored prompts whose codes were computed when they were stored; per step the target is
 hashed without rotary encoding, the most similar stored prompt is retrieved
-(semshare_retrieve), the target is hashed with it, matched against the winner's codes and the
-winner's K/V cache is gathered.
+(semshare_retrieve), the target is hashed with it, matched against the winner's codes
+(semshare_match_tc_selected reads the choice on the device) and the winner's K/V rows are
+gathered -- all enqueued back to back, with no host round trip.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl gb300|reference]
 
@@ -420,11 +421,12 @@ class RetrieveProblem:
       hash_plain  codes of the target rows without rotary encoding (retrieval precedes it)
       retrieve    similarity to every stored prompt, the best one (semshare_retrieve)
       hash        codes of the target rows with rotary encoding (Sec. 3.3.1)
-      match       1-NN against the winner's rotary codes (the host reads the winner first)
-      gather      the winner's K/V rows in the target's order"""
+      match       1-NN against the winner's rotary codes (the choice is read on the device)
+      gather      the winner's K/V rows in the target's order (pool rows over every member)"""
 
     STAGES = ("hash_plain", "retrieve", "hash", "match", "gather")
-    # hash 1, retrieve 3 (expand + key reset, search, per-candidate reduction), hash 1, match 3, gather 1
+    # hash 1, retrieve 3 (expand + key reset, search, per-candidate reduction), hash 1,
+    # selected match 3 (expand, search, split), gather 1
     LAUNCHES_PER_STEP = 9
 
     def __init__(self, wl: workloads.Workload, device, seed: int, matcher: str = "tc"):
@@ -469,19 +471,25 @@ class RetrieveProblem:
         self.h_choice = torch.zeros(2, dtype=torch.int32).pin_memory()
         self.idx = torch.empty(n_t, dtype=torch.int32, device=device)
         self.dist = torch.empty(n_t, dtype=torch.int32, device=device)
-        self.tc_ws = torch.empty(ss.semshare_match_tc_workspace_size(n_t, wl.seg_len, wl.nbits), dtype=torch.uint8,
-                                 device=device)
+        self.tc_ws = torch.empty(ss.semshare_match_tc_selected_workspace_size(n_t, self.offsets, wl.nbits),
+                                 dtype=torch.uint8, device=device)
         segs = [workloads.kv_cache_device(wl, device, seed=seed, segment=m) for m in range(wl.n_seg)]
         self.ref_k = [m[0] for m in segs]
         self.ref_v = [m[1] for m in segs]
         L, H, hd = wl.kv
         self.out_k = torch.empty((1, L, H, n_t, hd), dtype=torch.bfloat16, device=device)
         self.out_v = torch.empty_like(self.out_k)
-        self.winner = -1
         self.load_winner = None  # e2e: brings the winner's K/V rows (or whole cache) in from host memory
         self.gather_src = None   # e2e (inplace): the stored caches in pinned host memory, read in place
 
+    @property
+    def winner(self) -> int:
+        """The retrieved candidate of the last step (read after the stream has synchronised)."""
+        return int(self.h_choice[0])
+
     def step(self, ev=None):
+        """One target prompt, enqueued back to back: the retrieval's choice stays on the device
+        and the selected match and the gather read it there (no host round trip)."""
         ss, wl = self.ss, self.wl
         if ev:
             ev[0].record()
@@ -491,32 +499,24 @@ class RetrieveProblem:
             ev[1].record()
         ss.semshare_retrieve(self.t_rcodes, self.pool_rcodes, self.offsets, workspace=self.ret_ws,
                              err_flag=self.flag, out=self.ret)
-        self.h_choice.copy_(self.choice, non_blocking=True)  # best, applies
         if ev:
             ev[2].record()
         ss.semshare_hash(self.emb, self.table, self.hyp, self.pos, codes=self.codes, err_flag=self.flag,
                          workspace=self.hash_ws)
         if ev:
             ev[3].record()
-            ev[3].synchronize()
-        else:
-            import torch
-
-            torch.cuda.current_stream().synchronize()
-        m = self.winner = int(self.h_choice[0])
-        if not 0 <= m < wl.n_seg:
-            raise RuntimeError(f"retrieval returned candidate {m}")
-        ss.semshare_match_tc(self.codes, self.pool_codes[self.offsets[m]:self.offsets[m + 1]], idx=self.idx,
-                             dist=self.dist, workspace=self.tc_ws, err_flag=self.flag)
+        ss.semshare_match_tc_selected(self.codes, self.pool_codes, self.offsets, self.ret.best, idx=self.idx,
+                                      dist=self.dist, workspace=self.tc_ws, err_flag=self.flag)
         if self.load_winner is not None:
-            self.load_winner(m)
+            self.load_winner()
         if ev:
             ev[4].record()
         src_k, src_v = (self.ref_k, self.ref_v) if self.gather_src is None else self.gather_src
-        ss.semshare_gather_kv([src_k[m]], [src_v[m]], self.idx.view(1, wl.n_tgt), out_k=self.out_k,
-                              out_v=self.out_v, err_flag=self.flag)
+        ss.semshare_gather_kv(src_k, src_v, self.idx.view(1, wl.n_tgt), out_k=self.out_k, out_v=self.out_v,
+                              err_flag=self.flag)
         if ev:
             ev[5].record()
+        self.h_choice.copy_(self.choice, non_blocking=True)  # best, applies
 
     def unique_rows(self) -> int:
         return int(np.unique(self.idx.cpu().numpy()).size)
@@ -529,12 +529,12 @@ class RetrieveProblem:
 
     def e2e_plan(self, mode: str = "fetch"):
         """(one, h2d, d2h, read): the target's embedding rows and positions copied in; the stored
-        prompts' K/V caches stay in pinned host memory and, once the winner is known, the gather's
-        rows reach it one of three ways (`mode`): fetch -- semshare_fetch_rows copies each row the
-        match selects from the winner's cache into HBM once; inplace -- the gather reads them across
-        the host link, repeats included; copy_all -- the winner's whole cache is copied in first
-        (Sec. 3.2 loads the retrieved prompt onto the GPU with its KV cache).  The winner and the
-        match result (idx, dist) are copied back."""
+        prompts' K/V caches stay in pinned host memory and the gather's rows reach it one of three
+        ways (`mode`): fetch -- semshare_fetch_rows copies each row the match selects (pool rows of
+        the winner, known only on the device) into HBM once; inplace -- the gather reads them across
+        the host link, repeats included; copy_all -- the host reads the winner and its whole cache is
+        copied in first (Sec. 3.2 loads the retrieved prompt onto the GPU with its KV cache).  The
+        winner and the match result (idx, dist) are copied back."""
         import torch
 
         h_emb = self.emb.cpu().pin_memory()
@@ -547,16 +547,21 @@ class RetrieveProblem:
         h2d = h_emb.numel() * h_emb.element_size() + h_pos.numel() * 4 + kv_bytes
         d2h = (h_idx.numel() + h_dist.numel()) * 4 + self.h_choice.numel() * 4
         ss = self.ss
-        fetch_ws = torch.empty(max(16, ss.semshare_fetch_workspace_size(self.wl.seg_len)), dtype=torch.uint8,
+        fetch_ws = torch.empty(max(16, ss.semshare_fetch_workspace_size(self.wl.n_ref)), dtype=torch.uint8,
                                device=self.dev)
+        h_best = torch.zeros(1, dtype=torch.int32).pin_memory()
 
-        def load(m):
+        def load():
             if mode == "copy_all":
+                # the copy engines need the winner's address: the host waits for the retrieval
+                h_best.copy_(self.ret.best)
+                m = int(h_best[0])
                 self.ref_k[m].copy_(h_k[m], non_blocking=True)
                 self.ref_v[m].copy_(h_v[m], non_blocking=True)
             else:
-                ss.semshare_fetch_rows(h_k[m], h_v[m], self.idx, dev_k=self.ref_k[m], dev_v=self.ref_v[m],
-                                       workspace=fetch_ws, err_flag=self.flag)
+                # pool rows: the rows of whichever candidate won, found on the device
+                ss.semshare_fetch_rows(h_k, h_v, self.idx, dev_k=self.ref_k, dev_v=self.ref_v, workspace=fetch_ws,
+                                       err_flag=self.flag)
 
         def one():
             self.emb.copy_(h_emb, non_blocking=True)

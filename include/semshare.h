@@ -238,6 +238,39 @@ semshare_status semshare_retrieve(const uint32_t* tgt_codes, int64_t n_tgt, cons
                                   size_t workspace_bytes, uint32_t* err_flag, void* stream);
 
 /*
+ * semshare_match_tc_selected -- token matching (Sec. 3.3) against the candidate that a device
+ * value names, with no host round trip.
+ *
+ * After retrieval (semshare_retrieve, Sec. 3.2) the target's tokens are matched against the
+ * chosen reference prompt.  This entry point reads the choice (`best`, e.g. semshare_retrieve's
+ * output) on the device, so retrieval, matching and the gather can be enqueued back to back (and
+ * captured in one CUDA graph) without the host learning the winner first.  For every target
+ * token t, with c = *best:
+ *     idx[t]  = cand_offsets[c] + the nearest row of candidate c (ties to the lowest row)
+ *     dist[t] = its Hamming distance
+ * -- semshare_match_tc against candidate c's rows, shifted to pool rows, so that
+ * semshare_gather_kv over the pool's segments (one per candidate) gathers the right rows.
+ *
+ *   tgt_codes, nbits  as for semshare_match_tc
+ *   pool_codes        device, [n_pool][nbits/32], every candidate's codes back to back
+ *   cand_offsets      HOST, as for semshare_retrieve (strictly increasing, from 0)
+ *   best              device int32: the candidate; outside [0, n_cand) sets SEMSHARE_FLAG_INDEX
+ *                     and every idx/dist to -1
+ *   idx, dist         device int32[n_tgt] (dist may be NULL)
+ *   workspace         device scratch of at least semshare_match_tc_selected_workspace_size(
+ *                     n_tgt, cand_offsets, n_cand, nbits) bytes, 256-byte aligned
+ *   err_flag          as for semshare_match_tc
+ * The search is sized for the longest candidate; a shorter one leaves its tail columns masked.
+ * Returns EINVAL / EUNSUPPORTED for bad arguments, ECUDA if a launch fails.
+ */
+size_t semshare_match_tc_selected_workspace_size(int64_t n_tgt, const int64_t* cand_offsets, int32_t n_cand,
+                                                 int32_t nbits);
+semshare_status semshare_match_tc_selected(const uint32_t* tgt_codes, int64_t n_tgt, const uint32_t* pool_codes,
+                                           const int64_t* cand_offsets, int32_t n_cand, const int32_t* best,
+                                           int32_t nbits, int32_t* idx, int32_t* dist, void* workspace,
+                                           size_t workspace_bytes, uint32_t* err_flag, void* stream);
+
+/*
  * semshare_match_static -- semshare_match without a caller-provided workspace.
  *
  * The paper has no counterpart: this entry point exists for callers that cannot allocate

@@ -42,6 +42,8 @@ from ._native import (  # noqa: F401
     semshare_match,
     semshare_match_static,
     semshare_match_tc,
+    semshare_match_tc_selected,
+    semshare_match_tc_selected_workspace_size,
     semshare_match_tc_workspace_size,
     semshare_match_workspace_size,
     semshare_retrieve,

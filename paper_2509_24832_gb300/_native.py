@@ -78,6 +78,10 @@ def load():
                                           P, ctypes.c_size_t, P, P]
         lib.semshare_retrieve.restype = ctypes.c_int
         lib.semshare_match_static.argtypes = [P, i64, P, i64, i32, P, P, P]
+        lib.semshare_match_tc_selected_workspace_size.argtypes = [i64, P, i32, i32]
+        lib.semshare_match_tc_selected_workspace_size.restype = ctypes.c_size_t
+        lib.semshare_match_tc_selected.argtypes = [P, i64, P, P, i32, P, i32, P, P, P, ctypes.c_size_t, P, P]
+        lib.semshare_match_tc_selected.restype = ctypes.c_int
         lib.semshare_match_static.restype = ctypes.c_int
         lib.semshare_gather_kv.argtypes = [P, P, P, i32, KVLayout, P, i64, i32, P, P, KVLayout, P, P]
         lib.semshare_gather_kv.restype = ctypes.c_int
@@ -351,6 +355,48 @@ def semshare_retrieve(tgt_codes: torch.Tensor, pool_codes: torch.Tensor, cand_of
     if out is not None:
         return out
     return Retrieval(mean[:n_cand], sim[:n_cand], best, applies, idx, dist)
+
+
+def semshare_match_tc_selected_workspace_size(n_tgt: int, cand_offsets, nbits: int) -> int:
+    offs = (ctypes.c_int64 * len(cand_offsets))(*[int(o) for o in cand_offsets])
+    return int(load().semshare_match_tc_selected_workspace_size(int(n_tgt), offs, len(cand_offsets) - 1, int(nbits)))
+
+
+def semshare_match_tc_selected(tgt_codes: torch.Tensor, pool_codes: torch.Tensor, cand_offsets, best: torch.Tensor,
+                               idx: torch.Tensor | None = None, dist: torch.Tensor | None = None,
+                               workspace: torch.Tensor | None = None, err_flag: torch.Tensor | None = None,
+                               nbits: int | None = None, stream=None):
+    """Token matching (Sec. 3.3) against candidate `best` (a device int32, e.g. the retrieval's
+    choice) of the pool delimited by cand_offsets, read on the device: no host round trip.
+    Returns (idx, dist) int32 [n_tgt] with idx in pool rows."""
+    for t, n in ((tgt_codes, "tgt_codes"), (pool_codes, "pool_codes"), (best, "best")):
+        _need_cuda(t, n)
+    if not tgt_codes.is_contiguous() or not pool_codes.is_contiguous():
+        raise ValueError("codes must be contiguous")
+    if best.dtype != torch.int32:
+        raise ValueError("best must be int32")
+    n_tgt, w = tgt_codes.shape
+    if pool_codes.shape[1] != w:
+        raise ValueError("code widths differ")
+    nbits = 32 * w if nbits is None else nbits
+    offs = (ctypes.c_int64 * len(cand_offsets))(*[int(o) for o in cand_offsets])
+    n_cand = len(cand_offsets) - 1
+    dev = tgt_codes.device
+    if idx is None:
+        idx = torch.empty(n_tgt, dtype=torch.int32, device=dev)
+    if dist is None:
+        dist = torch.empty(n_tgt, dtype=torch.int32, device=dev)
+    _need_cuda(idx, "idx")
+    _need_cuda(dist, "dist")
+    if workspace is None:
+        need = semshare_match_tc_selected_workspace_size(n_tgt, cand_offsets, nbits)
+        workspace = torch.empty(max(256, need), dtype=torch.uint8, device=dev)
+    st = load().semshare_match_tc_selected(_ptr(tgt_codes), n_tgt, _ptr(pool_codes), offs, n_cand, _ptr(best), nbits,
+                                           _ptr(idx), _ptr(dist), _ptr(workspace),
+                                           workspace.numel() * workspace.element_size(), _ptr(err_flag),
+                                           _stream(stream))
+    _check(st, "semshare_match_tc_selected")
+    return idx, dist
 
 
 def semshare_match_static(tgt_codes: torch.Tensor, ref_codes: torch.Tensor, idx: torch.Tensor | None = None,

@@ -59,6 +59,7 @@ struct SegTable {
 struct TcArgs {
     int64_t n_tgt;
     int64_t n_ref;
+    const int64_t* n_ref_dev;  // non-null: the columns actually searched, [0, *n_ref_dev) (<= n_ref)
     int64_t n_rb;
     int64_t total;  // target blocks x reference blocks
     int32_t nbits;
@@ -70,15 +71,44 @@ struct TcArgs {
     uint64_t wait_limit_ns;
 };
 
+// Offsets of the candidates of a pool, passed by value (semshare_match_tc_selected; kMax = 1
+// for the other searches, which do not read it).
+template <int kMax>
+struct CandTable {
+    int32_t n_cand;
+    int64_t off[kMax + 1];
+};
+constexpr int kSelMax = SEMSHARE_RETRIEVE_MAX_CANDIDATES;
+template <bool kSelect>
+using CandTableFor = CandTable<kSelect ? kSelMax : 1>;
+
 // e4m3 +1 is 0x38, -1 is 0xB8: byte = 0xB8 ^ (bit << 7).  Rows are padded with zero bytes to
-// kpad; the keys of the search are reset on the way.
+// kpad; the keys of the search are reset on the way.  kSelect: the reference rows are those of
+// candidate *best of the pool `ref` (offsets `cand`), read on the device; rows past its length
+// are zero, and sel[0] = its length, sel[1] = its first pool row (0 and -1 for an invalid
+// *best, which also raises SEMSHARE_FLAG_INDEX).
+template <bool kSelect>
 __global__ void expand_codes_kernel(const uint32_t* __restrict__ tgt, int64_t n_tgt, const uint32_t* __restrict__ ref,
                                     int64_t n_ref, int32_t nbits, int32_t kpad, uint8_t* __restrict__ tpm,
                                     uint8_t* __restrict__ rpm, unsigned long long* __restrict__ keys, int64_t n_keys,
-                                    unsigned int* __restrict__ counter) {
+                                    unsigned int* __restrict__ counter, const int32_t* __restrict__ best,
+                                    const __grid_constant__ CandTableFor<kSelect> cand, int64_t* __restrict__ sel,
+                                    uint32_t* err_flag) {
     pdl_prologue();
     const int W = nbits >> 5;
     const int per_row = kpad >> 4;  // 16-byte pieces per row
+    int64_t len = n_ref;
+    if (kSelect) {
+        const int32_t b = __ldg(best);
+        const bool ok = b >= 0 && b < cand.n_cand;
+        len = ok ? cand.off[b + 1] - cand.off[b] : 0;
+        ref += ok ? cand.off[b] * W : 0;
+        if (blockIdx.x == 0 && threadIdx.x == 0) {
+            sel[0] = len;
+            sel[1] = ok ? cand.off[b] : -1;
+            if (!ok && err_flag) atomicOr(err_flag, SEMSHARE_FLAG_INDEX);
+        }
+    }
     const int64_t total = (n_tgt + n_ref) * per_row;
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
     for (int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; e < total; e += stride) {
@@ -86,7 +116,7 @@ __global__ void expand_codes_kernel(const uint32_t* __restrict__ tgt, int64_t n_
         const int piece = static_cast<int>(e - row * per_row);
         const int b0 = piece * 16;
         uint4 out = make_uint4(0u, 0u, 0u, 0u);
-        if (b0 < nbits) {
+        if (b0 < nbits && (!kSelect || row < n_tgt + len)) {
             const uint32_t* src = row < n_tgt ? tgt + row * W : ref + (row - n_tgt) * W;
             const uint32_t bits = __ldg(src + (b0 >> 5)) >> (b0 & 31);
             uint32_t w[4];
@@ -106,14 +136,18 @@ __global__ void expand_codes_kernel(const uint32_t* __restrict__ tgt, int64_t n_
     if (counter != nullptr && blockIdx.x == 0 && threadIdx.x == 0) *counter = 0u;
 }
 
+// sel non-null: idx are pool rows, local + sel[1]; a target with no key (an invalid candidate)
+// gets idx = dist = -1.
 __global__ void tc_keys_split_kernel(const unsigned long long* __restrict__ keys, int64_t n, int32_t* __restrict__ idx,
-                                     int32_t* __restrict__ dist) {
+                                     int32_t* __restrict__ dist, const int64_t* __restrict__ sel) {
     pdl_prologue();
+    const int64_t base = sel ? sel[1] : 0;
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const unsigned long long k = keys[i];
-        idx[i] = static_cast<int32_t>(static_cast<uint32_t>(k));
-        if (dist) dist[i] = static_cast<int32_t>(static_cast<uint32_t>(k >> 32));
+        const bool none = k == kNoKey;
+        idx[i] = none ? -1 : static_cast<int32_t>(static_cast<uint32_t>(k) + base);
+        if (dist) dist[i] = none ? -1 : static_cast<int32_t>(static_cast<uint32_t>(k >> 32));
     }
 }
 
@@ -270,6 +304,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         int64_t cur_tb = -1, col0 = 0, next_b = 0;
         int32_t cs = 0;
         unsigned long long best = kNoKey;
+        const int64_t n_cols = a.n_ref_dev ? *a.n_ref_dev : a.n_ref;  // columns searched
         // fold the best key 256*dot - j (j = column within this warp's half of the tile) into `best`
         auto fold = [&](float bk) {
             if (bk > -1.0e38f) {
@@ -323,7 +358,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             tc_fence_after_sync();
-            const int64_t rem = a.n_ref - col0;
+            const int64_t rem = n_cols - col0;
             const int valid = rem < kTN ? static_cast<int>(rem) : kTN;
             const int hv = valid - half * kHalfCols;  // valid columns of this half (may be <= 0)
             const uint32_t taddr =
@@ -489,11 +524,14 @@ __global__ void retrieve_select_kernel(const unsigned long long* __restrict__ ke
     }
 }
 
-// Expand the codes and run the search; leaves keys[n_seg][n_tgt] in the workspace.
-template <int kMaxSeg>
+// Expand the codes and run the search; leaves keys[n_seg][n_tgt] in the workspace.  kSelect:
+// the reference rows are candidate *best of the pool (cand), n_ref its longest candidate, and
+// sel (two int64 in device memory) receives the candidate's length and first pool row.
+template <int kMaxSeg, bool kSelect = false>
 semshare_status launch_search(const uint32_t* tgt_codes, int64_t n_tgt, const uint32_t* ref_codes, int64_t n_ref,
                               int32_t nbits, const SegTable<kMaxSeg>& seg, const TcPlan& plan, void* workspace,
-                              uint32_t* err_flag, cudaStream_t s, int sms, int dev) {
+                              uint32_t* err_flag, cudaStream_t s, int sms, int dev, const int32_t* best = nullptr,
+                              const CandTableFor<kSelect>* cand = nullptr, int64_t* sel = nullptr) {
     int smem_optin = 0;
     if (cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
         return SEMSHARE_ECUDA;
@@ -514,6 +552,7 @@ semshare_status launch_search(const uint32_t* tgt_codes, int64_t n_tgt, const ui
     a.a_bytes = static_cast<uint32_t>(kTM * plan.kpad);
     a.b_bytes = static_cast<uint32_t>(kTN * plan.kpad);
     a.keys = keys;
+    a.n_ref_dev = kSelect ? sel : nullptr;
     a.err_flag = err_flag;
     a.wait_limit_ns = wait_limit_ns();
     const size_t smem = kFixedSmem + 2 * static_cast<size_t>(a.a_bytes) + 2 * static_cast<size_t>(a.b_bytes);
@@ -531,9 +570,10 @@ semshare_status launch_search(const uint32_t* tgt_codes, int64_t n_tgt, const ui
 
     const int64_t pieces = (n_tgt + n_ref) * (plan.kpad / 16);
     const int64_t eg = (pieces + 255) / 256;
-    if (launch_pdl(expand_codes_kernel, dim3(static_cast<unsigned>(eg < sms * 8 ? eg : sms * 8)), dim3(256), 0, s,
-                   tgt_codes, n_tgt, ref_codes, n_ref, nbits, plan.kpad, tpm, rpm, keys, n_tgt * seg.n_seg,
-                   counter) != cudaSuccess)
+    CandTableFor<kSelect> none{};
+    if (launch_pdl(expand_codes_kernel<kSelect>, dim3(static_cast<unsigned>(eg < sms * 8 ? eg : sms * 8)), dim3(256), 0,
+                   s, tgt_codes, n_tgt, ref_codes, n_ref, nbits, plan.kpad, tpm, rpm, keys, n_tgt * seg.n_seg, counter,
+                   best, cand ? *cand : none, sel, err_flag) != cudaSuccess)
         return SEMSHARE_ECUDA;
     const int64_t grid = a.total < sms ? a.total : sms;
     if (launch_pdl(hamming_tc_kernel<kMaxSeg>, dim3(static_cast<unsigned>(grid)), dim3(kThreads), smem, s, tm_t, tm_r, a,
@@ -582,7 +622,75 @@ extern "C" semshare_status semshare_match_tc(const uint32_t* tgt_codes, int64_t 
     if (st != SEMSHARE_OK) return st;
     const int small = static_cast<int>((n_tgt + 255) / 256 < sms * 4 ? (n_tgt + 255) / 256 : sms * 4);
     if (launch_pdl(tc_keys_split_kernel, dim3(small), dim3(256), 0, s, static_cast<const unsigned long long*>(workspace),
-                   n_tgt, idx, dist) != cudaSuccess)
+                   n_tgt, idx, dist, static_cast<const int64_t*>(nullptr)) != cudaSuccess)
+        return SEMSHARE_ECUDA;
+    return launch_status();
+}
+
+namespace {
+// Longest candidate of a pool, or -1 for bad offsets.
+int64_t longest_candidate(const int64_t* off, int32_t n_cand) {
+    if (off[0] != 0) return -1;
+    int64_t m = 0;
+    for (int32_t c = 0; c < n_cand; ++c) {
+        if (off[c + 1] <= off[c]) return -1;
+        m = off[c + 1] - off[c] > m ? off[c + 1] - off[c] : m;
+    }
+    return m;
+}
+}  // namespace
+
+extern "C" size_t semshare_match_tc_selected_workspace_size(int64_t n_tgt, const int64_t* cand_offsets, int32_t n_cand,
+                                                           int32_t nbits) {
+    using namespace semshare;
+    if (n_tgt <= 0 || !cand_offsets || n_cand < 1 || n_cand > SEMSHARE_RETRIEVE_MAX_CANDIDATES || nbits < 32 ||
+        nbits > 256 || nbits % 32 != 0)
+        return 0;
+    const int64_t len = longest_candidate(cand_offsets, n_cand);
+    if (len < 1) return 0;
+    TcPlan p;
+    plan_tc(n_tgt, len, nbits, 0, &p);
+    return p.total() + 256;  // + the chosen candidate's length and first row
+}
+
+extern "C" semshare_status semshare_match_tc_selected(const uint32_t* tgt_codes, int64_t n_tgt,
+                                                      const uint32_t* pool_codes, const int64_t* cand_offsets,
+                                                      int32_t n_cand, const int32_t* best, int32_t nbits,
+                                                      int32_t* idx, int32_t* dist, void* workspace,
+                                                      size_t workspace_bytes, uint32_t* err_flag, void* stream) {
+    using namespace semshare;
+    if (n_cand < 1 || !cand_offsets || n_tgt < 0) return SEMSHARE_EINVAL;
+    if (n_cand > SEMSHARE_RETRIEVE_MAX_CANDIDATES) return SEMSHARE_EUNSUPPORTED;
+    if (nbits < 32 || nbits > 256 || nbits % 32 != 0) return SEMSHARE_EUNSUPPORTED;
+    const int64_t len = longest_candidate(cand_offsets, n_cand);
+    if (len < 1) return SEMSHARE_EINVAL;
+    if (n_tgt >= (int64_t(1) << 31) || cand_offsets[n_cand] >= (int64_t(1) << 31)) return SEMSHARE_EUNSUPPORTED;
+    if (n_tgt == 0) return SEMSHARE_OK;
+    if (!tgt_codes || !pool_codes || !best || !idx || !workspace) return SEMSHARE_EINVAL;
+    if (!aligned(tgt_codes, 4) || !aligned(pool_codes, 4) || !aligned(best, 4) || !aligned(idx, 4) ||
+        !aligned(workspace, 256) || (dist && !aligned(dist, 4)) || (err_flag && !aligned(err_flag, 4)))
+        return SEMSHARE_EINVAL;
+    TcPlan plan;
+    plan_tc(n_tgt, len, nbits, 0, &plan);
+    if (workspace_bytes < plan.total() + 256) return SEMSHARE_EINVAL;
+
+    int sms = 0, dev = 0;
+    if (current_sm_count(&sms, &dev) != SEMSHARE_OK) return SEMSHARE_ECUDA;
+    cudaStream_t s = as_stream(stream);
+    SegTable<1> seg{};
+    seg.n_seg = 1;
+    seg.off[0] = 0;
+    seg.off[1] = len;
+    CandTableFor<true> cand{};
+    cand.n_cand = n_cand;
+    for (int32_t c = 0; c <= n_cand; ++c) cand.off[c] = cand_offsets[c];
+    auto* sel = reinterpret_cast<int64_t*>(static_cast<uint8_t*>(workspace) + plan.total());
+    const semshare_status st = launch_search<1, true>(tgt_codes, n_tgt, pool_codes, len, nbits, seg, plan, workspace,
+                                                      err_flag, s, sms, dev, best, &cand, sel);
+    if (st != SEMSHARE_OK) return st;
+    const int small = static_cast<int>((n_tgt + 255) / 256 < sms * 4 ? (n_tgt + 255) / 256 : sms * 4);
+    if (launch_pdl(tc_keys_split_kernel, dim3(small), dim3(256), 0, s, static_cast<const unsigned long long*>(workspace),
+                   n_tgt, idx, dist, static_cast<const int64_t*>(sel)) != cudaSuccess)
         return SEMSHARE_ECUDA;
     return launch_status();
 }

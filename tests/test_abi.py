@@ -137,6 +137,26 @@ def test_retrieve_argument_errors(lib):
     assert lib.semshare_retrieve_workspace_size(10, 5, 1, 64) > lib.semshare_match_tc_workspace_size(10, 5, 64)
 
 
+def test_match_selected_argument_errors(lib):
+    m = lib.semshare_match_tc_selected
+
+    def call(offs, n_tgt=10, nbits=64, best=FAKE, ws_bytes=1 << 30, n_cand=None):
+        o = (ctypes.c_int64 * len(offs))(*offs)
+        n_cand = len(offs) - 1 if n_cand is None else n_cand
+        return m(FAKE, n_tgt, FAKE, o, n_cand, best, nbits, FAKE, None, FAKE, ws_bytes, None, None)
+
+    assert call([0, 5, 5]) == 1                        # empty candidate
+    assert call([1, 5]) == 1                           # does not start at row 0
+    assert call(list(range(258))) == 2                 # 257 candidates
+    assert call([0, 5], nbits=40) == 2
+    assert call([0, 5], best=None) == 1
+    assert call([0, 5], ws_bytes=100) == 1
+    assert call([0, 5], n_tgt=0) == 0                  # nothing to match
+    o = (ctypes.c_int64 * 3)(0, 300, 400)
+    assert lib.semshare_match_tc_selected_workspace_size(10, o, 2, 64) == \
+        lib.semshare_match_tc_workspace_size(10, 300, 64) + 256     # sized for the longest candidate
+
+
 def test_gather_retained_argument_errors(lib):
     import paper_2509_24832_gb300 as ss
 
