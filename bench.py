@@ -165,10 +165,33 @@ def load_peaks():
 
 
 def popc_peak_wordops(sm_mhz: float, sms: int) -> float:
-    """Word-op ceiling of the xor/popc/add Hamming loop: 16 population counts per clock per SM
-    (the CUDA C++ Programming Guide's throughput table for compute capability 10.x); one
-    word-op needs one popc, the xor and add issue on other pipes."""
+    """Word-op ceiling of the xor/popc/add Hamming loop from the CUDA C++ Programming Guide's
+    throughput table (16 population counts per clock per SM for compute capability 10.x); one
+    word-op needs one popc, the xor and add issue on other pipes.  A cross-check for the measured
+    rate below."""
     return 16.0 * sms * sm_mhz * 1e6
+
+
+def measure_hamming_rate(device, iters: int = 1 << 14, reps: int = 5) -> float:
+    """Sustained xor/popc/add word-ops per second of this GPU (semshare_probe_hamming_rate:
+    independent chains in registers, every SM fully occupied), best of `reps` launches timed
+    with CUDA events after a warm-up launch."""
+    import torch
+
+    import paper_2509_24832_gb300 as ss
+
+    sink = torch.empty(ss.semshare_probe_hamming_threads(), dtype=torch.int32, device=device)
+    ops = ss.semshare_probe_hamming_rate(iters, sink)
+    torch.cuda.synchronize()
+    best = float("inf")
+    for _ in range(reps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        ss.semshare_probe_hamming_rate(iters, sink)
+        b.record()
+        b.synchronize()
+        best = min(best, a.elapsed_time(b) * 1e-3)
+    return ops / best
 
 
 def kernel_sha(name: str) -> str:
@@ -716,8 +739,13 @@ def run_gpu_arm(args, rank, world, local_rank):
     props = torch.cuda.get_device_properties(device)
     clocks = sampler.summary() if not args.no_clocks else None
     sm_mhz = (clocks or {}).get("sm_mhz") or 2070.0
-    popc_peak = popc_peak_wordops(sm_mhz, props.multi_processor_count)
+    popc_table = popc_peak_wordops(sm_mhz, props.multi_processor_count)
+    popc_peak = measure_hamming_rate(device) if args.matcher == "popc" else popc_table
     stages = stage_report(wl, W, stage_ms, peaks, popc_peak, args.matcher)
+    if args.matcher == "popc":
+        stages["match"]["popc_peak"] = {"measured_wordops_per_s": popc_peak, "table_wordops_per_s": popc_table,
+                                        "source": "semshare_probe_hamming_rate (measured); table: 16 popc/clk/SM "
+                                                  "at the sampled SM clock, cross-check"}
 
     dominant = max(stage_ms, key=stage_ms.get)
     roof, tr = roofline_for(dominant, stages, peaks, args.matcher, wl.name)

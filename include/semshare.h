@@ -9,7 +9,12 @@
  * reference K/V cache to the target's token order (Sec. 3.3, Sec. 3.3.2).  This library
  * exposes them as three calls, semshare_hash (steps 1-2), semshare_match (step 3) and
  * semshare_gather_kv (step 4), plus semshare_rope_table, which precomputes the per-pair
- * rotation frequencies that semshare_hash consumes.
+ * rotation frequencies that semshare_hash consumes.  Around them: semshare_match_tc (step 3 on
+ * the tensor cores), semshare_retrieve (which stored prompt to reuse, Sec. 3.2) and
+ * semshare_match_tc_selected (step 3 against the retrieved prompt, chosen on the device),
+ * semshare_fetch_rows (the selected rows of a host-resident cache, brought in once each),
+ * semshare_gather_kv_retained (step 4 for each layer's retained tokens, Sec. 3.3.4) and
+ * semshare_kv_deviation / semshare_select_hd (the high-deviation tokens, App. A.4).
  *
  * Conventions shared by every call:
  *   - Buffers are owned by the caller.  Pointers marked "device" point to memory of the

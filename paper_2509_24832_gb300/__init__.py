@@ -17,6 +17,7 @@ from ._native import (  # noqa: F401
     KVLayout,
     LIB_PATH,
     MATCH_STATIC_MAX_TARGETS,
+    PROBE_CHAINS,
     RETAIN_MAX_LAYERS,
     RETRIEVE_MAX_CANDIDATES,
     SIMILARITY_MAX_DIST,
@@ -46,6 +47,8 @@ from ._native import (  # noqa: F401
     semshare_match_tc_selected_workspace_size,
     semshare_match_tc_workspace_size,
     semshare_match_workspace_size,
+    semshare_probe_hamming_rate,
+    semshare_probe_hamming_threads,
     semshare_retrieve,
     semshare_retrieve_workspace_size,
     semshare_rope_table,

@@ -95,6 +95,10 @@ def load():
         lib.semshare_kv_deviation.restype = ctypes.c_int
         lib.semshare_select_hd.argtypes = [P, i32, i64, i64, P, P, P]
         lib.semshare_select_hd.restype = ctypes.c_int
+        lib.semshare_probe_hamming_threads.argtypes = []
+        lib.semshare_probe_hamming_threads.restype = i64
+        lib.semshare_probe_hamming_rate.argtypes = [i64, P, i64, P]
+        lib.semshare_probe_hamming_rate.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -671,3 +675,24 @@ def semshare_gather_kv_retained(ref_k, ref_v, idx: torch.Tensor, retained, ret_o
                                             _ptr(out_k), _ptr(out_v), dst, _ptr(err_flag), _stream(stream))
     _check(st, "semshare_gather_kv_retained")
     return out_k, out_v
+
+
+PROBE_CHAINS = 8  # SEMSHARE_PROBE_CHAINS: word operations per thread and iteration
+
+
+def semshare_probe_hamming_threads() -> int:
+    n = int(load().semshare_probe_hamming_threads())
+    if n < 0:
+        raise SemshareError(3, "semshare_probe_hamming_threads")
+    return n
+
+
+def semshare_probe_hamming_rate(iters: int, sink: torch.Tensor, stream=None) -> int:
+    """Enqueues one launch of the word-operation probe (measurement support: the xor/popc/add
+    rate that bounds semshare_match).  sink: device int32/uint32 tensor of at least
+    semshare_probe_hamming_threads() words.  Returns the word operations the launch performs;
+    time it with CUDA events on the stream."""
+    _need_cuda(sink, "sink")
+    st = load().semshare_probe_hamming_rate(int(iters), _ptr(sink), sink.numel(), _stream(stream))
+    _check(st, "semshare_probe_hamming_rate")
+    return semshare_probe_hamming_threads() * int(iters) * PROBE_CHAINS

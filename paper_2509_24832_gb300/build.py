@@ -16,7 +16,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "libsemshare.so")
-SOURCES = ["api.cu", "hash.cu", "match.cu", "match_tc.cu", "gather.cu", "deviation.cu", "fetch.cu"]
+SOURCES = ["api.cu", "hash.cu", "match.cu", "match_tc.cu", "gather.cu", "deviation.cu", "fetch.cu", "probe.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 # -warn-spills: a register spill in a file with tensor-memory loads is a build error (below).  Those
 # kernels hand tcgen05.ld destination registers to later code before the load's wait; a spill placed

@@ -205,6 +205,13 @@ def test_fetch_argument_errors(lib):
     assert f(pk, pk, pd, pd, offs, 1, lay, None, 0, None, 0, None, None) == 0               # empty
 
 
+def test_probe_argument_errors(lib):
+    p = lib.semshare_probe_hamming_rate
+    assert p(0, FAKE, 1 << 30, None) == 1               # no iterations
+    assert p((1 << 24) + 1, FAKE, 1 << 30, None) == 1   # too many
+    assert p(16, None, 1 << 30, None) == 1              # no sink
+
+
 def test_deviation_and_select_argument_errors(lib):
     import paper_2509_24832_gb300 as ss
 

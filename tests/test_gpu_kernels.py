@@ -376,3 +376,13 @@ def test_gather_from_pinned_host_cache(ss):
     torch.cuda.synchronize()
     assert hk.is_cuda and int(flag.item()) == 0
     assert torch.equal(hk.view(torch.int16), dk.view(torch.int16)) and torch.equal(hv.view(torch.int16), dv.view(torch.int16))
+
+
+@pytest.mark.gpu
+def test_hamming_rate_probe_runs_and_is_plausible():
+    """The word-operation probe (the xor/popc matcher's roofline denominator) runs on every SM and
+    reports a rate between 1 and 100 T word-ops/s (the Programming Guide's table gives ~5 T)."""
+    import bench
+
+    rate = bench.measure_hamming_rate(torch.device("cuda"), iters=1 << 12, reps=3)
+    assert 1e12 < rate < 1e14, rate
