@@ -79,6 +79,9 @@ def parse_args(argv=None):
     p.add_argument("--hd", action="store_true",
                    help="append the first layer's KV deviation against a (synthetic) recomputed first layer "
                         "and the HD-token selection (App. A.4, Insight 1) to the step")
+    p.add_argument("--graph", action="store_true",
+                   help="capture one step in a CUDA graph and replay it for the timed steps (the host "
+                        "enqueues one graph instead of the library calls)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-clocks", action="store_true")
     return p.parse_args(argv)
@@ -688,6 +691,24 @@ def run_gpu_arm(args, rank, world, local_rank):
         prob.step()
     torch.cuda.synchronize()
     ss.check_flag(prob.flag, "warm-up")
+    run_step = prob.step
+    if args.graph:
+        # every library call only enqueues kernels on the current stream: the step records into one
+        # graph (programmatic-dependency edges between the kernels)
+        graph = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream(device)
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            prob.step()
+        torch.cuda.current_stream().wait_stream(side)
+        torch.cuda.synchronize()
+        with torch.cuda.graph(graph, capture_error_mode="thread_local"):
+            prob.step()
+        for _ in range(3):
+            graph.replay()
+        torch.cuda.synchronize()
+        ss.check_flag(prob.flag, "graph warm-up")
+        run_step = graph.replay
 
     K = args.steps
     # timed steps: one event pair per step (events between kernels would keep a kernel from being
@@ -708,7 +729,7 @@ def run_gpu_arm(args, rank, world, local_rank):
         for k in range(K):
             flush.zero_()  # evict the previous step's lines from the 129 MB L2 (untimed gap)
             evs[k][0].record()
-            prob.step()
+            run_step()
             evs[k][1].record()
         torch.cuda.synchronize()
         t_wall = time.perf_counter() - t_wall0
@@ -774,7 +795,7 @@ def run_gpu_arm(args, rank, world, local_rank):
     config = {"workload": wl.name, "n_ref": wl.n_ref, "n_tgt": wl.n_tgt, "n_batch": wl.n_batch,
               "n_seg": wl.n_seg, "d": wl.d, "nbits": wl.nbits, "kv": list(wl.kv),
               "parallelism": f"replicas x{world}", "l2": "flushed before every step (512 MB write)",
-              "matcher": args.matcher}
+              "matcher": args.matcher, "launch": "CUDA graph replay" if args.graph else "eager library calls"}
     if args.rope != "interleaved":
         config["rope"] = "pairs (k, k + d/2)"
     if args.retain:
