@@ -24,10 +24,12 @@
 //   warp 1        TMEM allocator and MMA issuer: 4 x tcgen05.mma (M=128, N=nbits, K=16) per
 //                 stage into one of two fp32 TMEM accumulators
 //   warps 4-11    RoPE: rotate each staged pair in shared memory, round to bf16 in the operand
-//                 tile, hand the stage to the MMA warp; the next stage's rotation table entries
-//                 are fetched while the current one is processed.  A thread owns 4 pairs of 4
-//                 rows 32 apart: when their positions are 32 apart too, only the first row's
-//                 angles go through sincos and the others step by the 32-position rotation
+//                 tile, hand the stage to the MMA warp.  Two groups of four warps take alternate
+//                 stages (interleaved pairing), so two stages are rotated at once; a group's next
+//                 rotation table entries are fetched while the other group works.  A thread owns
+//                 2 chunks (8 pairs) of 4 rows 32 apart: when their positions are 32 apart too,
+//                 only the first row's angles go through sincos and the others step by the
+//                 32-position rotation.  (Rotate-half pairing: all eight warps on every stage.)
 //   warps 12-15   epilogue: tcgen05.ld of the accumulator (lane = row), sign bits packed into
 //                 32-bit words, or the partial-sum hand-off of a shared tile
 // Every pipeline wait is bounded; on timeout the CTA raises SEMSHARE_FLAG_TIMEOUT, lets its
@@ -57,6 +59,15 @@ constexpr int kRopeWarps = 8;
 // (row, 16-byte chunk) items of a stage per RoPE thread: rows rbase + 32*i, i < kRopeRows
 constexpr int kRopeRows = kBM * (kBK * 2 / 16) / (kRopeWarps * 32);
 static_assert(kRopeRows >= 1 && kRopeRows <= 4 && kRopeRows * kRopeWarps * 32 == kBM * (kBK * 2 / 16), "RoPE split");
+// Interleaved pairing: the RoPE warps form kRopeGroups groups that rotate alternate stages; a
+// thread of a group covers kRopeRows rows and kGroupChunks of the 8 chunks of each.
+// Two groups measured fastest on GB300 (5k hash 47.3 us; one group 49.6, four 55.4).
+constexpr int kRopeGroups = 2;
+constexpr int kGroupThreads = kRopeWarps * 32 / kRopeGroups;
+constexpr int kGroupChunks = kRopeGroups;
+constexpr int kChunkStride = 8 / kGroupChunks;
+constexpr int kRowsPerPhase = 8 / kChunkStride;  // rows in one 8-thread shared-memory phase
+static_assert(kGroupThreads == kChunkStride * 32 && kRopeRows == 4, "grouped RoPE split: 32 row groups x chunks");
 constexpr int kEpiWarp0 = kRopeWarp0 + kRopeWarps;  // a multiple of 4: epilogue warp w reads TMEM lanes 32*(w%4)
 constexpr int kEpiWarps = 4;
 constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
@@ -232,7 +243,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t S = static_cast<uint32_t>(a.stages);
     const uint32_t bars = sbase + S * a.stage_bytes;
     const uint32_t bar_full = bars;                  // [S] TMA landed (count 1 + tx bytes)
-    const uint32_t bar_ready = bars + 8u * S;        // [S] operand tile rotated (count kRopeWarps)
+    const uint32_t bar_ready = bars + 8u * S;        // [S] operand tile rotated (count: the warps of a stage)
     const uint32_t bar_empty = bars + 16u * S;       // [S] MMAs done with the stage (commit)
     const uint32_t bar_accfull = bars + 24u * S;     // [2] accumulator complete (commit)
     const uint32_t bar_accempty = bar_accfull + 16u; // [2] accumulator drained (count kEpiWarps)
@@ -254,7 +265,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (uint32_t s = 0; s < S; ++s) {
             mbar_init(bar_full + 8u * s, 1);
-            mbar_init(bar_ready + 8u * s, kRopeWarps);
+            mbar_init(bar_ready + 8u * s, kHalf ? kRopeWarps : kRopeWarps / kRopeGroups);
             mbar_init(bar_empty + 8u * s, 1);
         }
         for (uint32_t b = 0; b < 2; ++b) {
@@ -463,24 +474,36 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if (!kHalf && warp >= kRopeWarp0 && warp < kRopeWarp0 + kRopeWarps) {
         // ---------------- RoPE (Eq. 1) on the staged tile ----------------
+        // kRopeGroups groups take turns: group g rotates the stages q = g, g + G, ..., so G stages
+        // are in flight at once and one group's chain of waits and latencies overlaps the others'.
+        // A thread of a group owns kRopeRows rows 32 apart and kGroupChunks 16-byte chunks of them.
         const int rt = threadIdx.x - kRopeWarp0 * 32;
-        const int c = rt & 7;                          // 16-byte chunk of the 128-byte row: pairs 4c..4c+3
-        const int rg = (rt >> 3) & 31;
-        const int rbase = rg + 32 * kRopeRows * (rt >> 8);  // rows rbase + 32*i, i < kRopeRows (row & 7 == rg & 7)
-        const uint32_t swz = static_cast<uint32_t>(rg & 7);
-        const uint32_t chunk_off = (static_cast<uint32_t>(c) ^ swz) << 4;
-        uint32_t q = 0;
-        int tile = static_cast<int>(i0 / nkb), kb = static_cast<int>(i0 % nkb), cur_tile = -1;
+        const int g = rt / kGroupThreads;
+        const int gt = rt - g * kGroupThreads;
+        const int c0 = gt % kChunkStride;             // chunks c0 + kChunkStride*j: pairs 4c .. 4c+3
+        // rows rbase + 32*i, i < kRopeRows.  The 8 threads of one 16-byte shared-memory access phase
+        // take chunks c0 .. c0 + kChunkStride - 1 of kRowsPerPhase rows whose swizzle phases
+        // (row & 7) differ by multiples of kChunkStride, so together they touch all 32 banks
+        const int u = gt / kChunkStride;
+        const int lowr = u % kRowsPerPhase, hir = u / kRowsPerPhase;
+        const int rbase = (hir / kChunkStride) * 8 + (hir % kChunkStride) + lowr * kChunkStride;
+        const uint32_t swz = static_cast<uint32_t>(rbase & 7);
         const int half = nkb * (kBK / 2);  // d/2: start of the 32-position rotations in the table
         uint32_t m[kRopeRows];
         bool steps32 = false;
-        Pairs4 tn;
-        load_pairs4(a.rope_table, half, kb, c, tn);
-        for (int64_t it = i0; it < i1; ++it, ++q) {
+        int cur_tile = -1;
+        Pairs4 tn[kGroupChunks];
+        if (i0 + g < i1) {
+            const int kb = static_cast<int>((i0 + g) % nkb);
+#pragma unroll
+            for (int j = 0; j < kGroupChunks; ++j) load_pairs4(a.rope_table, half, kb, c0 + kChunkStride * j, tn[j]);
+        }
+        for (int64_t it = i0 + g; it < i1; it += kRopeGroups) {
+            const uint32_t q = static_cast<uint32_t>(it - i0);
+            const int tile = static_cast<int>(it / nkb);
             if (tile != cur_tile) {
                 cur_tile = tile;
-                const int64_t row0 = static_cast<int64_t>(tile) * kBM;
-                const int64_t r0 = row0 + rbase;
+                const int64_t r0 = static_cast<int64_t>(tile) * kBM + rbase;
                 m[0] = r0 < a.n ? (a.positions ? static_cast<uint32_t>(__ldg(a.positions + r0)) : static_cast<uint32_t>(r0))
                                 : 0u;
                 steps32 = true;
@@ -494,76 +517,84 @@ __global__ void __launch_bounds__(kThreads, 1)
                     steps32 = steps32 && m[i] == m[0] + 32u * i;
                 }
             }
-            const Pairs4 tc = tn;
-            const int kb_next = kb + 1 == nkb ? 0 : kb + 1;
-            if (it + 1 < i1) load_pairs4(a.rope_table, half, kb_next, c, tn);  // next stage's table entries
-
             const uint32_t s = q % S, ph = (q / S) & 1u;
             const bool got = mbar_wait_bounded(bar_full + 8u * s, ph, abort_flag, a.err_flag, SEMSHARE_FLAG_TIMEOUT,
                                                a.wait_limit_ns);
             if (!__all_sync(0xFFFFFFFFu, got)) break;
             uint8_t* const st = gbase + s * a.stage_bytes;
-            float x[kRopeRows][8];
-            if (a.is_f32) {
-                const uint32_t c0 = static_cast<uint32_t>((c & 3) * 2);
 #pragma unroll
-                for (int i = 0; i < kRopeRows; ++i) {
-                    const uint8_t* stg = st + kABytes + a.b_bytes + (c >> 2) * (kF32Bytes / 2) + (rbase + 32 * i) * 128;
-                    const float4 f0 = *reinterpret_cast<const float4*>(stg + ((c0 ^ swz) << 4));
-                    const float4 f1 = *reinterpret_cast<const float4*>(stg + (((c0 + 1u) ^ swz) << 4));
-                    x[i][0] = f0.x; x[i][1] = f0.y; x[i][2] = f0.z; x[i][3] = f0.w;
-                    x[i][4] = f1.x; x[i][5] = f1.y; x[i][6] = f1.z; x[i][7] = f1.w;
-                }
-            } else {
+            for (int j = 0; j < kGroupChunks; ++j) {
+                const int c = c0 + kChunkStride * j;
+                const uint32_t chunk_off = (static_cast<uint32_t>(c) ^ swz) << 4;
+                float x[kRopeRows][8];
+                if (a.is_f32) {
+                    const uint32_t cc = static_cast<uint32_t>((c & 3) * 2);
 #pragma unroll
-                for (int i = 0; i < kRopeRows; ++i) {
-                    const uint4 v = *reinterpret_cast<const uint4*>(st + (rbase + 32 * i) * 128 + chunk_off);
-                    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-                    for (int p = 0; p < 4; ++p) {
-                        x[i][2 * p] = __uint_as_float(w[p] << 16);
-                        x[i][2 * p + 1] = __uint_as_float(w[p] & 0xFFFF0000u);
+                    for (int i = 0; i < kRopeRows; ++i) {
+                        const uint8_t* stg =
+                            st + kABytes + a.b_bytes + (c >> 2) * (kF32Bytes / 2) + (rbase + 32 * i) * 128;
+                        const float4 f0 = *reinterpret_cast<const float4*>(stg + ((cc ^ swz) << 4));
+                        const float4 f1 = *reinterpret_cast<const float4*>(stg + (((cc + 1u) ^ swz) << 4));
+                        x[i][0] = f0.x; x[i][1] = f0.y; x[i][2] = f0.z; x[i][3] = f0.w;
+                        x[i][4] = f1.x; x[i][5] = f1.y; x[i][6] = f1.z; x[i][7] = f1.w;
                     }
-                }
-            }
-            uint32_t y[kRopeRows][4];
-            if (steps32) {
-                // row i+1 sits 32 positions after row i: turn the angle on by the 32-step rotation
-                float cs[4], sn[4];
+                } else {
 #pragma unroll
-                for (int p = 0; p < 4; ++p) rotation(m[0], tc.turns[p], cs[p], sn[p]);
+                    for (int i = 0; i < kRopeRows; ++i) {
+                        const uint4 v = *reinterpret_cast<const uint4*>(st + (rbase + 32 * i) * 128 + chunk_off);
+                        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-                for (int i = 0; i < kRopeRows; ++i)
-#pragma unroll
-                    for (int p = 0; p < 4; ++p) {
-                        y[i][p] = rotate_to_bf16(x[i][2 * p], x[i][2 * p + 1], cs[p], sn[p]);
-                        if (i < kRopeRows - 1) {
-                            const float c32 = __uint_as_float(static_cast<uint32_t>(tc.cis32[p]));
-                            const float s32 = __uint_as_float(static_cast<uint32_t>(tc.cis32[p] >> 32));
-                            const float nc = fmaf(cs[p], c32, -sn[p] * s32);
-                            sn[p] = fmaf(cs[p], s32, sn[p] * c32);
-                            cs[p] = nc;
+                        for (int p = 0; p < 4; ++p) {
+                            x[i][2 * p] = __uint_as_float(w[p] << 16);
+                            x[i][2 * p + 1] = __uint_as_float(w[p] & 0xFFFF0000u);
                         }
                     }
-            } else {
+                }
+                const Pairs4& tc = tn[j];
+                uint32_t y[kRopeRows][4];
+                if (steps32) {
+                    // row i+1 sits 32 positions after row i: turn the angle on by the 32-step rotation
+                    float cs[4], sn[4];
+#pragma unroll
+                    for (int p = 0; p < 4; ++p) rotation(m[0], tc.turns[p], cs[p], sn[p]);
+#pragma unroll
+                    for (int i = 0; i < kRopeRows; ++i)
+#pragma unroll
+                        for (int p = 0; p < 4; ++p) {
+                            y[i][p] = rotate_to_bf16(x[i][2 * p], x[i][2 * p + 1], cs[p], sn[p]);
+                            if (i < kRopeRows - 1) {
+                                const float c32 = __uint_as_float(static_cast<uint32_t>(tc.cis32[p]));
+                                const float s32 = __uint_as_float(static_cast<uint32_t>(tc.cis32[p] >> 32));
+                                const float nc = fmaf(cs[p], c32, -sn[p] * s32);
+                                sn[p] = fmaf(cs[p], s32, sn[p] * c32);
+                                cs[p] = nc;
+                            }
+                        }
+                } else {
+#pragma unroll
+                    for (int i = 0; i < kRopeRows; ++i)
+#pragma unroll
+                        for (int p = 0; p < 4; ++p) {
+                            float cs, sn;
+                            rotation(m[i], tc.turns[p], cs, sn);
+                            y[i][p] = rotate_to_bf16(x[i][2 * p], x[i][2 * p + 1], cs, sn);
+                        }
+                }
 #pragma unroll
                 for (int i = 0; i < kRopeRows; ++i)
-#pragma unroll
-                    for (int p = 0; p < 4; ++p) {
-                        float cs, sn;
-                        rotation(m[i], tc.turns[p], cs, sn);
-                        y[i][p] = rotate_to_bf16(x[i][2 * p], x[i][2 * p + 1], cs, sn);
-                    }
+                    *reinterpret_cast<uint4*>(st + (rbase + 32 * i) * 128 + chunk_off) =
+                        make_uint4(y[i][0], y[i][1], y[i][2], y[i][3]);
             }
-#pragma unroll
-            for (int i = 0; i < kRopeRows; ++i)
-                *reinterpret_cast<uint4*>(st + (rbase + 32 * i) * 128 + chunk_off) =
-                    make_uint4(y[i][0], y[i][1], y[i][2], y[i][3]);
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) mbar_arrive(bar_ready + 8u * s);
-            kb = kb_next;
-            if (kb == 0) ++tile;
+            // this group's next stage: its table entries load while the other groups work
+            if (it + kRopeGroups < i1) {
+                const int kb = static_cast<int>((it + kRopeGroups) % nkb);
+#pragma unroll
+                for (int j = 0; j < kGroupChunks; ++j)
+                    load_pairs4(a.rope_table, half, kb, c0 + kChunkStride * j, tn[j]);
+            }
         }
     } else if (warp >= kEpiWarp0) {
         // ---------------- epilogue: signs -> packed codes, or partial hand-off ----------------
