@@ -8,9 +8,9 @@
 // of the same layout; semshare_gather_kv then runs on the device copy.  The copy is bitwise.
 //
 // mark_rows_kernel: one byte per reference row, set where some target selects it (an index
-// outside the reference sets SEMSHARE_FLAG_INDEX).  fetch_rows_kernel: a CTA owns 64 reference
-// rows of one (layer, head) plane and moves the marked ones' K and V rows as 16-byte vectors,
-// all loads of a thread issued before its stores; unmarked rows are neither read nor written.
+// outside the reference sets SEMSHARE_FLAG_INDEX).  fetch_rows_kernel: for each 64 reference rows
+// of one (layer, head) plane, the marked rows' K and V move as 16-byte vectors, all loads of a
+// thread issued before its stores; unmarked rows are neither read nor written.
 #include "common.cuh"
 
 namespace semshare {
@@ -19,6 +19,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kRows = 64;  // reference rows per CTA
 constexpr int kMaxSeg = 64;
+constexpr int kCtasPerSm = 4;  // resident copy CTAs per SM: 4 x 16 KB of requests in flight per SM
 
 struct FetchArgs {
     const uint8_t* src_k[kMaxSeg];
@@ -57,51 +58,59 @@ __device__ __forceinline__ uint4 ld_nc(const void* p) {
     return v;
 }
 
-__global__ void __launch_bounds__(kThreads) fetch_rows_kernel(const __grid_constant__ FetchArgs a, int64_t n_rows) {
+// Work item w = (plane, row block): plane = w / rblocks is one (layer, head), row block w % rblocks
+// holds reference rows [64*rb, 64*rb + 64).  A persistent grid of a few CTAs per SM strides over
+// the items: enough requests stay in flight to fill the host link (or HBM), and the SMs keep
+// room for kernels of other streams (a gather of rows already fetched) to run alongside.
+__global__ void __launch_bounds__(kThreads) fetch_rows_kernel(const __grid_constant__ FetchArgs a, int64_t n_rows,
+                                                              int64_t rblocks, int64_t n_items) {
     pdl_prologue();
     __shared__ int64_t s_off[kRows];  // byte offset of the row inside its segment
     __shared__ int32_t s_seg[kRows];  // segment, -1 = not selected
-    const int64_t plane = blockIdx.y + static_cast<int64_t>(gridDim.y) * blockIdx.z;  // (l, h)
-    const int h = static_cast<int>(plane % a.n_heads);
-    const int l = static_cast<int>(plane / a.n_heads);
-    const int64_t r0 = static_cast<int64_t>(blockIdx.x) * kRows;
-    if (threadIdx.x < kRows) {
-        const int64_t r = r0 + threadIdx.x;
-        int32_t seg = -1;
-        int64_t off = 0;
-        if (r < n_rows && a.map[r]) {
-            seg = 0;
-            while (r >= a.seg_off[seg + 1]) ++seg;
-            off = l * a.s_layer + h * a.s_head + (r - a.seg_off[seg]) * a.s_token;
+    const int total = 2 * kRows * a.chunks;  // 2 * kRows rows (K then V) x chunks pieces
+    for (int64_t w = blockIdx.x; w < n_items; w += gridDim.x) {
+        const int64_t plane = w / rblocks;  // (l, h)
+        const int h = static_cast<int>(plane % a.n_heads);
+        const int l = static_cast<int>(plane / a.n_heads);
+        const int64_t r0 = (w - plane * rblocks) * kRows;
+        if (threadIdx.x < kRows) {
+            const int64_t r = r0 + threadIdx.x;
+            int32_t seg = -1;
+            int64_t off = 0;
+            if (r < n_rows && a.map[r]) {
+                seg = 0;
+                while (r >= a.seg_off[seg + 1]) ++seg;
+                off = l * a.s_layer + h * a.s_head + (r - a.seg_off[seg]) * a.s_token;
+            }
+            s_seg[threadIdx.x] = seg;
+            s_off[threadIdx.x] = off;
         }
-        s_seg[threadIdx.x] = seg;
-        s_off[threadIdx.x] = off;
-    }
-    __syncthreads();
-    // 2 * kRows rows (K then V) x chunks pieces, 4 pieces per thread in flight
-    const int total = 2 * kRows * a.chunks;
-    for (int e0 = threadIdx.x; e0 < total; e0 += 4 * kThreads) {
-        uint4 v[4];
-        uint8_t* dst[4];
+        __syncthreads();
+        // 4 pieces per thread in flight: all loads before the stores
+        for (int e0 = threadIdx.x; e0 < total; e0 += 4 * kThreads) {
+            uint4 v[4];
+            uint8_t* dst[4];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            dst[i] = nullptr;
-            const int e = e0 + i * kThreads;
-            if (e < total) {
-                const int row = e / a.chunks, c = e - row * a.chunks;
-                const int rr = row % kRows;
-                const int seg = s_seg[rr];
-                if (seg >= 0) {
-                    const bool is_v = row >= kRows;
-                    const int64_t o = s_off[rr] + c * 16;
-                    v[i] = ld_nc((is_v ? a.src_v[seg] : a.src_k[seg]) + o);
-                    dst[i] = (is_v ? a.dst_v[seg] : a.dst_k[seg]) + o;
+            for (int i = 0; i < 4; ++i) {
+                dst[i] = nullptr;
+                const int e = e0 + i * kThreads;
+                if (e < total) {
+                    const int row = e / a.chunks, c = e - row * a.chunks;
+                    const int rr = row % kRows;
+                    const int seg = s_seg[rr];
+                    if (seg >= 0) {
+                        const bool is_v = row >= kRows;
+                        const int64_t o = s_off[rr] + c * 16;
+                        v[i] = ld_nc((is_v ? a.src_v[seg] : a.src_k[seg]) + o);
+                        dst[i] = (is_v ? a.dst_v[seg] : a.dst_k[seg]) + o;
+                    }
                 }
             }
-        }
 #pragma unroll
-        for (int i = 0; i < 4; ++i)
-            if (dst[i]) *reinterpret_cast<uint4*>(dst[i]) = v[i];
+            for (int i = 0; i < 4; ++i)
+                if (dst[i]) *reinterpret_cast<uint4*>(dst[i]) = v[i];
+        }
+        __syncthreads();  // the next item rewrites the row table
     }
 }
 
@@ -173,10 +182,10 @@ extern "C" semshare_status semshare_fetch_rows(const void* const* ref_k, const v
     a.map = map;
     const int64_t planes = static_cast<int64_t>(layout.n_layers) * layout.n_heads;
     const int64_t rblocks = (n_rows + kRows - 1) / kRows;
-    int64_t gy = planes < 65535 ? planes : 65535;
-    while (planes % gy != 0) --gy;
-    if (planes / gy > 65535 || rblocks > 0x7FFFFFFF) return SEMSHARE_EUNSUPPORTED;
-    const dim3 grid(static_cast<unsigned>(rblocks), static_cast<unsigned>(gy), static_cast<unsigned>(planes / gy));
-    if (launch_pdl(fetch_rows_kernel, grid, dim3(kThreads), 0, s, a, n_rows) != cudaSuccess) return SEMSHARE_ECUDA;
+    const int64_t n_items = planes * rblocks;
+    const int64_t cap = static_cast<int64_t>(kCtasPerSm) * sms;
+    const unsigned grid = static_cast<unsigned>(n_items < cap ? n_items : cap);
+    if (launch_pdl(fetch_rows_kernel, dim3(grid), dim3(kThreads), 0, s, a, n_rows, rblocks, n_items) != cudaSuccess)
+        return SEMSHARE_ECUDA;
     return launch_status();
 }
