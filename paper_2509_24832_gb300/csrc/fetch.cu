@@ -30,6 +30,7 @@ struct FetchArgs {
     int32_t n_seg, n_layers, n_heads, chunks;  // chunks: 16-byte pieces per row
     int64_t s_layer, s_head, s_token;          // strides of every segment, bytes
     const uint8_t* map;                        // [n_rows] 1 = selected
+    const uint8_t* block_map;                  // [rblocks] 1 = some row of the block is selected
 };
 
 __global__ void clear_map_kernel(uint8_t* __restrict__ map, int64_t n) {
@@ -39,14 +40,19 @@ __global__ void clear_map_kernel(uint8_t* __restrict__ map, int64_t n) {
         map[i] = 0;
 }
 
+// map[r] = 1 for every selected row r, and block_map[r / kRows] = 1 for its block of rows.
 __global__ void mark_rows_kernel(const int32_t* __restrict__ idx, int64_t n, int64_t n_rows, uint8_t* __restrict__ map,
-                                 uint32_t* err_flag) {
+                                 uint8_t* __restrict__ block_map, uint32_t* err_flag) {
     pdl_prologue();
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const int32_t r = __ldg(idx + i);
-        if (r >= 0 && r < n_rows) map[r] = 1;
-        else if (err_flag) atomicOr(err_flag, SEMSHARE_FLAG_INDEX);
+        if (r >= 0 && r < n_rows) {
+            map[r] = 1;
+            block_map[r / kRows] = 1;
+        } else if (err_flag) {
+            atomicOr(err_flag, SEMSHARE_FLAG_INDEX);
+        }
     }
 }
 
@@ -70,9 +76,11 @@ __global__ void __launch_bounds__(kThreads) fetch_rows_kernel(const __grid_const
     const int total = 2 * kRows * a.chunks;  // 2 * kRows rows (K then V) x chunks pieces
     for (int64_t w = blockIdx.x; w < n_items; w += gridDim.x) {
         const int64_t plane = w / rblocks;  // (l, h)
+        const int64_t rb = w - plane * rblocks;
+        if (!a.block_map[rb]) continue;  // no selected row here (the same for the whole CTA)
         const int h = static_cast<int>(plane % a.n_heads);
         const int l = static_cast<int>(plane / a.n_heads);
-        const int64_t r0 = (w - plane * rblocks) * kRows;
+        const int64_t r0 = rb * kRows;
         if (threadIdx.x < kRows) {
             const int64_t r = r0 + threadIdx.x;
             int32_t seg = -1;
@@ -119,9 +127,15 @@ bool stride_ok(int64_t s, int64_t elem) { return s >= 0 && ((s * elem) % 16) == 
 }  // namespace
 }  // namespace semshare
 
+namespace {
+size_t round256(size_t x) { return ((x + 255) / 256) * 256; }
+}  // namespace
+
 extern "C" size_t semshare_fetch_workspace_size(int64_t n_rows) {
+    using namespace semshare;
     if (n_rows <= 0) return 0;
-    return ((static_cast<size_t>(n_rows) + 255) / 256) * 256;
+    const size_t rblocks = (static_cast<size_t>(n_rows) + kRows - 1) / kRows;
+    return round256(static_cast<size_t>(n_rows)) + round256(rblocks);
 }
 
 extern "C" semshare_status semshare_fetch_rows(const void* const* ref_k, const void* const* ref_v,
@@ -157,12 +171,17 @@ extern "C" semshare_status semshare_fetch_rows(const void* const* ref_k, const v
     int sms = 0;
     if (current_sm_count(&sms, nullptr) != SEMSHARE_OK) return SEMSHARE_ECUDA;
     cudaStream_t s = as_stream(stream);
+    // workspace: the row map, then (256-byte aligned) the row-block map; both cleared here
     auto* map = static_cast<uint8_t*>(workspace);
-    const int64_t gm = (n_rows + 255) / 256, gi = (n_idx + 255) / 256;
+    const int64_t rblocks = (n_rows + kRows - 1) / kRows;
+    const int64_t map_bytes = static_cast<int64_t>(round256(static_cast<size_t>(n_rows)));
+    uint8_t* block_map = map + map_bytes;
+    const int64_t clear_bytes = map_bytes + rblocks;
+    const int64_t gm = (clear_bytes + 255) / 256, gi = (n_idx + 255) / 256;
     if (launch_pdl(clear_map_kernel, dim3(static_cast<unsigned>(gm < sms * 8 ? gm : sms * 8)), dim3(256), 0, s, map,
-                   n_rows) != cudaSuccess ||
+                   clear_bytes) != cudaSuccess ||
         launch_pdl(mark_rows_kernel, dim3(static_cast<unsigned>(gi < sms * 8 ? gi : sms * 8)), dim3(256), 0, s, idx, n_idx,
-                   n_rows, map, err_flag) != cudaSuccess)
+                   n_rows, map, block_map, err_flag) != cudaSuccess)
         return SEMSHARE_ECUDA;
     FetchArgs a{};
     for (int i = 0; i < n_seg; ++i) {
@@ -180,8 +199,8 @@ extern "C" semshare_status semshare_fetch_rows(const void* const* ref_k, const v
     a.s_head = layout.stride_head * eb;
     a.s_token = layout.stride_token * eb;
     a.map = map;
+    a.block_map = block_map;
     const int64_t planes = static_cast<int64_t>(layout.n_layers) * layout.n_heads;
-    const int64_t rblocks = (n_rows + kRows - 1) / kRows;
     const int64_t n_items = planes * rblocks;
     const int64_t cap = static_cast<int64_t>(kCtasPerSm) * sms;
     const unsigned grid = static_cast<unsigned>(n_items < cap ? n_items : cap);
