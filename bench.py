@@ -503,13 +503,11 @@ class RetrieveProblem:
         self.offsets = [m * wl.seg_len for m in range(wl.n_seg + 1)]
         # store time: every stored prompt's codes, plain and rotary (its own positions)
         pool = dev_rows(emb[:n_pool])
-        self.pool_rcodes = ss.semshare_hash(pool, self.table, self.hyp,
-                                            torch.zeros(n_pool, dtype=torch.int32, device=device))
+        self.pool_rcodes = ss.semshare_hash(pool, None, self.hyp, None, rope_layout="none")
         self.pool_codes = ss.semshare_hash(pool, self.table, self.hyp, torch.from_numpy(pos[:n_pool]).to(device))
         del pool
         self.emb = dev_rows(emb[n_pool:])
         self.pos = torch.from_numpy(pos[n_pool:]).to(device)
-        self.zeros = torch.zeros(n_t, dtype=torch.int32, device=device)
         self.t_rcodes = torch.empty((n_t, w), dtype=torch.int32, device=device)
         self.codes = torch.empty((n_t, w), dtype=torch.int32, device=device)
         self.hash_ws = torch.zeros(max(256, ss.semshare_hash_workspace_size(n_t, wl.d, wl.nbits)), dtype=torch.uint8,
@@ -547,8 +545,8 @@ class RetrieveProblem:
         ss, wl = self.ss, self.wl
         if ev:
             ev[0].record()
-        ss.semshare_hash(self.emb, self.table, self.hyp, self.zeros, codes=self.t_rcodes, err_flag=self.flag,
-                         workspace=self.hash_ws)
+        ss.semshare_hash(self.emb, None, self.hyp, None, codes=self.t_rcodes, err_flag=self.flag,
+                         workspace=self.hash_ws, rope_layout="none")
         if ev:
             ev[1].record()
         ss.semshare_retrieve(self.t_rcodes, self.pool_rcodes, self.offsets, workspace=self.ret_ws,

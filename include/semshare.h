@@ -139,11 +139,17 @@ size_t semshare_hash_workspace_size(int64_t n, int32_t d, int32_t nbits);
  *             SEMSHARE_ROPE_HALF: pairs (k, k + d/2) ("rotate-half", the arrangement of many
  *             model implementations), each turned by the same angle m * theta_k and rounded to
  *             bf16 the same way.  The rotation table is the same for both.
+ *             SEMSHARE_ROPE_NONE: no rotation -- the rows are hashed as they are (rounded to bf16
+ *             when fp32), the codes of y = x; positions and rope_table are ignored and may be
+ *             NULL.  (Used for the retrieval codes of Sec. 3.2, which compare whole prompts; it
+ *             equals SEMSHARE_ROPE_INTERLEAVED with every position 0, at which RoPE is the
+ *             identity, and skips the rotation work.)
  * SEMSHARE_ROPE_HALF takes bf16 rows and d a multiple of 128 (else EUNSUPPORTED).  Every other
  * argument, and the result for SEMSHARE_ROPE_INTERLEAVED, as for semshare_hash.
  */
 #define SEMSHARE_ROPE_INTERLEAVED 0u
 #define SEMSHARE_ROPE_HALF 1u
+#define SEMSHARE_ROPE_NONE 2u
 semshare_status semshare_hash_ex(const void* emb, semshare_dtype dtype, int64_t n, int32_t d, int64_t row_stride,
                                  const int32_t* positions, const uint64_t* rope_table, const uint16_t* hyperplanes,
                                  int32_t nbits, uint32_t rope_layout, uint32_t* codes, float* proj_out,

@@ -20,7 +20,7 @@ OK, EINVAL, EUNSUPPORTED, ECUDA, EINDEX, ETIMEOUT, ETOOLARGE = range(7)
 MATCH_STATIC_MAX_TARGETS = 262144
 FLAG_INDEX, FLAG_TIMEOUT = 1, 2
 BF16, F32 = 0, 1
-ROPE_LAYOUTS = {"interleaved": 0, "half": 1}
+ROPE_LAYOUTS = {"interleaved": 0, "half": 1, "none": 2}
 
 _lock = threading.Lock()
 _lib = None
@@ -194,8 +194,9 @@ def semshare_hash(emb: torch.Tensor, rope_table: torch.Tensor, hyperplanes: torc
     """LSH codes of RoPE-encoded rows.  emb [n][d] bf16/fp32 (rows may be strided),
     hyperplanes [nbits][d] bf16, positions [n] int32 (None: 0..n-1).  workspace: a zero-filled
     uint8 device buffer (default: the per-device one of hash_workspace()).  rope_layout:
-    "interleaved" (pairs (2k, 2k+1), Eq. 1) or "half" (pairs (k, k + d/2); bf16 rows, d a
-    multiple of 128).  Returns codes [n][nbits/32] int32 (uint32 bit patterns)."""
+    "interleaved" (pairs (2k, 2k+1), Eq. 1), "half" (pairs (k, k + d/2); bf16 rows, d a
+    multiple of 128) or "none" (no rotation: rope_table and positions are ignored and may be
+    None).  Returns codes [n][nbits/32] int32 (uint32 bit patterns)."""
     _need_cuda(emb, "emb")
     _need_cuda(hyperplanes, "hyperplanes")
     if emb.dim() != 2 or emb.stride(1) != 1:
@@ -222,6 +223,8 @@ def semshare_hash(emb: torch.Tensor, rope_table: torch.Tensor, hyperplanes: torc
     ws_bytes = workspace.numel() * workspace.element_size()
     if rope_layout not in ROPE_LAYOUTS:
         raise ValueError(f"rope_layout must be one of {sorted(ROPE_LAYOUTS)}")
+    if rope_layout != "none":
+        _need_cuda(rope_table, "rope_table")
     st = load().semshare_hash_ex(_ptr(emb), dt, n, d, emb.stride(0), _ptr(positions), _ptr(rope_table),
                                  _ptr(hyperplanes), nbits, ROPE_LAYOUTS[rope_layout], _ptr(codes), _ptr(proj_out),
                                  _ptr(workspace), ws_bytes, _ptr(err_flag), _stream(stream))

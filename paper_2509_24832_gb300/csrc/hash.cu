@@ -85,6 +85,7 @@ struct HashArgs {
     int32_t n_tiles;
     int32_t is_f32;
     int32_t stages;
+    int32_t no_rope;  // SEMSHARE_ROPE_NONE: rows hashed as they are (interleaved kernel only)
     uint32_t stage_bytes;
     uint32_t b_bytes;
     uint32_t tx_bytes;
@@ -493,7 +494,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool steps32 = false;
         int cur_tile = -1;
         Pairs4 tn[kGroupChunks];
-        if (i0 + g < i1) {
+        if (i0 + g < i1 && !a.no_rope) {
             const int kb = static_cast<int>((i0 + g) % nkb);
 #pragma unroll
             for (int j = 0; j < kGroupChunks; ++j) load_pairs4(a.rope_table, half, kb, c0 + kChunkStride * j, tn[j]);
@@ -522,6 +523,38 @@ __global__ void __launch_bounds__(kThreads, 1)
                                                a.wait_limit_ns);
             if (!__all_sync(0xFFFFFFFFu, got)) break;
             uint8_t* const st = gbase + s * a.stage_bytes;
+            if (a.no_rope) {
+                // rows hashed as they are: bf16 rows already are the MMA operand; fp32 rows are only
+                // rounded to bf16 (the rotation at position 0, which is the identity)
+                if (a.is_f32) {
+#pragma unroll
+                    for (int j = 0; j < kGroupChunks; ++j) {
+                        const int c = c0 + kChunkStride * j;
+                        const uint32_t chunk_off = (static_cast<uint32_t>(c) ^ swz) << 4;
+                        const uint32_t cc = static_cast<uint32_t>((c & 3) * 2);
+#pragma unroll
+                        for (int i = 0; i < kRopeRows; ++i) {
+                            const uint8_t* stg =
+                                st + kABytes + a.b_bytes + (c >> 2) * (kF32Bytes / 2) + (rbase + 32 * i) * 128;
+                            const float4 f0 = *reinterpret_cast<const float4*>(stg + ((cc ^ swz) << 4));
+                            const float4 f1 = *reinterpret_cast<const float4*>(stg + (((cc + 1u) ^ swz) << 4));
+                            const float xs[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
+                            uint32_t y[4];
+#pragma unroll
+                            for (int p = 0; p < 4; ++p) {
+                                __nv_bfloat162 r = __floats2bfloat162_rn(xs[2 * p], xs[2 * p + 1]);
+                                y[p] = *reinterpret_cast<uint32_t*>(&r);
+                            }
+                            *reinterpret_cast<uint4*>(st + (rbase + 32 * i) * 128 + chunk_off) =
+                                make_uint4(y[0], y[1], y[2], y[3]);
+                        }
+                    }
+                    fence_proxy_async_smem();
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar_ready + 8u * s);
+                continue;
+            }
 #pragma unroll
             for (int j = 0; j < kGroupChunks; ++j) {
                 const int c = c0 + kChunkStride * j;
@@ -589,7 +622,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive(bar_ready + 8u * s);
             // this group's next stage: its table entries load while the other groups work
-            if (it + kRopeGroups < i1) {
+            if (it + kRopeGroups < i1 && !a.no_rope) {
                 const int kb = static_cast<int>((it + kRopeGroups) % nkb);
 #pragma unroll
                 for (int j = 0; j < kGroupChunks; ++j)
@@ -824,8 +857,11 @@ extern "C" semshare_status semshare_hash_ex(const void* emb, semshare_dtype dtyp
                                             size_t workspace_bytes, uint32_t* err_flag, void* stream) {
     using namespace semshare;
     if (dtype != SEMSHARE_BF16 && dtype != SEMSHARE_F32) return SEMSHARE_EINVAL;
-    if (rope_layout != SEMSHARE_ROPE_INTERLEAVED && rope_layout != SEMSHARE_ROPE_HALF) return SEMSHARE_EINVAL;
+    if (rope_layout != SEMSHARE_ROPE_INTERLEAVED && rope_layout != SEMSHARE_ROPE_HALF &&
+        rope_layout != SEMSHARE_ROPE_NONE)
+        return SEMSHARE_EINVAL;
     const bool half = rope_layout == SEMSHARE_ROPE_HALF;
+    const bool none = rope_layout == SEMSHARE_ROPE_NONE;
     if (half && (dtype != SEMSHARE_BF16 || d % (2 * kBK) != 0)) return SEMSHARE_EUNSUPPORTED;
     if (n < 0 || d <= 0 || (d & 1) || row_stride < d) return SEMSHARE_EINVAL;
     if (d % kBK != 0 || d > 65536) return SEMSHARE_EUNSUPPORTED;
@@ -834,8 +870,8 @@ extern "C" semshare_status semshare_hash_ex(const void* emb, semshare_dtype dtyp
     const int64_t esize = dtype == SEMSHARE_BF16 ? 2 : 4;
     if ((row_stride * esize) % 16 != 0) return SEMSHARE_EINVAL;
     if (n == 0) return SEMSHARE_OK;
-    if (!emb || !rope_table || !hyperplanes || !codes || !workspace) return SEMSHARE_EINVAL;
-    if (!aligned(emb, 16) || !aligned(rope_table, 16) || !aligned(hyperplanes, 16) || !aligned(codes, 16) ||
+    if (!emb || (!rope_table && !none) || !hyperplanes || !codes || !workspace) return SEMSHARE_EINVAL;
+    if (!aligned(emb, 16) || (!none && !aligned(rope_table, 16)) || !aligned(hyperplanes, 16) || !aligned(codes, 16) ||
         !aligned(workspace, 256))
         return SEMSHARE_EINVAL;
     if ((proj_out && !aligned(proj_out, 16)) || (positions && !aligned(positions, 4)) ||
@@ -871,8 +907,9 @@ extern "C" semshare_status semshare_hash_ex(const void* emb, semshare_dtype dtyp
     // the last segment's partial accumulator (128 x nbits fp32) is staged in the stage buffers
     if (static_cast<size_t>(stages) * a.stage_bytes < static_cast<size_t>(kBM) * nbits * 4) return SEMSHARE_EUNSUPPORTED;
     a.stages = stages;
-    a.positions = positions;
+    a.positions = none ? nullptr : positions;
     a.rope_table = rope_table;
+    a.no_rope = none ? 1 : 0;
     a.codes = codes;
     a.proj = proj_out;
     a.err_flag = err_flag;

@@ -32,8 +32,7 @@ ALL = {**workloads.WORKLOADS, **workloads.RETRIEVAL_WORKLOADS}
 def _retrieval(a, wl, e, pd, R, table, flag, dev):
     n_pool = wl.n_ref
     offs = [m * wl.seg_len for m in range(wl.n_seg + 1)]
-    zeros = torch.zeros(e.shape[0], dtype=torch.int32, device=dev)
-    plain = ss.semshare_hash(e, table, R, zeros, err_flag=flag)
+    plain = ss.semshare_hash(e, None, R, None, err_flag=flag, rope_layout="none")
     ws = torch.empty(ss.semshare_retrieve_workspace_size(wl.n_tgt, n_pool, wl.n_seg, wl.nbits), dtype=torch.uint8,
                      device=dev)
     reps = a.reps if a.kernel == "retrieve" else 1
@@ -44,7 +43,7 @@ def _retrieval(a, wl, e, pd, R, table, flag, dev):
         return
     m = int(res.best.item())
     codes = ss.semshare_hash(e, table, R, pd, err_flag=flag)
-    del plain, zeros
+    del plain
     tc, rc = codes[n_pool:], codes[offs[m]:offs[m + 1]]
     idx = torch.empty(wl.n_tgt, dtype=torch.int32, device=dev)
     dist = torch.empty_like(idx)

@@ -79,7 +79,14 @@ def test_hash_ex_argument_errors(lib):
     def hx(layout, dtype=0, d=128):
         return lib.semshare_hash_ex(FAKE, dtype, 10, d, d, None, FAKE, FAKE, 64, layout, FAKE, None, FAKE, 1 << 30,
                                     None, None)
-    assert hx(2) == 1                    # unknown pairing
+    assert hx(3) == 1                    # unknown pairing
+    # no rotation (2) needs no rotation table: the call gets past the table check and stops at the
+    # device query (no GPU: ECUDA) or at the empty workspace (EINVAL) -- nothing is launched;
+    # with a rotation a missing table is an argument error
+    nt = lib.semshare_hash_ex(FAKE, 0, 10, 128, 128, None, None, FAKE, 64, 2, FAKE, None, FAKE, 0, None, None)
+    assert nt in (1, 3)
+    assert lib.semshare_hash_ex(FAKE, 0, 10, 128, 128, None, None, FAKE, 64, 0, FAKE, None, FAKE, 1 << 30, None,
+                                None) == 1
     assert hx(1, dtype=1) == 2           # rotate-half takes bf16 rows
     assert hx(1, d=192) == 2             # and d a multiple of 128
     assert lib.semshare_hash_ex(None, 0, 0, 128, 128, None, None, None, 64, 1, None, None, None, 0, None,
