@@ -139,15 +139,16 @@ def work(wl: workloads.Workload) -> dict:
 
 
 def work_retrieve(wl: workloads.Workload) -> dict:
-    """Retrieval step: two hashes of the target rows (plain and rotary), the retrieval GEMM over
-    the whole pool, the match against one member, the gather of one member's rows."""
+    """Retrieval step: the target rows hashed twice in one launch (plain and rotary codes), the
+    retrieval GEMM over the whole pool, the match against one member, the gather of one member's
+    rows."""
     n_t = wl.n_tgt
     esz = 4 if wl.emb_dtype == "f32" else 2
     L, H, hd = wl.kv
     kpad = ((wl.nbits + 127) // 128) * 128
     return {
-        "hash_flops": 2.0 * n_t * wl.d * wl.nbits,
-        "hash_bytes": n_t * wl.d * esz + n_t * wl.nbits / 8 + n_t * 4 + wl.nbits * wl.d * 2,
+        "hash_flops": 2.0 * 2.0 * n_t * wl.d * wl.nbits,
+        "hash_bytes": n_t * wl.d * esz + 2 * n_t * wl.nbits / 8 + n_t * 4 + wl.nbits * wl.d * 2,
         "retrieve_flops": 2.0 * n_t * wl.n_ref * kpad,
         "match_wordops": float(n_t) * wl.seg_len * (wl.nbits // 32),
         "match_flops": 2.0 * n_t * wl.seg_len * kpad,
@@ -470,16 +471,16 @@ class RetrieveProblem:
     """Reference retrieval in front of the path (Sec. 3.2).  The stored prompts' codes -- plain
     for retrieval, rotary-encoded for matching -- are computed once when they are stored; a step
     handles one new target prompt:
-      hash_plain  codes of the target rows without rotary encoding (retrieval precedes it)
+      hash        codes of the target rows without rotation (for retrieval, which precedes RoPE)
+                  and with it (Sec. 3.3.1), in one launch (semshare_hash_pair)
       retrieve    similarity to every stored prompt, the best one (semshare_retrieve)
-      hash        codes of the target rows with rotary encoding (Sec. 3.3.1)
       match       1-NN against the winner's rotary codes (the choice is read on the device)
       gather      the winner's K/V rows in the target's order (pool rows over every member)"""
 
-    STAGES = ("hash_plain", "retrieve", "hash", "match", "gather")
-    # hash 1, retrieve 3 (expand + key reset, search, per-candidate reduction), hash 1,
+    STAGES = ("hash", "retrieve", "match", "gather")
+    # hash pair 1, retrieve 3 (expand + key reset, search, per-candidate reduction),
     # selected match 3 (expand, search, split), gather 1
-    LAUNCHES_PER_STEP = 9
+    LAUNCHES_PER_STEP = 8
 
     def __init__(self, wl: workloads.Workload, device, seed: int, matcher: str = "tc"):
         import torch
@@ -510,8 +511,8 @@ class RetrieveProblem:
         self.pos = torch.from_numpy(pos[n_pool:]).to(device)
         self.t_rcodes = torch.empty((n_t, w), dtype=torch.int32, device=device)
         self.codes = torch.empty((n_t, w), dtype=torch.int32, device=device)
-        self.hash_ws = torch.zeros(max(256, ss.semshare_hash_workspace_size(n_t, wl.d, wl.nbits)), dtype=torch.uint8,
-                                   device=device)
+        self.hash_ws = torch.zeros(max(256, ss.semshare_hash_pair_workspace_size(n_t, wl.d, wl.nbits)),
+                                   dtype=torch.uint8, device=device)
         self.ret_ws = torch.empty(ss.semshare_retrieve_workspace_size(n_t, n_pool, wl.n_seg, wl.nbits),
                                   dtype=torch.uint8, device=device)
         self.choice = choice = torch.zeros(2, dtype=torch.int32, device=device)  # best, applies
@@ -545,18 +546,14 @@ class RetrieveProblem:
         ss, wl = self.ss, self.wl
         if ev:
             ev[0].record()
-        ss.semshare_hash(self.emb, None, self.hyp, None, codes=self.t_rcodes, err_flag=self.flag,
-                         workspace=self.hash_ws, rope_layout="none")
+        ss.semshare_hash_pair(self.emb, self.table, self.hyp, self.pos, codes_plain=self.t_rcodes,
+                              codes_rotary=self.codes, err_flag=self.flag, workspace=self.hash_ws)
         if ev:
             ev[1].record()
         ss.semshare_retrieve(self.t_rcodes, self.pool_rcodes, self.offsets, workspace=self.ret_ws,
                              err_flag=self.flag, out=self.ret)
         if ev:
             ev[2].record()
-        ss.semshare_hash(self.emb, self.table, self.hyp, self.pos, codes=self.codes, err_flag=self.flag,
-                         workspace=self.hash_ws)
-        if ev:
-            ev[3].record()
         ss.semshare_match_tc_selected(self.codes, self.pool_codes, self.offsets, self.ret.best, idx=self.idx,
                                       dist=self.dist, workspace=self.tc_ws, err_flag=self.flag)
         if self.fetch_gather is not None:
@@ -566,12 +563,12 @@ class RetrieveProblem:
             if self.load_winner is not None:
                 self.load_winner()
             if ev:
-                ev[4].record()
+                ev[3].record()
             src_k, src_v = (self.ref_k, self.ref_v) if self.gather_src is None else self.gather_src
             ss.semshare_gather_kv(src_k, src_v, self.idx.view(1, wl.n_tgt), out_k=self.out_k, out_v=self.out_v,
                                   err_flag=self.flag)
         if ev:
-            ev[5].record()
+            ev[4].record()
         self.h_choice.copy_(self.choice, non_blocking=True)  # best, applies
 
     def unique_rows(self) -> int:

@@ -154,6 +154,29 @@ semshare_status semshare_hash_ex(const void* emb, semshare_dtype dtype, int64_t 
                                  const int32_t* positions, const uint64_t* rope_table, const uint16_t* hyperplanes,
                                  int32_t nbits, uint32_t rope_layout, uint32_t* codes, float* proj_out,
                                  void* workspace, size_t workspace_bytes, uint32_t* err_flag, void* stream);
+/*
+ * semshare_hash_pair -- the codes of the same rows without and with rotation, in one launch.
+ *
+ * Reference retrieval (Sec. 3.2) compares prompts by the codes of their rows as they are; the
+ * token matching that follows (Sec. 3.3.1) uses the codes of the rows after RoPE.  For a target
+ * prompt both are needed; this call computes
+ *     codes_plain  = semshare_hash_ex(..., SEMSHARE_ROPE_NONE, ...)
+ *     codes_rotary = semshare_hash(..., positions, rope_table, ...)
+ * bit for bit, in one launch over twice the row tiles (one pipeline fill and one split of the
+ * work over the SMs instead of two).
+ *
+ *   emb, dtype, n (< 2^30), d, row_stride, positions, rope_table, hyperplanes, nbits, err_flag,
+ *   stream        as for semshare_hash
+ *   codes_plain, codes_rotary   device, [n][nbits/32] uint32 each, 16-byte aligned; written
+ *   workspace     as for semshare_hash, at least semshare_hash_pair_workspace_size(n, d, nbits)
+ *                 bytes (zero-filled before first use; left zero-filled by every call)
+ * No projections are written.  Returns as semshare_hash.
+ */
+size_t semshare_hash_pair_workspace_size(int64_t n, int32_t d, int32_t nbits);
+semshare_status semshare_hash_pair(const void* emb, semshare_dtype dtype, int64_t n, int32_t d, int64_t row_stride,
+                                   const int32_t* positions, const uint64_t* rope_table, const uint16_t* hyperplanes,
+                                   int32_t nbits, uint32_t* codes_plain, uint32_t* codes_rotary, void* workspace,
+                                   size_t workspace_bytes, uint32_t* err_flag, void* stream);
 semshare_status semshare_hash(const void* emb, semshare_dtype dtype, int64_t n, int32_t d, int64_t row_stride,
                               const int32_t* positions, const uint64_t* rope_table, const uint16_t* hyperplanes,
                               int32_t nbits, uint32_t* codes, float* proj_out, void* workspace,

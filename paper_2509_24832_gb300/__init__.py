@@ -38,6 +38,8 @@ from ._native import (  # noqa: F401
     semshare_gather_kv,
     semshare_gather_kv_retained,
     semshare_hash,
+    semshare_hash_pair,
+    semshare_hash_pair_workspace_size,
     semshare_hash_workspace_size,
     semshare_kv_deviation,
     semshare_match,

@@ -57,6 +57,10 @@ def load():
         lib.semshare_abi_version.restype = i32
         lib.semshare_rope_table.argtypes = [i32, ctypes.c_double, P, P]
         lib.semshare_rope_table.restype = ctypes.c_int
+        lib.semshare_hash_pair_workspace_size.argtypes = [i64, i32, i32]
+        lib.semshare_hash_pair_workspace_size.restype = ctypes.c_size_t
+        lib.semshare_hash_pair.argtypes = [P, ctypes.c_int, i64, i32, i64, P, P, P, i32, P, P, P, ctypes.c_size_t, P, P]
+        lib.semshare_hash_pair.restype = ctypes.c_int
         lib.semshare_hash_workspace_size.argtypes = [i64, i32, i32]
         lib.semshare_hash_workspace_size.restype = ctypes.c_size_t
         lib.semshare_hash.argtypes = [P, ctypes.c_int, i64, i32, i64, P, P, P, i32, P, P, P, ctypes.c_size_t, P, P]
@@ -230,6 +234,46 @@ def semshare_hash(emb: torch.Tensor, rope_table: torch.Tensor, hyperplanes: torc
                                  _ptr(workspace), ws_bytes, _ptr(err_flag), _stream(stream))
     _check(st, "semshare_hash")
     return codes
+
+
+def semshare_hash_pair_workspace_size(n: int, d: int, nbits: int) -> int:
+    return int(load().semshare_hash_pair_workspace_size(int(n), int(d), int(nbits)))
+
+
+def semshare_hash_pair(emb: torch.Tensor, rope_table: torch.Tensor, hyperplanes: torch.Tensor,
+                       positions: torch.Tensor | None = None, codes_plain: torch.Tensor | None = None,
+                       codes_rotary: torch.Tensor | None = None, err_flag: torch.Tensor | None = None,
+                       workspace: torch.Tensor | None = None, stream=None):
+    """The codes of the rows as they are and after RoPE (interleaved pairs), in one launch.
+    Arguments as for semshare_hash.  Returns (codes_plain, codes_rotary), each [n][nbits/32] int32."""
+    _need_cuda(emb, "emb")
+    _need_cuda(hyperplanes, "hyperplanes")
+    _need_cuda(rope_table, "rope_table")
+    if emb.dim() != 2 or emb.stride(1) != 1:
+        raise ValueError("emb must be [n][d] with unit stride along d")
+    dt = {torch.bfloat16: BF16, torch.float32: F32}.get(emb.dtype)
+    if dt is None:
+        raise ValueError("emb must be bfloat16 or float32")
+    if hyperplanes.dtype != torch.bfloat16 or not hyperplanes.is_contiguous():
+        raise ValueError("hyperplanes must be contiguous bfloat16 [nbits][d]")
+    n, d = emb.shape
+    nbits = hyperplanes.shape[0]
+    if hyperplanes.shape[1] != d:
+        raise ValueError("hyperplanes width differs from emb")
+    if positions is not None and (positions.dtype != torch.int32 or positions.numel() != n
+                                  or not positions.is_contiguous()):
+        raise ValueError("positions must be contiguous int32 [n]")
+    if codes_plain is None:
+        codes_plain = torch.empty((n, nbits // 32), dtype=torch.int32, device=emb.device)
+    if codes_rotary is None:
+        codes_rotary = torch.empty((n, nbits // 32), dtype=torch.int32, device=emb.device)
+    if workspace is None:
+        workspace = hash_workspace(2 * ((n + 127) // 128) * 128, d, nbits, emb.device)
+    st = load().semshare_hash_pair(_ptr(emb), dt, n, d, emb.stride(0), _ptr(positions), _ptr(rope_table),
+                                   _ptr(hyperplanes), nbits, _ptr(codes_plain), _ptr(codes_rotary), _ptr(workspace),
+                                   workspace.numel() * workspace.element_size(), _ptr(err_flag), _stream(stream))
+    _check(st, "semshare_hash_pair")
+    return codes_plain, codes_rotary
 
 
 def semshare_match_workspace_size(n_tgt: int) -> int:

@@ -85,7 +85,9 @@ struct HashArgs {
     int32_t n_tiles;
     int32_t is_f32;
     int32_t stages;
-    int32_t no_rope;  // SEMSHARE_ROPE_NONE: rows hashed as they are (interleaved kernel only)
+    int64_t pair_rows;  // semshare_hash_pair: n rounded up to a tile; logical tiles below it hash the rows
+                        // as they are into codes, those above it (the same rows again) rotated into codes2
+    uint32_t* codes2;
     uint32_t stage_bytes;
     uint32_t b_bytes;
     uint32_t tx_bytes;
@@ -109,6 +111,27 @@ __device__ __forceinline__ int64_t range_owner(int64_t i, int64_t total, int64_t
     while (b + 1 < G && range_begin(b + 1, total, G) <= i) ++b;
     while (b > 0 && range_begin(b, total, G) > i) --b;
     return b;
+}
+
+// Rotation variants of the kernel, fixed at compile time so that the plain rotary kernel carries
+// no test for the others: every row rotated; no row rotated (SEMSHARE_ROPE_NONE); a pair call,
+// which hashes every row twice -- logical tiles below pair_rows as they are, the tiles from
+// pair_rows on (the same rows again) rotated.
+enum RotVariant { kRotAll = 0, kRotNone = 1, kRotPair = 2 };
+
+// First source row of logical tile `tile`, whether its rows are rotated, and where its codes go.
+template <int kRot>
+__device__ __forceinline__ int64_t tile_src_row(const HashArgs& a, int64_t tile) {
+    const int64_t r = tile * kBM;
+    return (kRot == kRotPair && r >= a.pair_rows) ? r - a.pair_rows : r;
+}
+template <int kRot>
+__device__ __forceinline__ bool tile_rotates(const HashArgs& a, int64_t tile) {
+    return kRot == kRotAll || (kRot == kRotPair && tile * kBM >= a.pair_rows);
+}
+template <int kRot>
+__device__ __forceinline__ uint32_t* tile_codes(const HashArgs& a, int64_t tile) {
+    return (kRot == kRotPair && tile * kBM >= a.pair_rows) ? a.codes2 : a.codes;
 }
 
 // cos and sin of the rotation angle m * theta_k (Eq. 1).  turns_q64 = frac(theta_k/(2*pi)) as
@@ -232,7 +255,7 @@ __device__ __forceinline__ void store_codes(uint32_t* codes, int64_t row, int W,
     }
 }
 
-template <bool kHalf>
+template <bool kHalf, int kRot>
 __global__ void __launch_bounds__(kThreads, 1)
     lsh_hash_kernel(const __grid_constant__ CUtensorMap tmap_emb, const __grid_constant__ CUtensorMap tmap_hyp,
                     const HashArgs a) {
@@ -303,8 +326,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             int64_t pf_it = i0;
             auto prefetch_next = [&]() {
                 if (pf_it >= i1) return;
-                tma_prefetch_l2_2d(&tmap_emb, pf_kb * kBK, pf_tile * kBM);
-                if (a.is_f32) tma_prefetch_l2_2d(&tmap_emb, pf_kb * kBK + 32, pf_tile * kBM);
+                tma_prefetch_l2_2d(&tmap_emb, pf_kb * kBK, static_cast<int32_t>(tile_src_row<kRot>(a, pf_tile)));
+                if (a.is_f32) tma_prefetch_l2_2d(&tmap_emb, pf_kb * kBK + 32, static_cast<int32_t>(tile_src_row<kRot>(a, pf_tile)));
                 if (kHalf) tma_prefetch_l2_2d(&tmap_emb, partner_kb(pf_kb, nkb) * kBK, pf_tile * kBM);
                 ++pf_it;
                 if (++pf_kb == nkb) {
@@ -325,10 +348,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_arrive_expect_tx(full, a.tx_bytes);
                 if (a.is_f32) {
                     const uint32_t stg = st + kABytes + a.b_bytes;
-                    tma_load_2d(stg, &tmap_emb, full, kb * kBK, tile * kBM);
-                    tma_load_2d(stg + kF32Bytes / 2, &tmap_emb, full, kb * kBK + 32, tile * kBM);
+                    tma_load_2d(stg, &tmap_emb, full, kb * kBK, static_cast<int32_t>(tile_src_row<kRot>(a, tile)));
+                    tma_load_2d(stg + kF32Bytes / 2, &tmap_emb, full, kb * kBK + 32, static_cast<int32_t>(tile_src_row<kRot>(a, tile)));
                 } else {
-                    tma_load_2d(st, &tmap_emb, full, kb * kBK, tile * kBM);
+                    tma_load_2d(st, &tmap_emb, full, kb * kBK, static_cast<int32_t>(tile_src_row<kRot>(a, tile)));
                     if (kHalf) tma_load_2d(st + kABytes + a.b_bytes, &tmap_emb, full, partner_kb(kb, nkb) * kBK,
                                            tile * kBM);
                 }
@@ -491,10 +514,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t swz = static_cast<uint32_t>(rbase & 7);
         const int half = nkb * (kBK / 2);  // d/2: start of the 32-position rotations in the table
         uint32_t m[kRopeRows];
-        bool steps32 = false;
+        bool steps32 = false, rot = true;
         int cur_tile = -1;
         Pairs4 tn[kGroupChunks];
-        if (i0 + g < i1 && !a.no_rope) {
+        if (i0 + g < i1 && kRot != kRotNone) {
             const int kb = static_cast<int>((i0 + g) % nkb);
 #pragma unroll
             for (int j = 0; j < kGroupChunks; ++j) load_pairs4(a.rope_table, half, kb, c0 + kChunkStride * j, tn[j]);
@@ -504,7 +527,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int tile = static_cast<int>(it / nkb);
             if (tile != cur_tile) {
                 cur_tile = tile;
-                const int64_t r0 = static_cast<int64_t>(tile) * kBM + rbase;
+                rot = tile_rotates<kRot>(a, tile);
+                const int64_t r0 = tile_src_row<kRot>(a, tile) + rbase;
                 m[0] = r0 < a.n ? (a.positions ? static_cast<uint32_t>(__ldg(a.positions + r0)) : static_cast<uint32_t>(r0))
                                 : 0u;
                 steps32 = true;
@@ -523,7 +547,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                                a.wait_limit_ns);
             if (!__all_sync(0xFFFFFFFFu, got)) break;
             uint8_t* const st = gbase + s * a.stage_bytes;
-            if (a.no_rope) {
+            if (kRot != kRotAll && !rot) {
                 // rows hashed as they are: bf16 rows already are the MMA operand; fp32 rows are only
                 // rounded to bf16 (the rotation at position 0, which is the identity)
                 if (a.is_f32) {
@@ -622,7 +646,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive(bar_ready + 8u * s);
             // this group's next stage: its table entries load while the other groups work
-            if (it + kRopeGroups < i1 && !a.no_rope) {
+            if (it + kRopeGroups < i1 && kRot != kRotNone) {
                 const int kb = static_cast<int>((it + kRopeGroups) % nkb);
 #pragma unroll
                 for (int j = 0; j < kGroupChunks; ++j)
@@ -652,7 +676,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                                                SEMSHARE_FLAG_TIMEOUT, a.wait_limit_ns);
             if (!epilogue_all(got)) break;
             tc_fence_after_sync();
-            const int64_t row = static_cast<int64_t>(tile) * kBM + r;
+            const int64_t row = tile_src_row<kRot>(a, tile) + r;
+            uint32_t* const out_codes = tile_codes<kRot>(a, tile);
             const uint32_t taddr = tmem_base + (static_cast<uint32_t>(ew * 32) << 16) + buf * (a.tmem_cols >> 1);
             if (whole) {
                 uint32_t words[8];
@@ -669,7 +694,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_before_sync();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar_accempty + 8u * buf);
-                if (row < a.n) store_codes(a.codes, row, W, words);
+                if (row < a.n) store_codes(out_codes, row, W, words);
             } else {
                 // shared tile: this CTA's partial sum goes to its workspace slot.  The last segment's
                 // is staged in the idle pipeline buffers and published by the whole CTA at the end.
@@ -795,9 +820,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 uint32_t v[32];
 #pragma unroll
                 for (int j = 0; j < 32; ++j) v[j] = __float_as_uint(sum[j]);
-                const int64_t row = static_cast<int64_t>(tile) * kBM + rr;
+                const int64_t row = tile_src_row<kRot>(a, tile) + rr;
                 if (row < a.n) {
-                    a.codes[row * W + qq] = sign_word(v);
+                    tile_codes<kRot>(a, tile)[row * W + qq] = sign_word(v);
                     if (a.proj != nullptr) store_proj(a.proj, row, a.nbits, qq, v);
                 }
             }
@@ -850,12 +875,16 @@ extern "C" size_t semshare_hash_workspace_size(int64_t n, int32_t d, int32_t nbi
     return p.partial_bytes + p.count_bytes;
 }
 
-extern "C" semshare_status semshare_hash_ex(const void* emb, semshare_dtype dtype, int64_t n, int32_t d,
-                                            int64_t row_stride, const int32_t* positions, const uint64_t* rope_table,
-                                            const uint16_t* hyperplanes, int32_t nbits, uint32_t rope_layout,
-                                            uint32_t* codes, float* proj_out, void* workspace,
-                                            size_t workspace_bytes, uint32_t* err_flag, void* stream) {
-    using namespace semshare;
+namespace semshare {
+namespace {
+
+// semshare_hash_ex, and with codes2 non-null semshare_hash_pair (the rows as they are into codes,
+// rotated into codes2, in one launch over twice the tiles).
+semshare_status hash_impl(const void* emb, semshare_dtype dtype, int64_t n, int32_t d, int64_t row_stride,
+                          const int32_t* positions, const uint64_t* rope_table, const uint16_t* hyperplanes,
+                          int32_t nbits, uint32_t rope_layout, uint32_t* codes, uint32_t* codes2, float* proj_out,
+                          void* workspace, size_t workspace_bytes, uint32_t* err_flag, void* stream) {
+    const bool pair = codes2 != nullptr;
     if (dtype != SEMSHARE_BF16 && dtype != SEMSHARE_F32) return SEMSHARE_EINVAL;
     if (rope_layout != SEMSHARE_ROPE_INTERLEAVED && rope_layout != SEMSHARE_ROPE_HALF &&
         rope_layout != SEMSHARE_ROPE_NONE)
@@ -877,9 +906,11 @@ extern "C" semshare_status semshare_hash_ex(const void* emb, semshare_dtype dtyp
     if ((proj_out && !aligned(proj_out, 16)) || (positions && !aligned(positions, 4)) ||
         (err_flag && !aligned(err_flag, 4)))
         return SEMSHARE_EINVAL;
+    if (pair && (rope_layout != SEMSHARE_ROPE_INTERLEAVED || proj_out || !aligned(codes2, 16))) return SEMSHARE_EINVAL;
+    const int64_t n_pad = ((n + kBM - 1) / kBM) * kBM;
 
     HashPlan plan;
-    if (plan_hash(n, d, &plan) != SEMSHARE_OK) return SEMSHARE_ECUDA;
+    if (plan_hash(pair ? 2 * n_pad : n, d, &plan) != SEMSHARE_OK) return SEMSHARE_ECUDA;
     if (workspace_bytes < plan.partial_bytes + plan.count_bytes) return SEMSHARE_EINVAL;
     int dev = 0, smem_optin = 0;
     if (cudaGetDevice(&dev) != cudaSuccess ||
@@ -909,7 +940,8 @@ extern "C" semshare_status semshare_hash_ex(const void* emb, semshare_dtype dtyp
     a.stages = stages;
     a.positions = none ? nullptr : positions;
     a.rope_table = rope_table;
-    a.no_rope = none ? 1 : 0;
+    a.pair_rows = pair ? n_pad : 0;
+    a.codes2 = codes2;
     a.codes = codes;
     a.proj = proj_out;
     a.err_flag = err_flag;
@@ -927,12 +959,45 @@ extern "C" semshare_status semshare_hash_ex(const void* emb, semshare_dtype dtyp
                    static_cast<uint64_t>(nbits), static_cast<uint64_t>(d) * 2, 64u, static_cast<uint32_t>(nbits)))
         return SEMSHARE_ECUDA;
 
-    auto kernel = half ? lsh_hash_kernel<true> : lsh_hash_kernel<false>;
+    auto kernel = half   ? lsh_hash_kernel<true, kRotAll>
+                  : pair ? lsh_hash_kernel<false, kRotPair>
+                  : none ? lsh_hash_kernel<false, kRotNone>
+                         : lsh_hash_kernel<false, kRotAll>;
     if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) != cudaSuccess)
         return SEMSHARE_ECUDA;
     if (launch_pdl(kernel, dim3(plan.grid), dim3(kThreads), smem, as_stream(stream), tm_emb, tm_hyp, a) != cudaSuccess)
         return SEMSHARE_ECUDA;
     return launch_status();
+}
+
+}  // namespace
+}  // namespace semshare
+
+extern "C" semshare_status semshare_hash_ex(const void* emb, semshare_dtype dtype, int64_t n, int32_t d,
+                                            int64_t row_stride, const int32_t* positions, const uint64_t* rope_table,
+                                            const uint16_t* hyperplanes, int32_t nbits, uint32_t rope_layout,
+                                            uint32_t* codes, float* proj_out, void* workspace,
+                                            size_t workspace_bytes, uint32_t* err_flag, void* stream) {
+    return semshare::hash_impl(emb, dtype, n, d, row_stride, positions, rope_table, hyperplanes, nbits, rope_layout,
+                               codes, nullptr, proj_out, workspace, workspace_bytes, err_flag, stream);
+}
+
+extern "C" size_t semshare_hash_pair_workspace_size(int64_t n, int32_t d, int32_t nbits) {
+    if (n <= 0) return 0;
+    const int64_t n_pad = ((n + semshare::kBM - 1) / semshare::kBM) * semshare::kBM;
+    return semshare_hash_workspace_size(2 * n_pad, d, nbits);
+}
+
+extern "C" semshare_status semshare_hash_pair(const void* emb, semshare_dtype dtype, int64_t n, int32_t d,
+                                              int64_t row_stride, const int32_t* positions, const uint64_t* rope_table,
+                                              const uint16_t* hyperplanes, int32_t nbits, uint32_t* codes_plain,
+                                              uint32_t* codes_rotary, void* workspace, size_t workspace_bytes,
+                                              uint32_t* err_flag, void* stream) {
+    if (n > 0 && !codes_rotary) return SEMSHARE_EINVAL;
+    if (n >= (int64_t(1) << 30)) return SEMSHARE_EUNSUPPORTED;  // twice the rows stay below 2^31
+    return semshare::hash_impl(emb, dtype, n, d, row_stride, positions, rope_table, hyperplanes, nbits,
+                               SEMSHARE_ROPE_INTERLEAVED, codes_plain, n > 0 ? codes_rotary : nullptr, nullptr,
+                               workspace, workspace_bytes, err_flag, stream);
 }
 
 extern "C" semshare_status semshare_hash(const void* emb, semshare_dtype dtype, int64_t n, int32_t d,

@@ -93,6 +93,16 @@ def test_hash_ex_argument_errors(lib):
                                 None) == 0  # empty
 
 
+def test_hash_pair_argument_errors(lib):
+    hp = lib.semshare_hash_pair
+    assert hp(FAKE, 0, 10, 128, 128, None, FAKE, FAKE, 64, FAKE, None, FAKE, 1 << 30, None, None) == 1  # no 2nd output
+    assert hp(FAKE, 0, 1 << 30, 128, 128, None, FAKE, FAKE, 64, FAKE, FAKE, FAKE, 1 << 30, None, None) == 2  # too many
+    odd = ctypes.c_void_p((1 << 20) + 4)
+    assert hp(FAKE, 0, 10, 128, 128, None, FAKE, FAKE, 64, FAKE, odd, FAKE, 1 << 30, None, None) in (1, 3)
+    assert hp(None, 0, 0, 128, 128, None, None, None, 64, None, None, None, 0, None, None) == 0  # empty
+    assert lib.semshare_hash_pair_workspace_size(0, 128, 64) == 0
+
+
 def test_match_argument_errors(lib):
     m = lib.semshare_match
     assert m(FAKE, 10, FAKE, 0, 64, FAKE, None, FAKE, 80, None) == 1   # n_ref = 0
