@@ -55,7 +55,7 @@ NCU_TRAFFIC = {
     ("gather", "llama8b-5k"): {"file": "gather.cu", "sha": "05f4f810661f80c0", "bytes_per_launch": 1093.5e6},
     ("gather_retained", "llama8b-5k"): {"file": "gather.cu", "sha": "05f4f810661f80c0", "bytes_per_launch": 663.0e6},
     ("gather", "retrieve-16x4096"): {"file": "gather.cu", "sha": "05f4f810661f80c0", "bytes_per_launch": 1001.6e6},
-    ("hash", "llama8b-5k"): {"file": "hash.cu", "sha": "731e50da2e6842e4", "bytes_per_launch": 89.44e6},
+    ("hash", "llama8b-5k"): {"file": "hash.cu", "sha": "89eaa610817b640d", "bytes_per_launch": 89.34e6},
     ("match_tc", "llama8b-5k"): {"file": "match_tc.cu", "sha": "525d33ddbea4e539", "bytes_per_launch": 2.717e6},
     ("retrieve", "retrieve-16x4096"): {"file": "match_tc.cu", "sha": "525d33ddbea4e539", "bytes_per_launch": 18.41e6},
 }
