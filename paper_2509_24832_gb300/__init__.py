@@ -16,6 +16,7 @@ from ._native import (  # noqa: F401
     FLAG_TIMEOUT,
     KVLayout,
     LIB_PATH,
+    Prepared,
     MATCH_STATIC_MAX_TARGETS,
     PROBE_CHAINS,
     RETAIN_MAX_LAYERS,

@@ -43,6 +43,9 @@ class KVLayout(ctypes.Structure):
 def load():
     """Loads libsemshare.so (built in-tree by paper_2509_24832_gb300.build)."""
     global _lib
+    lib = _lib
+    if lib is not None:  # the common case, without the lock
+        return lib
     with _lock:
         if _lib is not None:
             return _lib
@@ -123,9 +126,33 @@ def _ptr(t: torch.Tensor | None):
     return None if t is None else ctypes.c_void_p(t.data_ptr())
 
 
+def _current_raw_stream() -> int:
+    """The current CUDA stream of the current device as a raw handle (what
+    torch.cuda.current_stream().cuda_stream returns, without building a Stream object)."""
+    return torch._C._cuda_getCurrentRawStream(torch._C._cuda_getDevice())
+
+
 def _stream(stream) -> ctypes.c_void_p:
-    s = torch.cuda.current_stream() if stream is None else stream
-    return ctypes.c_void_p(s.cuda_stream)
+    return ctypes.c_void_p(_current_raw_stream() if stream is None else stream.cuda_stream)
+
+
+class Prepared:
+    """A library call whose arguments were checked and marshalled once (`prepare=True` on
+    semshare_hash, semshare_match_tc, semshare_gather_kv).  Calling it enqueues the same work on
+    the current stream (or `stream`) and returns the call's outputs, for a few microseconds of
+    host time instead of the binding's checks.  It keeps its tensors alive; their storage must
+    not be resized or reallocated while it is used."""
+
+    __slots__ = ("_fn", "_args", "_where", "_keep", "result")
+
+    def __init__(self, fn, args, where, keep, result):
+        self._fn, self._args, self._where, self._keep, self.result = fn, args, where, keep, result
+
+    def __call__(self, stream=None):
+        st = self._fn(*self._args, _stream(stream))
+        if st != OK:
+            raise SemshareError(st, self._where)
+        return self.result
 
 
 def _need_cuda(t: torch.Tensor, name: str):
@@ -194,7 +221,8 @@ def hash_workspace(n: int, d: int, nbits: int, device=None) -> torch.Tensor:
 def semshare_hash(emb: torch.Tensor, rope_table: torch.Tensor, hyperplanes: torch.Tensor,
                   positions: torch.Tensor | None = None, codes: torch.Tensor | None = None,
                   proj_out: torch.Tensor | None = None, err_flag: torch.Tensor | None = None,
-                  workspace: torch.Tensor | None = None, stream=None, rope_layout: str = "interleaved") -> torch.Tensor:
+                  workspace: torch.Tensor | None = None, stream=None, rope_layout: str = "interleaved",
+                  *, prepare: bool = False):
     """LSH codes of RoPE-encoded rows.  emb [n][d] bf16/fp32 (rows may be strided),
     hyperplanes [nbits][d] bf16, positions [n] int32 (None: 0..n-1).  workspace: a zero-filled
     uint8 device buffer (default: the per-device one of hash_workspace()).  rope_layout:
@@ -229,11 +257,11 @@ def semshare_hash(emb: torch.Tensor, rope_table: torch.Tensor, hyperplanes: torc
         raise ValueError(f"rope_layout must be one of {sorted(ROPE_LAYOUTS)}")
     if rope_layout != "none":
         _need_cuda(rope_table, "rope_table")
-    st = load().semshare_hash_ex(_ptr(emb), dt, n, d, emb.stride(0), _ptr(positions), _ptr(rope_table),
-                                 _ptr(hyperplanes), nbits, ROPE_LAYOUTS[rope_layout], _ptr(codes), _ptr(proj_out),
-                                 _ptr(workspace), ws_bytes, _ptr(err_flag), _stream(stream))
-    _check(st, "semshare_hash")
-    return codes
+    args = (_ptr(emb), dt, n, d, emb.stride(0), _ptr(positions), _ptr(rope_table), _ptr(hyperplanes), nbits,
+            ROPE_LAYOUTS[rope_layout], _ptr(codes), _ptr(proj_out), _ptr(workspace), ws_bytes, _ptr(err_flag))
+    call = Prepared(load().semshare_hash_ex, args, "semshare_hash",
+                    (emb, positions, rope_table, hyperplanes, proj_out, workspace, err_flag), codes)
+    return call if prepare else call(stream)
 
 
 def semshare_hash_pair_workspace_size(n: int, d: int, nbits: int) -> int:
@@ -314,7 +342,8 @@ def semshare_match_tc_workspace_size(n_tgt: int, n_ref: int, nbits: int) -> int:
 
 def semshare_match_tc(tgt_codes: torch.Tensor, ref_codes: torch.Tensor, idx: torch.Tensor | None = None,
                       dist: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
-                      err_flag: torch.Tensor | None = None, nbits: int | None = None, stream=None):
+                      err_flag: torch.Tensor | None = None, nbits: int | None = None, stream=None, *,
+                      prepare: bool = False):
     """semshare_match computed on the tensor cores (same result).  Returns (idx, dist)."""
     _need_cuda(tgt_codes, "tgt_codes")
     _need_cuda(ref_codes, "ref_codes")
@@ -333,11 +362,11 @@ def semshare_match_tc(tgt_codes: torch.Tensor, ref_codes: torch.Tensor, idx: tor
     if workspace is None:
         workspace = torch.empty(max(256, semshare_match_tc_workspace_size(n_tgt, n_ref, nbits)), dtype=torch.uint8,
                                 device=dev)
-    st = load().semshare_match_tc(_ptr(tgt_codes), n_tgt, _ptr(ref_codes), n_ref, nbits, _ptr(idx), _ptr(dist),
-                                  _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(err_flag),
-                                  _stream(stream))
-    _check(st, "semshare_match_tc")
-    return idx, dist
+    args = (_ptr(tgt_codes), n_tgt, _ptr(ref_codes), n_ref, nbits, _ptr(idx), _ptr(dist), _ptr(workspace),
+            workspace.numel() * workspace.element_size(), _ptr(err_flag))
+    call = Prepared(load().semshare_match_tc, args, "semshare_match_tc", (tgt_codes, ref_codes, workspace, err_flag),
+                    (idx, dist))
+    return call if prepare else call(stream)
 
 
 RETRIEVE_MAX_CANDIDATES = 256
@@ -491,25 +520,34 @@ def kv_layout(t: torch.Tensor, batched: bool) -> KVLayout:
     return KVLayout(L, H, hd, t.element_size(), sb, sl, sh, st)
 
 
+def _segments(ref_k, ref_v):
+    """The K and V segments of a reference cache (a tensor or a list of tensors sharing one layout),
+    checked: CUDA or pinned host, [L][H][N][hd] with head_dim contiguous, one layout throughout.
+    Returns (seg_k, seg_v, layout of the first segment)."""
+    seg_k = ref_k if isinstance(ref_k, (list, tuple)) else (ref_k,)
+    seg_v = ref_v if isinstance(ref_v, (list, tuple)) else (ref_v,)
+    if len(seg_k) != len(seg_v) or not seg_k:
+        raise ValueError("ref_k and ref_v must have the same number of segments")
+    k0 = seg_k[0]
+    src = kv_layout(k0, batched=False)
+    key = (k0.stride()[:3], k0.shape[0], k0.shape[1], k0.shape[3], k0.element_size())
+    for t in (*seg_k, *seg_v):
+        _need_device_accessible(t, "ref")
+        if t.dim() != 4 or t.stride(3) != 1 or (t.stride()[:3], t.shape[0], t.shape[1], t.shape[3],
+                                                  t.element_size()) != key:
+            raise ValueError("all segments must share one layout")
+    return seg_k, seg_v, src
+
+
 def semshare_gather_kv(ref_k, ref_v, idx: torch.Tensor, out_k: torch.Tensor | None = None,
-                       out_v: torch.Tensor | None = None, err_flag: torch.Tensor | None = None, stream=None):
+                       out_v: torch.Tensor | None = None, err_flag: torch.Tensor | None = None, stream=None, *,
+                       prepare: bool = False):
     """Reordered K/V cache: out[b][l][h][t] = ref[l][h][idx[b][t]].
 
     ref_k/ref_v: a [L][H][N][hd] CUDA or pinned host tensor, or a list of them (a pool of reference prompts
     with identical strides; global row r = running offset of its segment + local row).
     idx: [n_batch][n_tgt] or [n_tgt] int32.  Returns (out_k, out_v), [n_batch][L][H][n_tgt][hd]."""
-    seg_k = list(ref_k) if isinstance(ref_k, (list, tuple)) else [ref_k]
-    seg_v = list(ref_v) if isinstance(ref_v, (list, tuple)) else [ref_v]
-    if len(seg_k) != len(seg_v) or not seg_k:
-        raise ValueError("ref_k and ref_v must have the same number of segments")
-    for t in seg_k + seg_v:
-        _need_device_accessible(t, "ref")
-    src = kv_layout(seg_k[0], batched=False)
-    for t in seg_k[1:] + seg_v:
-        o = kv_layout(t, batched=False)
-        if (o.stride_layer, o.stride_head, o.stride_token, o.head_dim, o.elem_bytes) != \
-                (src.stride_layer, src.stride_head, src.stride_token, src.head_dim, src.elem_bytes):
-            raise ValueError("all segments must share one layout")
+    seg_k, seg_v, src = _segments(ref_k, ref_v)
     _need_cuda(idx, "idx")
     idx2 = idx if idx.dim() == 2 else idx.view(1, -1)
     if idx2.dtype != torch.int32 or not idx2.is_contiguous():
@@ -523,21 +561,24 @@ def semshare_gather_kv(ref_k, ref_v, idx: torch.Tensor, out_k: torch.Tensor | No
     _need_cuda(out_k, "out_k")
     _need_cuda(out_v, "out_v")
     dst = kv_layout(out_k, batched=True)
-    dv = kv_layout(out_v, batched=True)
-    if (dst.stride_batch, dst.stride_layer, dst.stride_head, dst.stride_token) != \
-            (dv.stride_batch, dv.stride_layer, dv.stride_head, dv.stride_token):
+    if out_v.dim() != 5 or out_v.stride() != out_k.stride():
         raise ValueError("out_k and out_v must share one layout")
     n_seg = len(seg_k)
-    offs = [0]
-    for t in seg_k:
-        offs.append(offs[-1] + t.shape[2])
-    pk = (ctypes.c_void_p * n_seg)(*[t.data_ptr() for t in seg_k])
-    pv = (ctypes.c_void_p * n_seg)(*[t.data_ptr() for t in seg_v])
-    po = (ctypes.c_int64 * (n_seg + 1))(*offs)
-    st = load().semshare_gather_kv(pk, pv, po, n_seg, src, _ptr(idx2), n_tgt, n_batch, _ptr(out_k), _ptr(out_v), dst,
-                                   _ptr(err_flag), _stream(stream))
-    _check(st, "semshare_gather_kv")
-    return out_k, out_v
+    if n_seg == 1:
+        pk = (ctypes.c_void_p * 1)(seg_k[0].data_ptr())
+        pv = (ctypes.c_void_p * 1)(seg_v[0].data_ptr())
+        po = (ctypes.c_int64 * 2)(0, seg_k[0].shape[2])
+    else:
+        offs = [0]
+        for t in seg_k:
+            offs.append(offs[-1] + t.shape[2])
+        pk = (ctypes.c_void_p * n_seg)(*[t.data_ptr() for t in seg_k])
+        pv = (ctypes.c_void_p * n_seg)(*[t.data_ptr() for t in seg_v])
+        po = (ctypes.c_int64 * (n_seg + 1))(*offs)
+    args = (pk, pv, po, n_seg, src, _ptr(idx2), n_tgt, n_batch, _ptr(out_k), _ptr(out_v), dst, _ptr(err_flag))
+    call = Prepared(load().semshare_gather_kv, args, "semshare_gather_kv", (seg_k, seg_v, idx2, err_flag),
+                    (out_k, out_v))
+    return call if prepare else call(stream)
 
 
 def semshare_fetch_workspace_size(n_rows: int) -> int:
@@ -553,18 +594,8 @@ def semshare_fetch_rows(ref_k, ref_v, idx: torch.Tensor, dev_k=None, dev_v=None,
     sources are lists; semshare_gather_kv on them with the same idx gives the gather of the
     sources."""
     as_list = isinstance(ref_k, (list, tuple))
-    seg_k = list(ref_k) if as_list else [ref_k]
-    seg_v = list(ref_v) if isinstance(ref_v, (list, tuple)) else [ref_v]
-    if len(seg_k) != len(seg_v) or not seg_k:
-        raise ValueError("ref_k and ref_v must have the same number of segments")
-    for t in seg_k + seg_v:
-        _need_device_accessible(t, "ref")
-    lay = kv_layout(seg_k[0], batched=False)
-    for t in seg_k[1:] + seg_v:
-        o = kv_layout(t, batched=False)
-        if (o.stride_layer, o.stride_head, o.stride_token, o.head_dim, o.elem_bytes) != \
-                (lay.stride_layer, lay.stride_head, lay.stride_token, lay.head_dim, lay.elem_bytes):
-            raise ValueError("all segments must share one layout")
+    seg_k, seg_v, lay = _segments(ref_k, ref_v)
+    seg_k, seg_v = list(seg_k), list(seg_v)
     _need_cuda(idx, "idx")
     if idx.dtype != torch.int32 or not idx.is_contiguous():
         raise ValueError("idx must be contiguous int32")
@@ -680,18 +711,7 @@ def semshare_gather_kv_retained(ref_k, ref_v, idx: torch.Tensor, retained, ret_o
     ref_k/ref_v: a [L][H][N][hd] CUDA or pinned host tensor, or a list of them (as semshare_gather_kv).
     idx: int32 [n_tgt].  retained: int32 CUDA tensor, the layers' lists back to back;
     ret_offsets: host sequence of L + 1 ints.  Returns (out_k, out_v), [L][H][longest][hd]."""
-    seg_k = list(ref_k) if isinstance(ref_k, (list, tuple)) else [ref_k]
-    seg_v = list(ref_v) if isinstance(ref_v, (list, tuple)) else [ref_v]
-    if len(seg_k) != len(seg_v) or not seg_k:
-        raise ValueError("ref_k and ref_v must have the same number of segments")
-    for t in seg_k + seg_v:
-        _need_device_accessible(t, "ref")
-    src = kv_layout(seg_k[0], batched=False)
-    for t in seg_k[1:] + seg_v:
-        o = kv_layout(t, batched=False)
-        if (o.stride_layer, o.stride_head, o.stride_token, o.head_dim, o.elem_bytes) != \
-                (src.stride_layer, src.stride_head, src.stride_token, src.head_dim, src.elem_bytes):
-            raise ValueError("all segments must share one layout")
+    seg_k, seg_v, src = _segments(ref_k, ref_v)
     _need_cuda(idx, "idx")
     _need_cuda(retained, "retained")
     if idx.dtype != torch.int32 or not idx.is_contiguous() or retained.dtype != torch.int32 or \

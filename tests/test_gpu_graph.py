@@ -76,3 +76,51 @@ def test_retrieval_step_in_a_graph(ss):
     prob = bench.make_problem(wl, torch.device("cuda"), wl.base_seed, "tc")
     _capture_and_compare(ss, prob)
     assert prob.winner == workloads.retrieval_member(wl)
+
+
+def test_prepared_calls_match_the_plain_calls(ss):
+    """Prepared calls (arguments checked and marshalled once) give the plain calls' results, on
+    the current stream or a given one, for a fraction of the host time."""
+    import time
+
+    import bench
+
+    wl = workloads.WORKLOADS["llama8b-1k"]
+    prob = bench.make_problem(wl, torch.device("cuda"), wl.base_seed, "tc")
+    prob.step()
+    torch.cuda.synchronize()
+    want = _outputs(prob)
+    n_ref = wl.n_ref
+    calls = [
+        ss.semshare_hash(prob.emb, prob.table, prob.hyp, prob.pos, codes=prob.codes, err_flag=prob.flag,
+                         workspace=prob.hash_ws, prepare=True),
+        ss.semshare_match_tc(prob.codes[n_ref:], prob.codes[:n_ref], idx=prob.idx, dist=prob.dist,
+                             workspace=prob.tc_ws, err_flag=prob.flag, prepare=True),
+        ss.semshare_gather_kv(prob.ref_k, prob.ref_v, prob.idx.view(1, -1), out_k=prob.out_k, out_v=prob.out_v,
+                              err_flag=prob.flag, prepare=True),
+    ]
+    for stream in (None, torch.cuda.Stream()):
+        _scramble(prob)
+        torch.cuda.synchronize()
+        if stream is None:
+            for c in calls:
+                c()
+        else:
+            stream.wait_stream(torch.cuda.current_stream())
+            with torch.cuda.stream(stream):
+                for c in calls:
+                    c(stream)
+            torch.cuda.current_stream().wait_stream(stream)
+        torch.cuda.synchronize()
+        for a, b in zip(_outputs(prob), want):
+            assert torch.equal(a, b)
+    ss.check_flag(prob.flag, "prepared calls")
+    assert calls[1]()[0] is prob.idx  # the outputs are returned
+    # host time of a prepared call: enqueue-only, averaged
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(200):
+        calls[2]()
+    dt = (time.perf_counter() - t0) / 200
+    torch.cuda.synchronize()
+    assert dt < 1e-3
