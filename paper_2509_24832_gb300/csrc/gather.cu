@@ -116,10 +116,13 @@ __global__ void __launch_bounds__(kThreads)
     __shared__ int64_t s_src_off[kTokens];  // byte offset of the source row inside its segment
     __shared__ int32_t s_seg[kTokens];      // segment, -1 = skip (tail or bad index)
 
-    const int64_t plane = blockIdx.y + static_cast<int64_t>(gridDim.y) * blockIdx.z;  // (b, l, h)
-    const int h = static_cast<int>(plane % a.n_heads);
-    const int l = static_cast<int>((plane / a.n_heads) % a.n_layers);
-    const int64_t b = plane / (static_cast<int64_t>(a.n_heads) * a.n_layers);
+    // planes in (l, h, b) order, b fastest: the target prompts that read one reference plane
+    // (l, h) run back to back, so the plane's rows are still in L2 for all of them
+    const int64_t plane = blockIdx.y + static_cast<int64_t>(gridDim.y) * blockIdx.z;
+    const int64_t b = plane % a.n_batch;
+    const int64_t lh = plane / a.n_batch;
+    const int h = static_cast<int>(lh % a.n_heads);
+    const int l = static_cast<int>(lh / a.n_heads);
     const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kTokens;
     if (!resolve_rows<kRetain>(a, rt, l, h, b, t0, s_src_off, s_seg)) return;
 
@@ -156,10 +159,11 @@ __global__ void __launch_bounds__(kThreads)
     pdl_prologue();
     __shared__ int64_t s_src_off[kTokens];
     __shared__ int32_t s_seg[kTokens];
-    const int64_t plane = blockIdx.y + static_cast<int64_t>(gridDim.y) * blockIdx.z;
-    const int h = static_cast<int>(plane % a.n_heads);
-    const int l = static_cast<int>((plane / a.n_heads) % a.n_layers);
-    const int64_t b = plane / (static_cast<int64_t>(a.n_heads) * a.n_layers);
+    const int64_t plane = blockIdx.y + static_cast<int64_t>(gridDim.y) * blockIdx.z;  // (l, h, b), b fastest
+    const int64_t b = plane % a.n_batch;
+    const int64_t lh = plane / a.n_batch;
+    const int h = static_cast<int>(lh % a.n_heads);
+    const int l = static_cast<int>(lh / a.n_heads);
     const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kTokens;
     if (!resolve_rows<kRetain>(a, rt, l, h, b, t0, s_src_off, s_seg)) return;
     const int64_t dst_plane = b * a.d_batch + l * a.d_layer + h * a.d_head;
