@@ -55,8 +55,8 @@ NCU_TRAFFIC = {
     ("gather", "llama8b-5k"): {"file": "gather.cu", "sha": "5238bf70b2493478", "bytes_per_launch": 1093.8e6},
     ("gather_retained", "llama8b-5k"): {"file": "gather.cu", "sha": "5238bf70b2493478", "bytes_per_launch": 664.1e6},
     ("hash", "llama8b-5k"): {"file": "hash.cu", "sha": "89eaa610817b640d", "bytes_per_launch": 89.34e6},
-    ("match_tc", "llama8b-5k"): {"file": "match_tc.cu", "sha": "525d33ddbea4e539", "bytes_per_launch": 2.717e6},
-    ("retrieve", "retrieve-16x4096"): {"file": "match_tc.cu", "sha": "525d33ddbea4e539", "bytes_per_launch": 18.41e6},
+    ("match_tc", "llama8b-5k"): {"file": "match_tc.cu", "sha": "06cdd7c30d30cf11", "bytes_per_launch": 2.717e6},
+    ("retrieve", "retrieve-16x4096"): {"file": "match_tc.cu", "sha": "06cdd7c30d30cf11", "bytes_per_launch": 18.41e6},
 }
 
 

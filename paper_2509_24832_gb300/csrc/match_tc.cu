@@ -29,6 +29,11 @@
 // boundary takes the plain arg-max, one with a boundary is cut into runs and the key of the
 // finished candidate is flushed with the atomicMin.  A reduction over targets then gives each
 // candidate's summed nearest distance, its similarity (App. A.3) and the arg-max candidate.
+//
+// Selected mode (semshare_match_tc_selected).  The reference rows are one candidate of a pool,
+// chosen by a device value (the retrieval's `best`): the expand kernel reads the choice, expands
+// that candidate's rows and publishes its length and first pool row; the search, sized for the
+// longest candidate, masks the columns past that length; the split adds the first pool row.
 #include <cuda.h>
 
 #include "common.cuh"
