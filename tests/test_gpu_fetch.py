@@ -130,3 +130,28 @@ def test_fetch_full_size_pinned(ss):
     torch.cuda.synchronize()
     assert torch.equal(got_k.view(torch.int16), want_k.view(torch.int16))
     assert torch.equal(got_v.view(torch.int16), want_v.view(torch.int16))
+
+
+def test_fetch_with_64_segments_and_f32_rows(ss, oracle_mod):
+    """The most segments a pool may have (64, some empty), fp32 rows of 16 bytes (4 elements)."""
+    g = np.random.default_rng(31)
+    sizes = g.integers(0, 40, size=64)
+    L, H, hd = 2, 3, 4
+    cap = 48
+    ks = [torch.randn((L, H, cap, hd), device="cuda")[:, :, :n] for n in sizes]
+    vs = [torch.randn((L, H, cap, hd), device="cuda")[:, :, :n] for n in sizes]
+    n_rows = int(sizes.sum())
+    idx = g.integers(0, n_rows, size=700).astype(np.int32)
+    dk = [torch.full((L, H, cap, hd), -7.0, device="cuda")[:, :, :n] for n in sizes]
+    dv = [torch.full((L, H, cap, hd), -7.0, device="cuda")[:, :, :n] for n in sizes]
+    ss.semshare_fetch_rows(ks, vs, torch.from_numpy(idx).cuda(), dev_k=dk, dev_v=dv)
+    torch.cuda.synchronize()
+    hk = [k.cpu().contiguous().numpy() for k in ks]
+    hv = [v.cpu().contiguous().numpy() for v in vs]
+    ek = [np.full_like(a, -7.0) for a in hk]
+    ev = [np.full_like(a, -7.0) for a in hv]
+    ek, ev, bad = oracle_mod.fetch_rows(hk, hv, idx, ek, ev)
+    assert bad == 0
+    for s in range(64):
+        assert np.array_equal(dk[s].cpu().contiguous().numpy(), ek[s]), s
+        assert np.array_equal(dv[s].cpu().contiguous().numpy(), ev[s]), s

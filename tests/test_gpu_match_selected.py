@@ -111,3 +111,21 @@ def test_retrieve_then_match_then_gather_without_sync(ss, oracle_mod):
     assert np.array_equal(idx.cpu().numpy(), ei) and np.array_equal(dist.cpu().numpy(), ed)
     want_k = torch.stack([ks[5][:, :, int(r) - int(offs[5])] for r in ei], dim=2)
     assert torch.equal(out_k[0].view(torch.int16), want_k.view(torch.int16))
+
+
+def test_selected_with_the_maximum_of_256_candidates(ss, oracle_mod):
+    """256 one- to three-row candidates (the most a pool may have), each chosen in turn for a few."""
+    nbits = 32
+    g = np.random.default_rng(21)
+    sizes = g.integers(1, 4, size=256)
+    offs = np.concatenate([[0], np.cumsum(sizes)]).astype(np.int64)
+    pool = workloads.random_codes(int(offs[-1]), nbits, seed=22)
+    tgt = workloads.random_codes(129, nbits, seed=23)
+    t, p = _dev(tgt), _dev(pool)
+    best = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for c in (0, 1, 127, 200, 255):
+        best.fill_(c)
+        idx, dist = ss.semshare_match_tc_selected(t, p, offs, best, nbits=nbits)
+        torch.cuda.synchronize()
+        ei, ed = _expect(oracle_mod, tgt, pool, offs, c, nbits)
+        assert np.array_equal(idx.cpu().numpy(), ei) and np.array_equal(dist.cpu().numpy(), ed), c
