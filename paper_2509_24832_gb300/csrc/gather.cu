@@ -117,12 +117,14 @@ __global__ void __launch_bounds__(kThreads)
     __shared__ int32_t s_seg[kTokens];      // segment, -1 = skip (tail or bad index)
 
     // planes in (l, h, b) order, b fastest: the target prompts that read one reference plane
-    // (l, h) run back to back, so the plane's rows are still in L2 for all of them
+    // (l, h) run back to back, so the plane's rows are still in L2 for all of them.  Layers go
+    // last to first, so the first layer's rearranged rows -- which the KV deviation of App. A.4
+    // reads next -- are the most recently written, still in L2.
     const int64_t plane = blockIdx.y + static_cast<int64_t>(gridDim.y) * blockIdx.z;
     const int64_t b = plane % a.n_batch;
     const int64_t lh = plane / a.n_batch;
     const int h = static_cast<int>(lh % a.n_heads);
-    const int l = static_cast<int>(lh / a.n_heads);
+    const int l = a.n_layers - 1 - static_cast<int>(lh / a.n_heads);
     const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kTokens;
     if (!resolve_rows<kRetain>(a, rt, l, h, b, t0, s_src_off, s_seg)) return;
 
@@ -163,7 +165,7 @@ __global__ void __launch_bounds__(kThreads)
     const int64_t b = plane % a.n_batch;
     const int64_t lh = plane / a.n_batch;
     const int h = static_cast<int>(lh % a.n_heads);
-    const int l = static_cast<int>(lh / a.n_heads);
+    const int l = a.n_layers - 1 - static_cast<int>(lh / a.n_heads);  // last layer first
     const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kTokens;
     if (!resolve_rows<kRetain>(a, rt, l, h, b, t0, s_src_off, s_seg)) return;
     const int64_t dst_plane = b * a.d_batch + l * a.d_layer + h * a.d_head;
