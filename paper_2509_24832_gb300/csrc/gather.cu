@@ -9,9 +9,13 @@
 // Kernel design.  Pure streaming copy, bound by HBM bandwidth.  A CTA owns 64 target tokens
 // of one (b, l, h) plane and moves their 64 K rows and 64 V rows: it resolves the 64 indices
 // once (segment and local row, bounds-checked) into shared memory, then every thread issues
-// all of its 16-byte loads (read-only path, no L1 allocation) before any of its stores, so
-// each thread keeps 2*64*row_bytes/(16*256) requests in flight.  Consecutive threads touch
-// consecutive 16-byte chunks of a row and consecutive rows of the destination.
+// all of its 16-byte loads (read-only path) before any of its stores, so each thread keeps
+// 2*64*row_bytes/(16*256) requests in flight.  Consecutive threads touch consecutive 16-byte
+// chunks of a row and consecutive rows of the destination.  The loads are cached in L1: the
+// CTAs resident on one SM often read the same reference rows (a row several targets select;
+// with several target prompts, the same token block of each prompt, which similar prompts map
+// to nearby reference rows).  With several target prompts the stores are marked evict-first,
+// so the reference planes that every prompt re-reads stay in L2 while the output streams out.
 //
 // Retention (semshare_gather_kv_retained; Sec. 3.3.4, App. A: Retain[i] = T * prod alpha_retain,
 // evicted tokens dropped): each layer keeps only the target tokens of its list, and its cache
@@ -44,6 +48,7 @@ struct GatherArgs {
     int32_t n_layers;
     int32_t n_heads;
     int32_t n_batch;
+    int32_t stream_out;  // 1: evict-first stores (several target prompts share the reference)
     int64_t n_tgt;
     int64_t s_layer, s_head, s_token;           // source strides, bytes
     int64_t d_batch, d_layer, d_head, d_token;  // destination strides, bytes
@@ -53,24 +58,28 @@ struct GatherArgs {
     uint32_t* err_flag;
 };
 
-__device__ __forceinline__ uint4 load_stream(const void* p) {
+__device__ __forceinline__ uint4 load_row(const void* p) {
     uint4 v;
-    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                 : "l"(p));
+    asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
     return v;
 }
 
-__device__ __forceinline__ void store_vec(void* p, const uint4& v) {
-    asm volatile("st.global.v4.u32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
-                 : "memory");
+// stream = 1: evict-first (st.global.cs), the output is not re-read soon.  Uniform over the grid.
+__device__ __forceinline__ void store_vec(void* p, const uint4& v, int32_t stream) {
+    if (stream)
+        asm volatile("st.global.cs.v4.u32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                     : "memory");
+    else
+        asm volatile("st.global.v4.u32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                     : "memory");
 }
 
-// Resolves the CTA's kTokens rows (segment, source offset; -1 = skip) into shared memory.
-// Returns false when the CTA has nothing to move (past its layer's retained count).
+// Resolves the CTA's kTokens rows into their source row addresses in shared memory (K and V;
+// nullptr = skip: tail or bad index).  Returns false when the CTA has nothing to move (past its
+// layer's retained count).
 template <bool kRetain, typename RT>
 __device__ __forceinline__ bool resolve_rows(const GatherArgs& a, const RT& rt, int l, int h, int64_t b, int64_t t0,
-                                             int64_t* s_src_off, int32_t* s_seg) {
+                                             const uint8_t** s_src_k, const uint8_t** s_src_v) {
     int64_t count = a.n_tgt, base = 0;
     if (kRetain) {
         base = rt.off[l];
@@ -79,8 +88,8 @@ __device__ __forceinline__ bool resolve_rows(const GatherArgs& a, const RT& rt, 
     }
     if (threadIdx.x < kTokens) {
         const int64_t t = t0 + threadIdx.x;
-        int32_t seg = -1;
-        int64_t off = 0;
+        const uint8_t* pk = nullptr;
+        const uint8_t* pv = nullptr;
         if (t < count) {
             int64_t tok = t;
             bool ok = true;
@@ -90,31 +99,39 @@ __device__ __forceinline__ bool resolve_rows(const GatherArgs& a, const RT& rt, 
             }
             const int64_t r = ok ? __ldg(a.idx + b * a.n_tgt + tok) : -1;
             if (ok && r >= 0 && r < a.seg_off[a.n_seg]) {
-                seg = 0;
+                int seg = 0;
                 while (r >= a.seg_off[seg + 1]) ++seg;
-                off = l * a.s_layer + h * a.s_head + (r - a.seg_off[seg]) * a.s_token;
+                const int64_t off = l * a.s_layer + h * a.s_head + (r - a.seg_off[seg]) * a.s_token;
+                pk = a.src_k[seg] + off;
+                pv = a.src_v[seg] + off;
             } else if (a.err_flag) {
                 atomicOr(a.err_flag, SEMSHARE_FLAG_INDEX);
             }
         }
-        s_seg[threadIdx.x] = seg;
-        s_src_off[threadIdx.x] = off;
+        s_src_k[threadIdx.x] = pk;
+        s_src_v[threadIdx.x] = pv;
     }
     __syncthreads();
     return true;
 }
 
+// Rows of up to 16 chunks: at most 48 registers, so that 5 CTAs (1280 threads, 160 KB of loads in
+// flight) are resident per SM; measured on GB300 against 4 CTAs (58 registers): equal at one
+// prompt, 5% faster with 64 prompts sharing the reference; 6 CTAs spill.
+template <int C>
+constexpr int gather_min_ctas() { return C <= 16 ? 5 : 2; }
+
 // C = 16-byte chunks per row (row_bytes / 16).
 template <int C, bool kRetain, typename RT>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, gather_min_ctas<C>())
     kv_gather_kernel(const __grid_constant__ GatherArgs a, const __grid_constant__ RT rt) {
     pdl_prologue();
     constexpr int kRowsPerPass = kThreads / C;
     constexpr int kPasses = 2 * kTokens / kRowsPerPass;  // K rows then V rows
     static_assert(kThreads % C == 0 && (2 * kTokens) % kRowsPerPass == 0, "row split");
 
-    __shared__ int64_t s_src_off[kTokens];  // byte offset of the source row inside its segment
-    __shared__ int32_t s_seg[kTokens];      // segment, -1 = skip (tail or bad index)
+    __shared__ const uint8_t* s_src_k[kTokens];  // source rows, nullptr = skip (tail or bad index)
+    __shared__ const uint8_t* s_src_v[kTokens];
 
     // planes in (l, h, b) order, b fastest: the target prompts that read one reference plane
     // (l, h) run back to back, so the plane's rows are still in L2 for all of them.  Layers go
@@ -126,30 +143,23 @@ __global__ void __launch_bounds__(kThreads)
     const int h = static_cast<int>(lh % a.n_heads);
     const int l = a.n_layers - 1 - static_cast<int>(lh / a.n_heads);
     const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kTokens;
-    if (!resolve_rows<kRetain>(a, rt, l, h, b, t0, s_src_off, s_seg)) return;
+    if (!resolve_rows<kRetain>(a, rt, l, h, b, t0, s_src_k, s_src_v)) return;
 
     const int c = threadIdx.x % C;
     const int rr = threadIdx.x / C;
-    const int64_t dst_plane = b * a.d_batch + l * a.d_layer + h * a.d_head;
     uint4 v[kPasses];
 #pragma unroll
-    for (int p = 0; p < kPasses; ++p) {
-        const int row = rr + p * kRowsPerPass;  // 0..2*kTokens-1: K rows, then V rows
-        const int tt = row % kTokens;
-        const int seg = s_seg[tt];
-        if (seg >= 0) {
-            const uint8_t* base = (row < kTokens) ? a.src_k[seg] : a.src_v[seg];
-            v[p] = load_stream(base + s_src_off[tt] + c * 16);
-        }
+    for (int p = 0; p < kPasses; ++p) {  // passes below kPasses/2 move K rows, the rest V rows
+        const int tt = (rr + p * kRowsPerPass) % kTokens;
+        const uint8_t* src = p < kPasses / 2 ? s_src_k[tt] : s_src_v[tt];
+        if (src) v[p] = load_row(src + c * 16);
     }
+    uint8_t* const dst_k = a.dst_k + b * a.d_batch + l * a.d_layer + h * a.d_head + t0 * a.d_token + c * 16;
+    uint8_t* const dst_v = a.dst_v + (dst_k - a.dst_k);
 #pragma unroll
     for (int p = 0; p < kPasses; ++p) {
-        const int row = rr + p * kRowsPerPass;
-        const int tt = row % kTokens;
-        if (s_seg[tt] >= 0) {
-            uint8_t* base = (row < kTokens) ? a.dst_k : a.dst_v;
-            store_vec(base + dst_plane + (t0 + tt) * a.d_token + c * 16, v[p]);
-        }
+        const int tt = (rr + p * kRowsPerPass) % kTokens;
+        if (s_src_k[tt]) store_vec((p < kPasses / 2 ? dst_k : dst_v) + tt * a.d_token, v[p], a.stream_out);
     }
 }
 
@@ -159,25 +169,24 @@ template <bool kRetain, typename RT>
 __global__ void __launch_bounds__(kThreads)
     kv_gather_generic_kernel(const __grid_constant__ GatherArgs a, const __grid_constant__ RT rt, int chunks) {
     pdl_prologue();
-    __shared__ int64_t s_src_off[kTokens];
-    __shared__ int32_t s_seg[kTokens];
+    __shared__ const uint8_t* s_src_k[kTokens];
+    __shared__ const uint8_t* s_src_v[kTokens];
     const int64_t plane = blockIdx.y + static_cast<int64_t>(gridDim.y) * blockIdx.z;  // (l, h, b), b fastest
     const int64_t b = plane % a.n_batch;
     const int64_t lh = plane / a.n_batch;
     const int h = static_cast<int>(lh % a.n_heads);
     const int l = a.n_layers - 1 - static_cast<int>(lh / a.n_heads);  // last layer first
     const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kTokens;
-    if (!resolve_rows<kRetain>(a, rt, l, h, b, t0, s_src_off, s_seg)) return;
+    if (!resolve_rows<kRetain>(a, rt, l, h, b, t0, s_src_k, s_src_v)) return;
     const int64_t dst_plane = b * a.d_batch + l * a.d_layer + h * a.d_head;
     const int total = 2 * kTokens * chunks;
     for (int e = threadIdx.x; e < total; e += kThreads) {
         const int row = e / chunks, c = e - row * chunks;
         const int tt = row % kTokens;
-        const int seg = s_seg[tt];
-        if (seg < 0) continue;
-        const uint8_t* src = ((row < kTokens) ? a.src_k[seg] : a.src_v[seg]) + s_src_off[tt] + c * 16;
+        const uint8_t* src = row < kTokens ? s_src_k[tt] : s_src_v[tt];
+        if (!src) continue;
         uint8_t* dst = ((row < kTokens) ? a.dst_k : a.dst_v) + dst_plane + (t0 + tt) * a.d_token + c * 16;
-        store_vec(dst, load_stream(src));
+        store_vec(dst, load_row(src + c * 16), a.stream_out);
     }
 }
 
@@ -271,6 +280,7 @@ extern "C" semshare_status semshare_gather_kv(const void* const* ref_k, const vo
         (err_flag && !aligned(err_flag, 4)))
         return SEMSHARE_EINVAL;
     a.n_batch = n_batch;
+    a.stream_out = n_batch > 1 ? 1 : 0;
     a.n_tgt = n_tgt;
     a.idx = idx;
     NoRet none{};
