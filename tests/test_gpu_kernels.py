@@ -295,6 +295,25 @@ def test_gather_pool_batch_and_strided_output(ss, orc):
     assert int(big_k[:, :, :, :2].abs().sum()) == 0 and int(big_k[:, :, :, T + 2:].abs().sum()) == 0
 
 
+@pytest.mark.parametrize("hd,dtype", [(32, torch.bfloat16), (96, torch.bfloat16), (128, torch.bfloat16),
+                                      (256, torch.bfloat16), (128, torch.float32)])
+def test_gather_several_prompts_every_row_size(ss, orc, hd, dtype):
+    # several target prompts against one reference take the evict-first store path; row sizes of
+    # 4, 12 (generic kernel), 16 and 32 chunks
+    L, H, n_ref, B, T = 3, 2, 257, 4, 131
+    k = _rand_kv((L, H, n_ref, hd), dtype, 21)
+    v = _rand_kv((L, H, n_ref, hd), dtype, 22)
+    idx = torch.randint(0, n_ref, (B, T), dtype=torch.int32, device="cuda")
+    idx[1, :] = idx[0, :]  # two prompts selecting the same rows
+    ok, ov = ss.semshare_gather_kv(k, v, idx)
+    torch.cuda.synchronize()
+    ek, ev, bad = orc.gather_kv(_np_bits(k).reshape(L, H, n_ref, -1), _np_bits(v).reshape(L, H, n_ref, -1),
+                                idx.cpu().numpy())
+    assert bad == 0
+    assert np.array_equal(_np_bits(ok).reshape(ek.shape), ek)
+    assert np.array_equal(_np_bits(ov).reshape(ev.shape), ev)
+
+
 def test_gather_out_of_range_flags_and_skips(ss):
     k = _rand_kv((2, 2, 50, 64), seed=5)
     v = _rand_kv((2, 2, 50, 64), seed=6)
