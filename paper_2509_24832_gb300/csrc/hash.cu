@@ -934,6 +934,11 @@ semshare_status hash_impl(const void* emb, semshare_dtype dtype, int64_t n, int3
     const size_t fixed = kFixedSmem;
     int stages = static_cast<int>((static_cast<size_t>(smem_optin) - fixed) / a.stage_bytes);
     if (stages > 6) stages = 6;
+    // Interleaved pairing: RoPE group g rotates the stages q = g (mod kRopeGroups), which sit in
+    // slot q mod S.  With S a multiple of kRopeGroups every slot belongs to one group, so a group
+    // never waits on a slot whose previous stage it has not seen land; otherwise it could wait
+    // two phases ahead, where the full barrier's parity test cannot tell the phases apart.
+    if (!half) stages -= stages % kRopeGroups;
     if (stages < 2) return SEMSHARE_EUNSUPPORTED;
     // the last segment's partial accumulator (128 x nbits fp32) is staged in the stage buffers
     if (static_cast<size_t>(stages) * a.stage_bytes < static_cast<size_t>(kBM) * nbits * 4) return SEMSHARE_EUNSUPPORTED;
