@@ -86,6 +86,8 @@ def _hash_case(ss, orc, n, d, nbits, dtype, pos_kind, pad=0, seed=0):
         (1, 128, 160, "f32", "random", 0),
         (2000, 256, 224, "bf16", "large", 0),     # positions up to 2^31-1
         (385, 2048, 256, "f32", "large", 32),
+        (1536, 1024, 192, "bf16", "own", 0),     # 192-bit codes: the slot count rounded to the RoPE groups
+        (700, 512, 128, "f32", "random", 0),      # fp32 rows with 128-bit codes: two pipeline slots
     ],
 )
 def test_hash_parity(ss, orc, n, d, nbits, dtype, pos_kind, pad):
