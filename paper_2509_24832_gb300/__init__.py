@@ -52,6 +52,7 @@ from ._native import (  # noqa: F401
     semshare_match_workspace_size,
     semshare_probe_hamming_rate,
     semshare_probe_hamming_threads,
+    semshare_probe_operand_stream,
     semshare_retrieve,
     semshare_retrieve_workspace_size,
     semshare_rope_table,

@@ -106,6 +106,8 @@ def load():
         lib.semshare_probe_hamming_threads.restype = i64
         lib.semshare_probe_hamming_rate.argtypes = [i64, P, i64, P]
         lib.semshare_probe_hamming_rate.restype = ctypes.c_int
+        lib.semshare_probe_operand_stream.argtypes = [P, i64, i32, P, i32, i32, i32, P, P]
+        lib.semshare_probe_operand_stream.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -763,3 +765,26 @@ def semshare_probe_hamming_rate(iters: int, sink: torch.Tensor, stream=None) -> 
     st = load().semshare_probe_hamming_rate(int(iters), _ptr(sink), sink.numel(), _stream(stream))
     _check(st, "semshare_probe_hamming_rate")
     return semshare_probe_hamming_threads() * int(iters) * PROBE_CHAINS
+
+
+def semshare_probe_operand_stream(emb: torch.Tensor, hyperplanes: torch.Tensor | None = None, slots: int = 4,
+                                  prefetch: int = 0, err_flag: torch.Tensor | None = None, stream=None) -> None:
+    """Enqueues one launch that moves semshare_hash's operand blocks (the 128 x 64 embedding
+    block and, if given, the nbits x 64 hyperplane block of every (tile, K block) iteration)
+    through a ring of `slots` shared-memory slots with no rotation and no MMA (measurement
+    support: the floor the operand traffic sets for the hash kernel).  emb: contiguous bf16
+    [n][d] on the device, n a multiple of 128; hyperplanes: contiguous bf16 [nbits][d] or None.
+    Time the launch with CUDA events on the stream."""
+    _need_cuda(emb, "emb")
+    if emb.dtype != torch.bfloat16 or emb.dim() != 2 or not emb.is_contiguous():
+        raise SemshareError(EINVAL, "semshare_probe_operand_stream: emb must be a contiguous 2-D bf16 tensor")
+    nbits = 0
+    if hyperplanes is not None:
+        _need_cuda(hyperplanes, "hyperplanes")
+        if hyperplanes.dtype != torch.bfloat16 or hyperplanes.dim() != 2 or not hyperplanes.is_contiguous() \
+                or hyperplanes.shape[1] != emb.shape[1]:
+            raise SemshareError(EINVAL, "semshare_probe_operand_stream: hyperplanes must be contiguous bf16 [nbits][d]")
+        nbits = hyperplanes.shape[0]
+    st = load().semshare_probe_operand_stream(_ptr(emb), emb.shape[0], emb.shape[1], _ptr(hyperplanes), nbits,
+                                              int(slots), int(prefetch), _ptr(err_flag), _stream(stream))
+    _check(st, "semshare_probe_operand_stream")

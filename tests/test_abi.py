@@ -227,6 +227,17 @@ def test_probe_argument_errors(lib):
     assert p(0, FAKE, 1 << 30, None) == 1               # no iterations
     assert p((1 << 24) + 1, FAKE, 1 << 30, None) == 1   # too many
     assert p(16, None, 1 << 30, None) == 1              # no sink
+    s = lib.semshare_probe_operand_stream
+    s.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
+                  ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p]
+    assert s(None, 1024, 512, None, 0, 4, 0, None, None) == 1      # no rows
+    assert s(FAKE, 1000, 512, None, 0, 4, 0, None, None) == 1      # rows not a multiple of 128
+    assert s(FAKE, 1024, 96, None, 0, 4, 0, None, None) == 1       # d not a multiple of 64
+    assert s(FAKE, 1024, 512, None, 0, 0, 0, None, None) == 1      # no slot
+    assert s(FAKE, 1024, 512, None, 0, 13, 0, None, None) == 1     # more than 12
+    assert s(FAKE, 1024, 512, None, 0, 4, 65, None, None) == 1     # prefetch too deep
+    assert s(FAKE, 1024, 512, FAKE, 40, 4, 0, None, None) == 2     # code length
+    assert s(ctypes.c_void_p((1 << 20) + 8), 1024, 512, None, 0, 4, 0, None, None) == 1  # misaligned rows
 
 
 def test_deviation_and_select_argument_errors(lib):
