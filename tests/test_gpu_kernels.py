@@ -88,6 +88,8 @@ def _hash_case(ss, orc, n, d, nbits, dtype, pos_kind, pad=0, seed=0):
         (385, 2048, 256, "f32", "large", 32),
         (1536, 1024, 192, "bf16", "own", 0),     # 192-bit codes: the slot count rounded to the RoPE groups
         (700, 512, 128, "f32", "random", 0),      # fp32 rows with 128-bit codes: two pipeline slots
+        (300, 8192, 256, "bf16", "own", 0),       # wider rows than any workload: 128 K blocks per tile
+        (257, 64, 64, "bf16", "random", 0),       # one K block per tile
     ],
 )
 def test_hash_parity(ss, orc, n, d, nbits, dtype, pos_kind, pad):
