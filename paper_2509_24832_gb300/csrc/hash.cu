@@ -577,6 +577,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar_ready + 8u * s);
+                // a pair call's range may go on into rotated tiles: this group's next stage needs its
+                // table entries whichever kind of tile this one was
+                if (kRot == kRotPair && it + kRopeGroups < i1) {
+                    const int kb = static_cast<int>((it + kRopeGroups) % nkb);
+#pragma unroll
+                    for (int j = 0; j < kGroupChunks; ++j)
+                        load_pairs4(a.rope_table, half, kb, c0 + kChunkStride * j, tn[j]);
+                }
                 continue;
             }
 #pragma unroll
