@@ -304,12 +304,20 @@ void oracle_kv_deviation(const void* k_re, const void* v_re, const void* k_rc, c
 
 /* High-deviation tokens (Insight 1: the tokens of highest deviation, 40% of them in the paper):
  * for each layer, the k tokens of largest sigma (ties to the lower token index), listed in
- * ascending token order in hd_idx[l][0..k).  A plain sort of (-sigma, t). */
+ * ascending token order in hd_idx[l][0..k).  A plain sort of (-sigma, t) under a total order:
+ * every NaN (either sign, any payload) ranks above +inf and NaNs tie with each other; -0 and +0
+ * are the same number; equal values go to the lower token.  The comparator is therefore
+ * transitive, so qsort's result is defined even when sigma holds NaNs. */
 static const double* g_sort_sigma;
 static int cmp_desc_sigma(const void* a, const void* b) {
     const int64_t i = *(const int64_t*)a, j = *(const int64_t*)b;
-    if (g_sort_sigma[i] > g_sort_sigma[j]) return -1;
-    if (g_sort_sigma[i] < g_sort_sigma[j]) return 1;
+    const double x = g_sort_sigma[i], y = g_sort_sigma[j];
+    const int nx = isnan(x) != 0, ny = isnan(y) != 0;
+    if (nx != ny) return nx ? -1 : 1;     /* a NaN comes before every number */
+    if (!nx) {                            /* two numbers (-0 == +0 here) */
+        if (x > y) return -1;
+        if (x < y) return 1;
+    }
     return i < j ? -1 : (i > j ? 1 : 0);
 }
 static int cmp_i64(const void* a, const void* b) {

@@ -105,3 +105,77 @@ def test_select_brute_force(oracle_mod, T, k):
     np.testing.assert_array_equal(got, _brute_select(sigma, k))
     np.testing.assert_array_equal(got[2], np.arange(k))
     assert all(np.all(np.diff(r) > 0) for r in got)
+
+
+def _nan(bits: int) -> float:
+    return float(np.array([bits], dtype=np.uint64).view(np.float64)[0])
+
+
+def _total_order_key(v: float, t: int):
+    """Python's own sort key of the selection order: NaN (any sign or payload) first, then larger
+    values first (-0 and +0 equal: Python's == says so), then the lower token."""
+    return (0, 0.0, t) if v != v else (1, -v, t)
+
+
+def _brute_select_total(sigma, k):
+    return np.array([sorted(sorted(range(len(row)), key=lambda t: _total_order_key(row[t], t))[:k]) for row in sigma],
+                    dtype=np.int64).reshape(len(sigma), k)
+
+
+@pytest.mark.parametrize("k", list(range(0, 14)))
+def test_select_nan_inf_signed_zero(oracle_mod, k):
+    """Special values at every k: NaNs of both signs and several payloads rank above +inf and tie
+    with each other (lower token first), -inf ranks last, -0 ties with +0."""
+    qnan, neg_qnan = _nan(0x7FF8000000000000), _nan(0xFFF8000000000000)
+    payload, neg_payload = _nan(0x7FF0000000000123), _nan(0xFFF4000000000001)
+    row = [0.5, neg_qnan, -0.0, np.inf, 0.0, qnan, -np.inf, 0.5, payload, 1e300, -0.0, neg_payload, 0.25]
+    assert len(row) == 13
+    sigma = np.array([row, row[::-1]], dtype=np.float64)
+    got = oracle_mod.select_hd(sigma, min(k, 13))
+    np.testing.assert_array_equal(got, _brute_select_total(sigma, min(k, 13)))
+    # by hand: the four NaNs first (tokens 1, 5, 8, 11), then +inf (3), 1e300 (9), the two 0.5
+    # (0, 7), 0.25 (12), the three zeros in token order (2, 4, 10), -inf (6)
+    rank = [1, 5, 8, 11, 3, 9, 0, 7, 12, 2, 4, 10, 6]
+    np.testing.assert_array_equal(got[0], sorted(rank[:min(k, 13)]))
+
+
+def test_select_zeros_tie_by_token(oracle_mod):
+    """-0 and +0 are one value: among them the lower tokens win, whatever their signs."""
+    sigma = np.array([[0.0, -0.0, 0.0, -0.0, -0.0, 0.0]])
+    for k in range(7):
+        np.testing.assert_array_equal(oracle_mod.select_hd(sigma, k)[0], np.arange(k))
+    sigma = np.array([[-0.0, 0.0, -0.0, 0.0, -0.0, 0.0]])
+    np.testing.assert_array_equal(oracle_mod.select_hd(sigma, 3)[0], [0, 1, 2])
+
+
+def test_select_random_special_values(oracle_mod):
+    """Random rows drawn from a small pool of specials and ties, against the Python sort."""
+    g = np.random.default_rng(77)
+    pool = np.array([np.nan, -np.nan, np.inf, -np.inf, 0.0, -0.0, 1.0, 1.0, 2.0, -1.0, 3.5])
+    pool[1] = _nan(0xFFF8000000000000)
+    for T in (1, 2, 7, 64, 301):
+        sigma = pool[g.integers(0, len(pool), size=(4, T))]
+        for k in sorted({0, 1, T // 3, (40 * T + 99) // 100, T}):
+            np.testing.assert_array_equal(oracle_mod.select_hd(sigma, k), _brute_select_total(sigma, k))
+
+
+def test_kv_deviation_nan_and_inf_payloads(oracle_mod):
+    """A NaN anywhere in a token's rows makes its deviation NaN; inf minus a finite value is inf;
+    inf minus inf is NaN.  The other tokens are unaffected."""
+    shape = (1, 2, 4, 8)
+    k_re, k_rc, v_re, v_rc = _bf16_arrays(shape, seed=5)
+    base = oracle_mod.kv_deviation(k_re, v_re, k_rc, v_rc)
+    k_re2 = k_re.copy()
+    k_re2[0, 1, 1, 3] = 0x7FC1          # NaN in token 1's K
+    k_re2[0, 0, 2, 0] = 0x7F80          # +inf in token 2's K (the recomputed value is finite)
+    v_re2, v_rc2 = v_re.copy(), v_rc.copy()
+    v_re2[0, 1, 3, 5] = 0xFF80          # -inf - (-inf) = NaN in token 3's V
+    v_rc2[0, 1, 3, 5] = 0xFF80
+    sk, sv, skv = oracle_mod.kv_deviation(k_re2, v_re2, k_rc, v_rc2)
+    assert np.isnan(sk[0, 1]) and np.isnan(skv[0, 1])
+    assert np.isinf(sk[0, 2]) and np.isinf(skv[0, 2])
+    assert np.isnan(sv[0, 3]) and np.isnan(skv[0, 3])
+    np.testing.assert_array_equal(skv[0, 0], base[2][0, 0])
+    # the selection ranks the NaN tokens first, then the inf token
+    np.testing.assert_array_equal(oracle_mod.select_hd(skv, 2)[0], [1, 3])
+    np.testing.assert_array_equal(oracle_mod.select_hd(skv, 3)[0], [1, 2, 3])
