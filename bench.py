@@ -175,22 +175,51 @@ def popc_peak_wordops(sm_mhz: float, sms: int) -> float:
     return 16.0 * sms * sm_mhz * 1e6
 
 
+PROBE_CHAINS = 8  # SEMSHARE_PROBE_CHAINS (include/semshare_probe.h): word operations per thread and iteration
+
+
+def load_probe():
+    """libsemshare_probe.so (measurement support, built beside libsemshare.so by build.py)."""
+    import ctypes
+
+    from paper_2509_24832_gb300 import build
+
+    if not os.path.exists(build.PROBE_LIB):
+        raise RuntimeError(f"{build.PROBE_LIB} is missing: build the library first")
+    lib = ctypes.CDLL(build.PROBE_LIB)
+    lib.semshare_probe_hamming_threads.argtypes = []
+    lib.semshare_probe_hamming_threads.restype = ctypes.c_int64
+    lib.semshare_probe_hamming_rate.argtypes = [ctypes.c_int64, ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p]
+    lib.semshare_probe_hamming_rate.restype = ctypes.c_int
+    return lib
+
+
 def measure_hamming_rate(device, iters: int = 1 << 14, reps: int = 5) -> float:
     """Sustained xor/popc/add word-ops per second of this GPU (semshare_probe_hamming_rate:
     independent chains in registers, every SM fully occupied), best of `reps` launches timed
     with CUDA events after a warm-up launch."""
     import torch
 
-    import paper_2509_24832_gb300 as ss
+    probe = load_probe()
+    threads = int(probe.semshare_probe_hamming_threads())
+    if threads <= 0:
+        raise RuntimeError("semshare_probe_hamming_threads failed")
+    sink = torch.empty(threads, dtype=torch.int32, device=device)
 
-    sink = torch.empty(ss.semshare_probe_hamming_threads(), dtype=torch.int32, device=device)
-    ops = ss.semshare_probe_hamming_rate(iters, sink)
+    def launch():
+        st = probe.semshare_probe_hamming_rate(iters, sink.data_ptr(), sink.numel(),
+                                               torch.cuda.current_stream(device).cuda_stream)
+        if st != 0:
+            raise RuntimeError(f"semshare_probe_hamming_rate: status {st}")
+
+    ops = threads * iters * PROBE_CHAINS
+    launch()
     torch.cuda.synchronize()
     best = float("inf")
     for _ in range(reps):
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record()
-        ss.semshare_probe_hamming_rate(iters, sink)
+        launch()
         b.record()
         b.synchronize()
         best = min(best, a.elapsed_time(b) * 1e-3)
@@ -309,7 +338,7 @@ class Problem:
         if with_retain:
             if wl.n_batch != 1 or with_hd:
                 raise ValueError("--retain takes a one-prompt workload and no --hd")
-            self.counts = ss.retain_counts(wl.n_tgt, workloads.retain_alphas(L))
+            self.counts = ss.retain_counts(wl.n_tgt, workloads.retain_alphas(L), workloads.RETAIN_DEN)
             ret = workloads.retained_tokens(wl.n_tgt, self.counts, seed)
             self.ret = torch.from_numpy(np.concatenate(ret)).to(device)
             self.ret_off = [0] + list(np.cumsum(self.counts))

@@ -318,8 +318,10 @@ semshare_status semshare_match_tc_selected(const uint32_t* tgt_codes, int64_t n_
  *   n_tgt      0 <= n_tgt <= SEMSHARE_MATCH_STATIC_MAX_TARGETS; larger requests return
  *              SEMSHARE_ETOOLARGE before anything is enqueued
  *   other arguments as for semshare_match
- * The first call on a device looks up that device's address of the array (once per device,
- * with the device current); make that first call before any stream capture.  All calls on a
+ * The first call on a device looks up that device's address of the array (with the device
+ * current), and looks it up again on the first call after the device's current context has
+ * changed (cudaDeviceReset, or a context the caller made current); make the first call on a
+ * device, and the first after such a change, before any stream capture.  All calls on a
  * device share the one array and it keeps the previous call's contents; each call resets the
  * keys it uses before its search.  Calls whose work overlaps on the GPU (other streams, other
  * host threads on the same device) race on the array and give wrong results: serialise them.
@@ -377,6 +379,36 @@ semshare_status semshare_gather_kv(const void* const* ref_k, const void* const* 
                                    int32_t n_seg, semshare_kv_layout src, const int32_t* idx, int64_t n_tgt,
                                    int32_t n_batch, void* out_k, void* out_v, semshare_kv_layout dst,
                                    uint32_t* err_flag, void* stream);
+
+/*
+ * semshare_hd_count -- how many tokens of a layer are high-deviation (HD) tokens.
+ *
+ * Insight 1 (App. A.4) names the tokens with the highest KV deviation, 40% of them, HD tokens.
+ * Returns ceil(n_tok * percent / 100) computed in integers (percent = 40 for the paper's
+ * figure), the k that semshare_select_hd takes.  Host-only, no device work.
+ *   n_tok     0 <= n_tok < 2^40
+ *   percent   0..100
+ * Returns -1 for arguments outside those ranges.
+ */
+int64_t semshare_hd_count(int64_t n_tok, int32_t percent);
+
+/*
+ * semshare_retain_counts -- retained tokens per layer, Retain[i] = T * prod_{j<=i} alpha[j].
+ *
+ * App. A gives the number of tokens layer i keeps as the product of T (the target's length)
+ * and the retention ratios of layers 0..i; Sec. 3.3.4 sets them.  The ratios are rationals
+ * alpha[j] = alpha_num[j] / alpha_den, and the count is rounded down exactly (integer
+ * arithmetic on the exact product, no floating point): counts[i] = floor(T * prod num / den^(i+1)).
+ * Host-only, no device work.
+ *   n_tok       T, 0 <= T < 2^31
+ *   alpha_num   host int32[n_layers], 0 <= alpha_num[j] <= alpha_den
+ *   alpha_den   >= 1 (e.g. 1000 for ratios given to three decimals)
+ *   n_layers    0..128
+ *   counts      host int64[n_layers], written
+ * Returns EINVAL for arguments outside those ranges.
+ */
+semshare_status semshare_retain_counts(int64_t n_tok, const int32_t* alpha_num, int32_t alpha_den,
+                                       int32_t n_layers, int64_t* counts);
 
 /*
  * semshare_gather_kv_retained -- step 4 with retention: each layer keeps only its retained tokens.
@@ -473,7 +505,9 @@ semshare_status semshare_kv_deviation(const void* k_reused, const void* v_reused
  * Insight 1 calls the tokens of highest KV deviation (40% of them) HD tokens; Sec. 3.2 hands
  * the ones found on the first layer to recomputation.  For each layer l < n_layers: the k tokens
  * with the largest sigma[l][t], ties at the k-th value going to the lower token index, listed in
- * ascending token order.  NaN counts as larger than every number.
+ * ascending token order.  The order is total: every NaN (either sign, any payload) counts as
+ * larger than every number, including +inf, and NaNs tie with each other (lower token first);
+ * -0 and +0 are the same value.
  *
  *   sigma     device float[n_layers][n_tok] (e.g. semshare_kv_deviation's sigma_kv)
  *   k         0 <= k <= n_tok (the paper's 40%: k = ceil(0.4 * n_tok))

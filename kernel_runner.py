@@ -1,6 +1,6 @@
 """Runs one library call on a workload's synthetic inputs, a few times, for profilers.
 
-    python -m paper_2509_24832_gb300.kernel_runner --kernel hash|match|match_tc|gather|retrieve
+    python kernel_runner.py --kernel hash|match|match_tc|gather|retrieve
         --workload NAME [--reps N]
 
 Only the buffers that call needs are allocated (e.g. the 5k-token hash holds ~100 MB, the
@@ -18,7 +18,7 @@ import sys
 import numpy as np
 import torch
 
-ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
@@ -101,7 +101,7 @@ def main(argv=None):
                 # the synthetic retention schedule of bench.py --retain (one prompt)
                 del e
                 k, v = workloads.kv_cache_device(wl, dev)
-                counts = ss.retain_counts(wl.n_tgt, workloads.retain_alphas(wl.n_layers))
+                counts = ss.retain_counts(wl.n_tgt, workloads.retain_alphas(wl.n_layers), workloads.RETAIN_DEN)
                 ret = workloads.retained_tokens(wl.n_tgt, counts, wl.base_seed)
                 flat = torch.from_numpy(np.concatenate(ret)).to(dev)
                 offs = [0] + list(np.cumsum(counts))

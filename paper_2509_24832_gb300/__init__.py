@@ -18,7 +18,6 @@ from ._native import (  # noqa: F401
     LIB_PATH,
     Prepared,
     MATCH_STATIC_MAX_TARGETS,
-    PROBE_CHAINS,
     RETAIN_MAX_LAYERS,
     RETRIEVE_MAX_CANDIDATES,
     SIMILARITY_MAX_DIST,
@@ -50,9 +49,6 @@ from ._native import (  # noqa: F401
     semshare_match_tc_selected_workspace_size,
     semshare_match_tc_workspace_size,
     semshare_match_workspace_size,
-    semshare_probe_hamming_rate,
-    semshare_probe_hamming_threads,
-    semshare_probe_operand_stream,
     semshare_retrieve,
     semshare_retrieve_workspace_size,
     semshare_rope_table,

@@ -6,7 +6,6 @@ library is missing the call raises."""
 from __future__ import annotations
 
 import ctypes
-import math
 import os
 import threading
 from typing import NamedTuple
@@ -102,12 +101,10 @@ def load():
         lib.semshare_kv_deviation.restype = ctypes.c_int
         lib.semshare_select_hd.argtypes = [P, i32, i64, i64, P, P, P]
         lib.semshare_select_hd.restype = ctypes.c_int
-        lib.semshare_probe_hamming_threads.argtypes = []
-        lib.semshare_probe_hamming_threads.restype = i64
-        lib.semshare_probe_hamming_rate.argtypes = [i64, P, i64, P]
-        lib.semshare_probe_hamming_rate.restype = ctypes.c_int
-        lib.semshare_probe_operand_stream.argtypes = [P, i64, i32, P, i32, i32, i32, P, P]
-        lib.semshare_probe_operand_stream.restype = ctypes.c_int
+        lib.semshare_hd_count.argtypes = [i64, i32]
+        lib.semshare_hd_count.restype = i64
+        lib.semshare_retain_counts.argtypes = [i64, P, i32, i32, P]
+        lib.semshare_retain_counts.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -634,8 +631,11 @@ HD_PERCENT = 40  # Insight 1: the 40% of tokens with the highest deviation are H
 
 
 def hd_count(n_tok: int, percent: int = HD_PERCENT) -> int:
-    """Number of HD tokens: ceil(percent% of n_tok), in integer arithmetic."""
-    return (int(n_tok) * int(percent) + 99) // 100
+    """Number of HD tokens, ceil(percent% of n_tok) (semshare_hd_count)."""
+    k = int(load().semshare_hd_count(int(n_tok), int(percent)))
+    if k < 0:
+        raise SemshareError(EINVAL, "semshare_hd_count")
+    return k
 
 
 def semshare_kv_deviation(k_reused: torch.Tensor, v_reused: torch.Tensor, k_recomp: torch.Tensor,
@@ -695,14 +695,15 @@ def semshare_select_hd(sigma: torch.Tensor, k: int | None = None, hd_idx: torch.
 RETAIN_MAX_LAYERS = 128
 
 
-def retain_counts(n_tok: int, alphas) -> list:
-    """Retained tokens per layer, Retain[i] = T * prod_{j<=i} alpha_retain[j] (App. A), rounded
-    down (a product within 1e-9 of an integer counts as that integer)."""
-    out, p = [], 1.0
-    for a in alphas:
-        p *= float(a)
-        out.append(int(math.floor(n_tok * p + 1e-9)))
-    return out
+def retain_counts(n_tok: int, alpha_num, alpha_den: int) -> list:
+    """Retained tokens per layer, Retain[i] = floor(T * prod_{j<=i} alpha_num[j] / alpha_den)
+    (App. A), computed exactly by semshare_retain_counts."""
+    num = [int(a) for a in alpha_num]
+    n = len(num)
+    arr = (ctypes.c_int32 * max(n, 1))(*num)
+    out = (ctypes.c_int64 * max(n, 1))()
+    _check(load().semshare_retain_counts(int(n_tok), arr, int(alpha_den), n, out), "semshare_retain_counts")
+    return [int(out[i]) for i in range(n)]
 
 
 def semshare_gather_kv_retained(ref_k, ref_v, idx: torch.Tensor, retained, ret_offsets,
@@ -744,47 +745,3 @@ def semshare_gather_kv_retained(ref_k, ref_v, idx: torch.Tensor, retained, ret_o
                                             _ptr(out_k), _ptr(out_v), dst, _ptr(err_flag), _stream(stream))
     _check(st, "semshare_gather_kv_retained")
     return out_k, out_v
-
-
-PROBE_CHAINS = 8  # SEMSHARE_PROBE_CHAINS: word operations per thread and iteration
-
-
-def semshare_probe_hamming_threads() -> int:
-    n = int(load().semshare_probe_hamming_threads())
-    if n < 0:
-        raise SemshareError(3, "semshare_probe_hamming_threads")
-    return n
-
-
-def semshare_probe_hamming_rate(iters: int, sink: torch.Tensor, stream=None) -> int:
-    """Enqueues one launch of the word-operation probe (measurement support: the xor/popc/add
-    rate that bounds semshare_match).  sink: device int32/uint32 tensor of at least
-    semshare_probe_hamming_threads() words.  Returns the word operations the launch performs;
-    time it with CUDA events on the stream."""
-    _need_cuda(sink, "sink")
-    st = load().semshare_probe_hamming_rate(int(iters), _ptr(sink), sink.numel(), _stream(stream))
-    _check(st, "semshare_probe_hamming_rate")
-    return semshare_probe_hamming_threads() * int(iters) * PROBE_CHAINS
-
-
-def semshare_probe_operand_stream(emb: torch.Tensor, hyperplanes: torch.Tensor | None = None, slots: int = 4,
-                                  prefetch: int = 0, err_flag: torch.Tensor | None = None, stream=None) -> None:
-    """Enqueues one launch that moves semshare_hash's operand blocks (the 128 x 64 embedding
-    block and, if given, the nbits x 64 hyperplane block of every (tile, K block) iteration)
-    through a ring of `slots` shared-memory slots with no rotation and no MMA (measurement
-    support: the floor the operand traffic sets for the hash kernel).  emb: contiguous bf16
-    [n][d] on the device, n a multiple of 128; hyperplanes: contiguous bf16 [nbits][d] or None.
-    Time the launch with CUDA events on the stream."""
-    _need_cuda(emb, "emb")
-    if emb.dtype != torch.bfloat16 or emb.dim() != 2 or not emb.is_contiguous():
-        raise SemshareError(EINVAL, "semshare_probe_operand_stream: emb must be a contiguous 2-D bf16 tensor")
-    nbits = 0
-    if hyperplanes is not None:
-        _need_cuda(hyperplanes, "hyperplanes")
-        if hyperplanes.dtype != torch.bfloat16 or hyperplanes.dim() != 2 or not hyperplanes.is_contiguous() \
-                or hyperplanes.shape[1] != emb.shape[1]:
-            raise SemshareError(EINVAL, "semshare_probe_operand_stream: hyperplanes must be contiguous bf16 [nbits][d]")
-        nbits = hyperplanes.shape[0]
-    st = load().semshare_probe_operand_stream(_ptr(emb), emb.shape[0], emb.shape[1], _ptr(hyperplanes), nbits,
-                                              int(slots), int(prefetch), _ptr(err_flag), _stream(stream))
-    _check(st, "semshare_probe_operand_stream")

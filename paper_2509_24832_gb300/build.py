@@ -16,7 +16,11 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "libsemshare.so")
-SOURCES = ["api.cu", "hash.cu", "match.cu", "match_tc.cu", "gather.cu", "deviation.cu", "fetch.cu", "probe.cu"]
+SOURCES = ["api.cu", "hash.cu", "match.cu", "match_tc.cu", "gather.cu", "deviation.cu", "fetch.cu"]
+# measurement support, linked into a library of its own so that libsemshare.so exports only the
+# entry points of include/semshare.h
+PROBE_SOURCES = ["probe.cu"]
+PROBE_LIB = os.path.join(LIBDIR, "libsemshare_probe.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 # -warn-spills: a register spill in a file with tensor-memory loads is a build error (below).  Those
 # kernels hand tcgen05.ld destination registers to later code before the load's wait; a spill placed
@@ -34,19 +38,20 @@ def nvcc() -> str:
 
 
 def _inputs():
-    return [os.path.join(CSRC, s) for s in SOURCES] + glob.glob(os.path.join(CSRC, "*.cuh")) + \
+    return [os.path.join(CSRC, s) for s in SOURCES + PROBE_SOURCES] + glob.glob(os.path.join(CSRC, "*.cuh")) + \
         glob.glob(os.path.join(INCLUDE, "*.h")) + [os.path.abspath(__file__)]
 
 
 def up_to_date() -> bool:
-    if not os.path.exists(LIB):
+    if not os.path.exists(LIB) or not os.path.exists(PROBE_LIB):
         return False
-    t = os.path.getmtime(LIB)
+    t = min(os.path.getmtime(LIB), os.path.getmtime(PROBE_LIB))
     return all(os.path.getmtime(p) <= t for p in _inputs())
 
 
 def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | None = None) -> str:
-    """Compile and link libsemshare.so; returns its path.  No-op when up to date."""
+    """Compile and link libsemshare.so (and the measurement probe library libsemshare_probe.so);
+    returns the path of libsemshare.so.  No-op when up to date."""
     if not force and not extra_flags and up_to_date():
         return LIB
     os.makedirs(os.path.join(LIBDIR, "obj"), exist_ok=True)
@@ -54,7 +59,7 @@ def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | N
     flags = NVCC_FLAGS + list(extra_flags or [])
     procs = []
     objs = []
-    for src in SOURCES:
+    for src in SOURCES + PROBE_SOURCES:
         obj = os.path.join(LIBDIR, "obj", src.replace(".cu", ".o"))
         objs.append(obj)
         cmd = [cc, *flags, "-c", os.path.join(CSRC, src), "-o", obj]
@@ -71,9 +76,11 @@ def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | N
             failed.append(src)
     if failed:
         raise RuntimeError(f"nvcc failed (or spilled registers) on {failed}")
-    tmp = LIB + f".tmp{os.getpid()}"
-    subprocess.run([cc, *ARCH, "-shared", "-Xcompiler", "-fPIC", *objs, "-o", tmp], check=True)
-    os.replace(tmp, LIB)
+    n = len(SOURCES)
+    for lib, parts in ((LIB, objs[:n]), (PROBE_LIB, objs[n:])):
+        tmp = lib + f".tmp{os.getpid()}"
+        subprocess.run([cc, *ARCH, "-shared", "-Xcompiler", "-fPIC", *parts, "-o", tmp], check=True)
+        os.replace(tmp, lib)
     return LIB
 
 

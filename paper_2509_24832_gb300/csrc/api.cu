@@ -59,3 +59,82 @@ extern "C" semshare_status semshare_rope_table(int32_t d, double rope_base, uint
         return SEMSHARE_ECUDA;
     return launch_status();
 }
+
+// ---- host-side counts of the method (no device work) --------------------------------------
+
+extern "C" int64_t semshare_hd_count(int64_t n_tok, int32_t percent) {
+    if (n_tok < 0 || n_tok >= (int64_t(1) << 40) || percent < 0 || percent > 100) return -1;
+    // ceil(n_tok * percent / 100) in integers
+    return (n_tok * percent + 99) / 100;
+}
+
+namespace semshare {
+namespace {
+
+// Unsigned integer of up to kLimbs 32-bit limbs (least significant first): just the two
+// operations Retain[i] needs, multiply and divide by a 32-bit value.
+constexpr int kRetainLimbs = 160;  // 31 bits of n_tok + 31 bits per layer for 128 layers, with room
+
+struct BigUint {
+    uint32_t limb[kRetainLimbs];
+    int n;  // limbs in use (the top one non-zero, or n == 0 for zero)
+};
+
+void big_set(BigUint& x, uint64_t v) {
+    x.n = 0;
+    while (v) {
+        x.limb[x.n++] = static_cast<uint32_t>(v);
+        v >>= 32;
+    }
+}
+
+bool big_mul(BigUint& x, uint32_t m) {
+    uint64_t carry = 0;
+    for (int i = 0; i < x.n; ++i) {
+        const uint64_t t = static_cast<uint64_t>(x.limb[i]) * m + carry;
+        x.limb[i] = static_cast<uint32_t>(t);
+        carry = t >> 32;
+    }
+    if (carry) {
+        if (x.n == kRetainLimbs) return false;
+        x.limb[x.n++] = static_cast<uint32_t>(carry);
+    }
+    while (x.n > 0 && x.limb[x.n - 1] == 0) --x.n;
+    return true;
+}
+
+void big_div(BigUint& x, uint32_t d) {  // x = floor(x / d)
+    uint64_t rem = 0;
+    for (int i = x.n - 1; i >= 0; --i) {
+        const uint64_t cur = (rem << 32) | x.limb[i];
+        x.limb[i] = static_cast<uint32_t>(cur / d);
+        rem = cur % d;
+    }
+    while (x.n > 0 && x.limb[x.n - 1] == 0) --x.n;
+}
+
+}  // namespace
+}  // namespace semshare
+
+extern "C" semshare_status semshare_retain_counts(int64_t n_tok, const int32_t* alpha_num, int32_t alpha_den,
+                                                  int32_t n_layers, int64_t* counts) {
+    using namespace semshare;
+    if (n_tok < 0 || n_tok >= (int64_t(1) << 31) || alpha_den < 1 || n_layers < 0 || n_layers > 128)
+        return SEMSHARE_EINVAL;
+    if (n_layers > 0 && (alpha_num == nullptr || counts == nullptr)) return SEMSHARE_EINVAL;
+    for (int32_t i = 0; i < n_layers; ++i)
+        if (alpha_num[i] < 0 || alpha_num[i] > alpha_den) return SEMSHARE_EINVAL;
+    // Retain[i] = floor(n_tok * prod_{j<=i} num_j / den^(i+1)), exact: the numerator as a big
+    // integer, then i+1 divisions by den (floor(floor(x/a)/b) = floor(x/(a*b)) for integers).
+    BigUint num;
+    big_set(num, static_cast<uint64_t>(n_tok));
+    for (int32_t i = 0; i < n_layers; ++i) {
+        if (!big_mul(num, static_cast<uint32_t>(alpha_num[i]))) return SEMSHARE_EUNSUPPORTED;
+        BigUint q = num;
+        for (int32_t j = 0; j <= i && q.n > 0; ++j) big_div(q, static_cast<uint32_t>(alpha_den));
+        uint64_t v = 0;
+        for (int k = q.n - 1; k >= 0; --k) v = (v << 32) | q.limb[k];  // <= n_tok < 2^31
+        counts[i] = static_cast<int64_t>(v);
+    }
+    return SEMSHARE_OK;
+}

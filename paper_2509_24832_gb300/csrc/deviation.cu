@@ -125,9 +125,13 @@ __global__ void __launch_bounds__(kDevThreads) kv_deviation_kernel(const DevArgs
         deviation_of_token(a, w, lane);
 }
 
-// Order-preserving image of an fp32 value as an unsigned integer (NaN above +inf).
+// Order-preserving image of an fp32 value as an unsigned integer under the selection's total
+// order: every NaN, of either sign and any payload, maps to the one largest key (above +inf, and
+// tied with every other NaN, so the lower token wins); -0 maps to the key of +0.
 __device__ __forceinline__ uint32_t order_key(float f) {
-    const uint32_t u = __float_as_uint(f);
+    uint32_t u = __float_as_uint(f);
+    if ((u & 0x7FFFFFFFu) > 0x7F800000u) return 0xFFFFFFFFu;  // NaN (exponent all ones, mantissa != 0)
+    if (u == 0x80000000u) u = 0u;
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 

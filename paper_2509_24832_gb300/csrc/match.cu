@@ -14,6 +14,8 @@
 // block, each target's best (distance << 32 | global index) goes to a 64-bit atomicMin in the
 // workspace.  atomicMin of that key is exactly "smallest distance, then lowest index", so the
 // result does not depend on the partition.  A final pass splits the keys into idx and dist.
+#include <cuda.h>
+
 #include <mutex>
 
 #include "common.cuh"
@@ -227,22 +229,59 @@ namespace {
 
 constexpr int kStaticMaxDevices = 64;
 std::mutex g_static_keys_mutex;
-unsigned long long* g_static_keys_addr[kStaticMaxDevices] = {};
+struct StaticKeysEntry {
+    unsigned long long ctx_id;  // the context the address belongs to (0: none looked up yet)
+    unsigned long long* addr;
+};
+StaticKeysEntry g_static_keys[kStaticMaxDevices] = {};
 
-// Device address of g_static_match_keys on the current device.  In host code the array's name
-// is only a host-side stand-in, so the address is looked up once per device (with that device
-// current) and cached.
+// Unique id of the calling thread's current CUDA context (0 if there is none or the driver
+// cannot say).  Ids are never reused within a process, unlike context handles.
+unsigned long long current_context_id() {
+    using GetCurrentFn = CUresult (*)(CUcontext*);
+    using GetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+    static GetCurrentFn get_current = nullptr;  // resolved once per process
+    static GetIdFn get_id = nullptr;
+    if (get_current == nullptr || get_id == nullptr) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            return 0;
+        get_current = reinterpret_cast<GetCurrentFn>(p);
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            return 0;
+        get_id = reinterpret_cast<GetIdFn>(p);
+    }
+    CUcontext ctx = nullptr;
+    unsigned long long id = 0;
+    if (get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr || get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+    return id;
+}
+
+// Device address of g_static_match_keys in the current device's current context.  In host code
+// the array's name is only a host-side stand-in, so the address is looked up (with the device
+// current) the first time a device is used, and again whenever the device's current context is
+// not the one the cached address belongs to (after cudaDeviceReset, or when the caller switches
+// to a context of its own), since the array lives at a per-context address.
 semshare_status static_keys_on_current_device(unsigned long long** keys) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return SEMSHARE_ECUDA;
     if (dev < 0 || dev >= kStaticMaxDevices) return SEMSHARE_EUNSUPPORTED;
     std::lock_guard<std::mutex> lock(g_static_keys_mutex);
-    if (g_static_keys_addr[dev] == nullptr) {
+    StaticKeysEntry& e = g_static_keys[dev];
+    unsigned long long ctx_id = current_context_id();
+    if (ctx_id == 0 || e.ctx_id != ctx_id || e.addr == nullptr) {
+        // the lookup also makes the device's primary context current when no context is yet
         void* p = nullptr;
         if (cudaGetSymbolAddress(&p, g_static_match_keys) != cudaSuccess || p == nullptr) return SEMSHARE_ECUDA;
-        g_static_keys_addr[dev] = static_cast<unsigned long long*>(p);
+        if (ctx_id == 0) ctx_id = current_context_id();
+        if (ctx_id == 0) return SEMSHARE_ECUDA;
+        e.addr = static_cast<unsigned long long*>(p);
+        e.ctx_id = ctx_id;
     }
-    *keys = g_static_keys_addr[dev];
+    *keys = e.addr;
     return SEMSHARE_OK;
 }
 

@@ -19,21 +19,33 @@ def lib():
     return ss.load()
 
 
-def _declared():
-    names = set()
-    for fn in os.listdir(os.path.join(ROOT, "include")):
-        if fn.endswith(".h"):
-            text = open(os.path.join(ROOT, "include", fn)).read()
-            text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-            names |= set(re.findall(r"\b(semshare_\w+)\s*\(", text))
-    return sorted(names)
+@pytest.fixture(scope="module")
+def probe_lib(lib):
+    from paper_2509_24832_gb300 import build
+
+    p = ctypes.CDLL(build.PROBE_LIB)
+    p.semshare_probe_hamming_rate.argtypes = [ctypes.c_int64, ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p]
+    return p
 
 
-def test_every_declared_symbol_is_exported(lib):
-    names = _declared()
+def _declared(header):
+    text = open(os.path.join(ROOT, "include", header)).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(semshare_\w+)\s*\(", text)))
+
+
+def test_every_declared_symbol_is_exported(lib, probe_lib):
+    assert sorted(f for f in os.listdir(os.path.join(ROOT, "include")) if f.endswith(".h")) == \
+        ["semshare.h", "semshare_probe.h"]
+    names = _declared("semshare.h")
     assert {"semshare_hash", "semshare_match", "semshare_gather_kv", "semshare_rope_table"} <= set(names)
     for n in names:
         assert hasattr(lib, n), n
+    probes = _declared("semshare_probe.h")
+    assert probes == ["semshare_probe_hamming_rate", "semshare_probe_hamming_threads"]
+    for n in probes:
+        assert hasattr(probe_lib, n), n
+        assert not hasattr(lib, n), f"{n} is measurement support: it belongs to libsemshare_probe.so only"
 
 
 def test_status_helpers(lib):
@@ -222,22 +234,11 @@ def test_fetch_argument_errors(lib):
     assert f(pk, pk, pd, pd, offs, 1, lay, None, 0, None, 0, None, None) == 0               # empty
 
 
-def test_probe_argument_errors(lib):
-    p = lib.semshare_probe_hamming_rate
+def test_probe_argument_errors(probe_lib):
+    p = probe_lib.semshare_probe_hamming_rate
     assert p(0, FAKE, 1 << 30, None) == 1               # no iterations
     assert p((1 << 24) + 1, FAKE, 1 << 30, None) == 1   # too many
     assert p(16, None, 1 << 30, None) == 1              # no sink
-    s = lib.semshare_probe_operand_stream
-    s.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
-                  ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p]
-    assert s(None, 1024, 512, None, 0, 4, 0, None, None) == 1      # no rows
-    assert s(FAKE, 1000, 512, None, 0, 4, 0, None, None) == 1      # rows not a multiple of 128
-    assert s(FAKE, 1024, 96, None, 0, 4, 0, None, None) == 1       # d not a multiple of 64
-    assert s(FAKE, 1024, 512, None, 0, 0, 0, None, None) == 1      # no slot
-    assert s(FAKE, 1024, 512, None, 0, 13, 0, None, None) == 1     # more than 12
-    assert s(FAKE, 1024, 512, None, 0, 4, 65, None, None) == 1     # prefetch too deep
-    assert s(FAKE, 1024, 512, FAKE, 40, 4, 0, None, None) == 2     # code length
-    assert s(ctypes.c_void_p((1 << 20) + 8), 1024, 512, None, 0, 4, 0, None, None) == 1  # misaligned rows
 
 
 def test_deviation_and_select_argument_errors(lib):

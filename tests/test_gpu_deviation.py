@@ -161,3 +161,64 @@ def test_workload_layer0_after_gather(ss, orc):
     fresh = src[0] < 0
     frac = float(np.isin(np.nonzero(fresh)[0], hd.cpu().numpy()[0]).mean())
     print(f"HD tokens {hd.shape[1]} of {wl.n_tgt}; fresh tokens among them {frac:.3f}")
+
+
+def _f32_specials():
+    bits = np.array([0x7FC00000, 0xFFC00000, 0x7F800001, 0xFFBFFFFF,   # NaNs: both signs, several payloads
+                     0x7F800000, 0xFF800000, 0x00000000, 0x80000000,   # +inf, -inf, +0, -0
+                     0x3F800000, 0x3F800000, 0x40000000, 0xBF800000,   # 1, 1 (a tie), 2, -1
+                     0x00000001, 0x7F7FFFFF], dtype=np.uint32)          # a subnormal, the largest float
+    return bits.view(np.float32)
+
+
+@pytest.mark.parametrize("T", [13, 600, 70000])
+def test_select_nan_inf_signed_zero(ss, orc, T):
+    """NaNs of both signs rank above +inf and tie with each other (lower token first), -0 ties
+    with +0: element for element against the oracle's total order, on the staged (T <= ~57 K)
+    and the global selection paths, at every k around the special values."""
+    g = np.random.default_rng(T)
+    pool = _f32_specials()
+    s = pool[g.integers(0, len(pool), size=(3, T))].astype(np.float32)
+    s[2] = g.random(T).astype(np.float32)
+    s[2, g.integers(0, T, size=max(1, T // 50))] = pool[1]   # a few negative NaNs among ordinary values
+    s[2, g.integers(0, T, size=max(1, T // 50))] = -0.0
+    sd = torch.from_numpy(s).cuda()
+    n_nan = int(np.isnan(s).sum(axis=1).max())
+    ks = sorted({0, 1, 2, n_nan - 1, n_nan, n_nan + 1, (40 * T + 99) // 100, T - 1, T} & set(range(T + 1)))
+    for k in ks:
+        idx, mask = ss.semshare_select_hd(sd, k, want_mask=True)
+        torch.cuda.synchronize()
+        with np.errstate(invalid="ignore"):  # widening a signalling NaN raises the invalid flag
+            want = orc.select_hd(s.astype(np.float64), k)
+        np.testing.assert_array_equal(idx.cpu().numpy(), want, err_msg=f"T={T} k={k}")
+        m = np.zeros((3, T), dtype=np.uint8)
+        for l in range(3):
+            m[l, want[l]] = 1
+        np.testing.assert_array_equal(mask.cpu().numpy(), m)
+
+
+def test_deviation_nan_inf_payloads(ss, orc):
+    """K/V rows holding NaN and inf payloads: NaN and inf deviations land on the same tokens as the
+    oracle's, the finite ones agree within the tolerance, and the selection ranks them the same."""
+    shape = (2, 4, 333, 64)
+    k_re, v_re, k_rc, v_rc = _caches(shape, torch.bfloat16, seed=91)
+    kb = k_re.view(torch.int16)
+    vb, vcb = v_re.view(torch.int16), v_rc.view(torch.int16)
+    kb[0, 1, 7, 3] = 0x7FC1           # NaN in token 7 of layer 0
+    kb[1, 0, 100, 0] = -128           # 0xFF80 = -inf against a finite recomputed value
+    vb[0, 3, 200, 63] = -128          # -inf minus -inf: NaN
+    vcb[0, 3, 200, 63] = -128
+    kb[1, 2, 5, 9] = 0x7F80           # +inf
+    kb[1, 2, 6, 9] = -63              # 0xFFC1: a NaN with the sign bit set
+    sk, sv, skv = ss.semshare_kv_deviation(k_re, v_re, k_rc, v_rc, want_parts=True)
+    torch.cuda.synchronize()
+    ok, ov, okv = orc.kv_deviation(*(_host(t) for t in (k_re, v_re, k_rc, v_rc)))
+    for got, want in ((sk, ok), (sv, ov), (skv, okv)):
+        g = got.cpu().numpy().astype(np.float64)
+        np.testing.assert_array_equal(np.isnan(g), np.isnan(want))
+        np.testing.assert_array_equal(np.isinf(g), np.isinf(want))
+        fin = np.isfinite(want)
+        np.testing.assert_allclose(g[fin], want[fin], rtol=RTOL, atol=1e-30)
+    assert np.isnan(okv[0, 7]) and np.isnan(okv[0, 200]) and np.isnan(okv[1, 6]) and np.isinf(okv[1, 100])
+    for k in (1, 2, 3, 4, 133, 333):
+        _check_select(ss, orc, skv, okv, k)

@@ -123,7 +123,7 @@ def test_retained_workload_5k(ss, orc):
     k, v = workloads.kv_cache_device(wl, dev)
     g = np.random.default_rng(11)
     idx = g.integers(0, wl.n_ref, size=wl.n_tgt).astype(np.int32)
-    counts = ss.retain_counts(wl.n_tgt, workloads.retain_alphas(wl.n_layers))
+    counts = ss.retain_counts(wl.n_tgt, workloads.retain_alphas(wl.n_layers), workloads.RETAIN_DEN)
     ret = workloads.retained_tokens(wl.n_tgt, counts, seed=wl.base_seed)
     ok, ov = _run(ss, [k], [v], idx, ret)
     for l in (0, 1, 17, wl.n_layers - 1):

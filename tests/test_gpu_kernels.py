@@ -409,45 +409,3 @@ def test_hamming_rate_probe_runs_and_is_plausible():
 
     rate = bench.measure_hamming_rate(torch.device("cuda"), iters=1 << 12, reps=3)
     assert 1e12 < rate < 1e14, rate
-
-
-@pytest.mark.gpu
-def test_operand_stream_probe_runs_and_is_bounded(ss):
-    """The hash kernel's operand stream on its own: the probe runs with and without the hyperplane
-    blocks, with and without L2 prefetch, over a ragged split of iterations (rows not a multiple of
-    the SM count's tiles), raises no timeout, refuses a ring that does not fit shared memory, and
-    is not slower than the hash kernel that adds rotation and MMAs to the same traffic."""
-    g = torch.Generator(device="cuda")
-    g.manual_seed(17)
-    emb = torch.randn((128 * 37, 1024), device="cuda", generator=g).to(torch.bfloat16)
-    hyp = torch.randn((256, 1024), device="cuda", generator=g).to(torch.bfloat16)
-    flag = ss.new_err_flag()
-    for h, slots, pf in [(None, 1, 0), (None, 12, 0), (hyp, 4, 8), (hyp[:64].contiguous(), 2, 3)]:
-        ss.semshare_probe_operand_stream(emb, h, slots, pf, flag)
-    torch.cuda.synchronize()
-    ss.check_flag(flag, "operand stream")
-    with pytest.raises(ss.SemshareError) as e:
-        ss.semshare_probe_operand_stream(emb, hyp, 12, 0, flag)  # 12 x 48 KB slots
-    assert e.value.status == 2
-
-    big = torch.randn((10240, 4096), device="cuda", generator=g).to(torch.bfloat16)
-    hyp = torch.randn((256, 4096), device="cuda", generator=g).to(torch.bfloat16)
-    pos = torch.arange(10240, dtype=torch.int32, device="cuda") % 5120
-    table = ss.semshare_rope_table(4096)
-    codes = ss.semshare_hash(big, table, hyp, pos)
-
-    def med(fn):
-        ts = []
-        for _ in range(7):
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            a.record()
-            fn()
-            b.record()
-            b.synchronize()
-            ts.append(a.elapsed_time(b))
-        return sorted(ts)[3]
-
-    t_stream = med(lambda: ss.semshare_probe_operand_stream(big, hyp, 4, 8, flag))
-    t_hash = med(lambda: ss.semshare_hash(big, table, hyp, pos, codes=codes))
-    ss.check_flag(flag, "operand stream")
-    assert 0 < t_stream <= t_hash * 1.05, (t_stream, t_hash)

@@ -3,13 +3,15 @@
 allocations, or a serving loop that must not allocate on its hot path).  It uses a fixed
 scratch array inside the library instead of a caller workspace.
 
-Its results must equal semshare_match's, bit for bit, on two calls in a row: the scratch array
-keeps the first call's keys, so the second call (a different, smaller problem) also checks
-that each call resets what it uses.  Sizes beyond the array's capacity must be refused before
-anything is enqueued.  This file is named to be collected last."""
+Its results must equal semshare_match's, bit for bit, on two calls in a row, and both must
+equal the CPU oracle's exhaustive search on the same codes: the scratch array keeps the first
+call's keys, so the second call (a different, smaller problem) also checks that each call
+resets what it uses.  Sizes beyond the array's capacity must be refused before anything is
+enqueued.  This file is named to be collected last."""
 import numpy as np
 import pytest
 
+import oracle
 import workloads
 
 torch = pytest.importorskip("torch")
@@ -24,6 +26,11 @@ def ss():
 
     ss.load()
     return ss
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _oracle_built():
+    oracle.build()
 
 
 def _codes(n, nbits, seed, stream):
@@ -43,6 +50,10 @@ def test_static_scratch_match_equals_workspace_match_on_two_calls(ss):
         torch.cuda.synchronize()
         assert torch.equal(idx, want_idx), f"idx differs on the {n_tgt}-target call"
         assert torch.equal(dist, want_dist), f"dist differs on the {n_tgt}-target call"
+        # both against the oracle's exhaustive scan (ties to the lowest reference index)
+        oi, od = oracle.match(tgt.cpu().numpy().view(np.uint32), ref.cpu().numpy().view(np.uint32))
+        np.testing.assert_array_equal(idx.cpu().numpy(), oi, err_msg=f"{n_tgt}-target call vs the oracle")
+        np.testing.assert_array_equal(dist.cpu().numpy(), od, err_msg=f"{n_tgt}-target call vs the oracle")
 
 
 def test_static_scratch_match_refuses_sizes_beyond_capacity(ss):

@@ -283,8 +283,13 @@ def recomputed_kv_device(wl: Workload, device, k_ref, v_ref, src, seed: int | No
 # Retention schedule for the synthetic workloads (Sec. 3.3.4, App. A: alpha_retain larger in
 # shallow layers, smaller in deep ones; the first layer keeps max(0.8, r_dynamic)): 0.8 on the
 # first layer, then 0.98 per layer.
+RETAIN_DEN = 1000  # the synthetic retention ratios are given in thousandths
+
+
 def retain_alphas(n_layers: int) -> list:
-    return [0.8] + [0.98] * (n_layers - 1)
+    """Numerators over RETAIN_DEN of the synthetic per-layer retention ratios: 0.8 on the first
+    layer, then 0.98 per layer."""
+    return [800] + [980] * (n_layers - 1)
 
 
 def retained_tokens(n_tok: int, counts, seed: int) -> list:
