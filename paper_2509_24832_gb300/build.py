@@ -16,7 +16,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "libsemshare.so")
-SOURCES = ["api.cu", "hash.cu", "match.cu", "match_tc.cu", "gather.cu", "deviation.cu", "fetch.cu"]
+SOURCES = ["api.cu", "hash.cu", "hash_2sm.cu", "match.cu", "match_tc.cu", "gather.cu", "deviation.cu", "fetch.cu"]
 # measurement support, linked into a library of its own so that libsemshare.so exports only the
 # entry points of include/semshare.h
 PROBE_SOURCES = ["probe.cu"]
@@ -25,7 +25,7 @@ ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 # -warn-spills: a register spill in a file with tensor-memory loads is a build error (below).  Those
 # kernels hand tcgen05.ld destination registers to later code before the load's wait; a spill placed
 # in between would store them before the data arrives.
-NO_SPILL = {"hash.cu", "match_tc.cu"}
+NO_SPILL = {"hash.cu", "hash_2sm.cu", "match_tc.cu"}
 NVCC_FLAGS = ARCH + ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2", "-Xptxas", "-warn-spills",
                      "-I", INCLUDE, "-I", CSRC]
 

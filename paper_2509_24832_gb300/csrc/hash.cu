@@ -45,11 +45,15 @@
 #include <cuda_bf16.h>
 
 #include "common.cuh"
+#include "hash_2sm.cuh"
+#include "hash_common.cuh"
 #include "ptx.cuh"
 #include "tma_host.cuh"
 
 namespace semshare {
 namespace {
+
+using namespace hashk;
 
 constexpr int kBM = 128;                       // rows per tile (MMA M, one TMEM lane per row)
 constexpr int kBK = 64;                        // K elements per stage: one 128-byte row of bf16
@@ -102,22 +106,6 @@ struct HashArgs {
     uint64_t wait_limit_ns;
 };
 
-// First iteration of CTA b's range (b = gridDim.x gives the end).
-__device__ __forceinline__ int64_t range_begin(int64_t b, int64_t total, int64_t G) { return (b * total) / G; }
-
-// The CTA whose range holds iteration i.
-__device__ __forceinline__ int64_t range_owner(int64_t i, int64_t total, int64_t G) {
-    int64_t b = (i * G) / total;
-    while (b + 1 < G && range_begin(b + 1, total, G) <= i) ++b;
-    while (b > 0 && range_begin(b, total, G) > i) --b;
-    return b;
-}
-
-// Rotation variants of the kernel, fixed at compile time so that the plain rotary kernel carries
-// no test for the others: every row rotated; no row rotated (SEMSHARE_ROPE_NONE); a pair call,
-// which hashes every row twice -- logical tiles below pair_rows as they are, the tiles from
-// pair_rows on (the same rows again) rotated.
-enum RotVariant { kRotAll = 0, kRotNone = 1, kRotPair = 2 };
 
 // First source row of logical tile `tile`, whether its rows are rotated, and where its codes go.
 template <int kRot>
@@ -132,28 +120,6 @@ __device__ __forceinline__ bool tile_rotates(const HashArgs& a, int64_t tile) {
 template <int kRot>
 __device__ __forceinline__ uint32_t* tile_codes(const HashArgs& a, int64_t tile) {
     return (kRot == kRotPair && tile * kBM >= a.pair_rows) ? a.codes2 : a.codes;
-}
-
-// cos and sin of the rotation angle m * theta_k (Eq. 1).  turns_q64 = frac(theta_k/(2*pi)) as
-// a 0.64 fixed-point fraction, so bits 32..63 of m * turns_q64 (mod 2^64) are the angle's
-// fraction of a full turn: the reduction modulo 2*pi is exact integer arithmetic for every
-// int32 position.  The fraction, centred on [-1/2, 1/2) and rounded to 23 bits, becomes a
-// float through the mantissa (a wrap from +1/2 to -1/2 is the same angle).
-__device__ __forceinline__ void rotation(uint32_t m, uint64_t turns_q64, float& c, float& s) {
-    const uint32_t lo = static_cast<uint32_t>(turns_q64);
-    const uint32_t hi = static_cast<uint32_t>(turns_q64 >> 32);
-    const uint32_t frac = __umulhi(m, lo) + m * hi;
-    const float t = __uint_as_float(0x3F800000u | ((frac + 0x80000100u) >> 9)) - 1.5f;
-    __sincosf(t * 6.28318530717958647692f, &s, &c);
-}
-
-// (x0, x1) turned counter-clockwise by the angle with cosine c and sine s, rounded to a bf16
-// pair (x0 in the low half, the lower address).
-__device__ __forceinline__ uint32_t rotate_to_bf16(float x0, float x1, float c, float s) {
-    const float y0 = fmaf(x0, c, -x1 * s);
-    const float y1 = fmaf(x0, s, x1 * c);
-    __nv_bfloat162 r = __floats2bfloat162_rn(y0, y1);
-    return *reinterpret_cast<uint32_t*>(&r);
 }
 
 // The K block holding the rotate-half partners of block kb's columns (d/2 = nkb/2 blocks away).
@@ -224,35 +190,6 @@ __device__ __forceinline__ void load_pairs4(const uint64_t* table, int half, int
     const ulonglong2 t01 = __ldg(tp), t23 = __ldg(tp + 1), c01 = __ldg(cp), c23 = __ldg(cp + 1);
     t.turns[0] = t01.x; t.turns[1] = t01.y; t.turns[2] = t23.x; t.turns[3] = t23.y;
     t.cis32[0] = c01.x; t.cis32[1] = c01.y; t.cis32[2] = c23.x; t.cis32[3] = c23.y;
-}
-
-// Sign bits of 32 fp32 values given as bit patterns: bit j = [v_j > 0].
-__device__ __forceinline__ uint32_t sign_word(const uint32_t (&v)[32]) {
-    uint32_t bits = 0u;
-#pragma unroll
-    for (int j = 0; j < 32; ++j) bits |= (static_cast<int32_t>(v[j]) > 0 ? 1u : 0u) << j;
-    return bits;
-}
-
-__device__ __forceinline__ void store_proj(float* proj, int64_t row, int nbits, int q, const uint32_t (&v)[32]) {
-    float4* pp = reinterpret_cast<float4*>(proj + row * nbits + q * 32);
-#pragma unroll
-    for (int j = 0; j < 8; ++j)
-        pp[j] = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]), __uint_as_float(v[4 * j + 2]),
-                            __uint_as_float(v[4 * j + 3]));
-}
-
-__device__ __forceinline__ void store_codes(uint32_t* codes, int64_t row, int W, const uint32_t (&words)[8]) {
-    uint32_t* cp = codes + row * W;
-    if ((W & 3) == 0) {
-#pragma unroll
-        for (int q = 0; q < 8; q += 4)
-            if (q < W) *reinterpret_cast<uint4*>(cp + q) = make_uint4(words[q], words[q + 1], words[q + 2], words[q + 3]);
-    } else {
-#pragma unroll
-        for (int q = 0; q < 8; ++q)
-            if (q < W) cp[q] = words[q];
-    }
 }
 
 template <bool kHalf, int kRot>
@@ -868,7 +805,9 @@ semshare_status plan_hash(int64_t n, int32_t d, HashPlan* p) {
     p->total_iters = p->n_tiles * (d / kBK);
     p->grid = static_cast<int>(p->total_iters < sms ? p->total_iters : sms);
     p->partial_bytes = static_cast<size_t>(2) * sms * kBM * static_cast<size_t>(kMaxBits) * 4;
-    p->count_bytes = ((static_cast<size_t>(p->n_tiles) * 4 + 255) / 256) * 256;
+    // counters of 128-row tiles (this kernel) or of the two halves of 256-row pair tiles
+    // (hash_2sm.cu): n_tiles + 4 words covers both, for single and pair calls
+    p->count_bytes = (((static_cast<size_t>(p->n_tiles) + 4) * 4 + 255) / 256) * 256;
     return SEMSHARE_OK;
 }
 
@@ -920,6 +859,31 @@ semshare_status hash_impl(const void* emb, semshare_dtype dtype, int64_t n, int3
     HashPlan plan;
     if (plan_hash(pair ? 2 * n_pad : n, d, &plan) != SEMSHARE_OK) return SEMSHARE_ECUDA;
     if (workspace_bytes < plan.partial_bytes + plan.count_bytes) return SEMSHARE_EINVAL;
+    if (dtype == SEMSHARE_BF16 && !half) {
+        // bf16 rows, interleaved pairing or none: the CTA-pair kernel (hash_2sm.cu)
+        Hash2smCall c{};
+        c.emb = emb;
+        c.n = n;
+        c.d = d;
+        c.row_stride = row_stride;
+        c.positions = none ? nullptr : positions;
+        c.rope_table = rope_table;
+        c.hyperplanes = hyperplanes;
+        c.nbits = nbits;
+        c.none = none;
+        c.pair = pair;
+        c.pair_rows = ((n + 255) / 256) * 256;
+        c.codes = codes;
+        c.codes2 = codes2;
+        c.proj = proj_out;
+        c.err_flag = err_flag;
+        c.partials = workspace;
+        c.partial_bytes = plan.partial_bytes;
+        c.tile_count = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(workspace) + plan.partial_bytes);
+        c.count_bytes = plan.count_bytes;
+        c.stream = stream;
+        return launch_hash_2sm(c);
+    }
     int dev = 0, smem_optin = 0;
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
