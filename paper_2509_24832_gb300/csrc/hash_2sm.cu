@@ -417,15 +417,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         int64_t cur_tile = -1;
         // The rotation table, a few tens of KB that every stage reads from, does not fit in the L1
         // left beside the pipeline's shared memory: the RoPE warps copy it into shared memory first.
-        const uint64_t* tbl = a.rope_table;
-        if (a.table_bytes != 0) {
+        const bool staged = a.table_bytes != 0;
+        const uint64_t* const tbl_sh = reinterpret_cast<const uint64_t*>(gbase + (table_s - sbase));
+        if (staged) {
             const uint4* src = reinterpret_cast<const uint4*>(a.rope_table);
             uint4* dst = reinterpret_cast<uint4*>(gbase + (table_s - sbase));
             for (uint32_t e = threadIdx.x - kRopeWarp0 * 32; e < a.table_bytes / 16; e += 4 * kRopeGroups * 32)
                 dst[e] = __ldg(src + e);
             asm volatile("bar.sync %0, %1;" ::"n"(kRopeBarrier), "n"(4 * kRopeGroups * 32) : "memory");
-            tbl = reinterpret_cast<const uint64_t*>(dst);
         }
+        // table words k, k+1 (k even), from shared memory when staged
+        auto table_pair = [&](int k) -> ulonglong2 {
+            return staged ? *reinterpret_cast<const ulonglong2*>(tbl_sh + k)
+                          : __ldg(reinterpret_cast<const ulonglong2*>(a.rope_table + k));
+        };
         // this thread's turn entries of a stage, pairs k, k+1 (k = kb*32 + 8c + 2*t4) for c < 4, are
         // fetched a stage ahead; their 32-step rotations are fetched when used
         ulonglong2 tturn[4];
@@ -435,7 +440,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 const int k = kb * (kBK / 2) + 8 * c + 2 * t4;
-                tturn[c] = *reinterpret_cast<const ulonglong2*>(tbl + k);
+                tturn[c] = table_pair(k);
             }
         };
         // stage q = g, g+2, ...: its tile and K block, and its slots and phase parities, kept
@@ -461,6 +466,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                                      : m[0] + 32u * j;
                     steps32 = steps32 && m[j] == m[0] + 32u * j;
                 }
+                // one path per warp: the branches below hold warp-wide tcgen05.st instructions, which
+                // all lanes must execute together (rows past n can make the pattern differ by lane)
+                steps32 = __all_sync(0xFFFFFFFFu, steps32);
             }
             const bool got = pair_wait(bar_afull + 8u * sa, pa, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns);
             if (!__all_sync(0xFFFFFFFFu, got)) break;
@@ -479,6 +487,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(bar_aempty + 8u * sa);
+            // the TMEM operand slot is free once the MMAs of the stage SB before have finished
+            const bool slot_free =
+                pair_wait(bar_done + 8u * sb, pb ^ 1u, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns);
+            if (!__all_sync(0xFFFFFFFFu, slot_free)) break;
+            tc_fence_after_sync();
+            const uint32_t tcol = tmem_base + kAccCols + sb * kAStageCols + lane_field;
             if ((kRot == kRotAll || rot) && steps32) {
                 // the usual case, one branch for the whole stage so that the four column groups'
                 // independent chains interleave: row j+1 sits 32 positions after row j, so only
@@ -489,8 +503,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ulonglong2 tstep[2];
 #pragma unroll
                     for (int cc = 0; cc < 2; ++cc)
-                        tstep[cc] = *reinterpret_cast<const ulonglong2*>(tbl + half + kb_table * (kBK / 2) +
-                                                                         8 * (ch + cc) + 2 * t4);
+                        tstep[cc] = table_pair(half + kb_table * (kBK / 2) + 8 * (ch + cc) + 2 * t4);
 #pragma unroll
                     for (int cc = 0; cc < 2; ++cc) {
                         rotation(m[0], tturn[ch + cc].x, cs[cc][0], sn[cc][0]);
@@ -516,8 +529,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                             }
                         }
                     }
+                    // these two column groups go to tensor memory while the next two are rotated
+#pragma unroll
+                    for (int h = 0; h < 2; ++h)
+#pragma unroll
+                        for (int cc = 0; cc < 2; ++cc)
+                            tmem_st_16x256b(tcol + ((16u * h) << 16) + 8u * (ch + cc), y[2 * h][ch + cc][0],
+                                            y[2 * h][ch + cc][1], y[2 * h + 1][ch + cc][0], y[2 * h + 1][ch + cc][1]);
                 }
-            } else if (kRot == kRotAll || rot) {
+            } else {
+                if (kRot == kRotAll || rot) {
                 // positions not 32 apart: every row's own angles
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
@@ -529,19 +550,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                         y[j][c][0] = rotate_to_bf16(bf16_lo(y[j][c][0]), bf16_hi(y[j][c][0]), cs0, sn0);
                         y[j][c][1] = rotate_to_bf16(bf16_lo(y[j][c][1]), bf16_hi(y[j][c][1]), cs1, sn1);
                     }
-            }  // rows hashed as they are: the bf16 pairs already are the MMA operand
-            // the TMEM operand slot is free once the MMAs of the stage SB before have finished
-            const bool slot_free =
-                pair_wait(bar_done + 8u * sb, pb ^ 1u, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns);
-            if (!__all_sync(0xFFFFFFFFu, slot_free)) break;
-            tc_fence_after_sync();
-            const uint32_t tcol = tmem_base + kAccCols + sb * kAStageCols + lane_field;
+                }  // rows hashed as they are: the bf16 pairs already are the MMA operand
 #pragma unroll
-            for (int h = 0; h < 2; ++h)
+                for (int h = 0; h < 2; ++h)
 #pragma unroll
-                for (int c = 0; c < 4; ++c)
-                    tmem_st_16x256b(tcol + ((16u * h) << 16) + 8u * c, y[2 * h][c][0], y[2 * h][c][1],
-                                    y[2 * h + 1][c][0], y[2 * h + 1][c][1]);
+                    for (int c = 0; c < 4; ++c)
+                        tmem_st_16x256b(tcol + ((16u * h) << 16) + 8u * c, y[2 * h][c][0], y[2 * h][c][1],
+                                        y[2 * h + 1][c][0], y[2 * h + 1][c][1]);
+            }
             tmem_st_wait();
             // this CTA's hyperplane half of the stage must have landed before the MMA reads it
             const bool b_in = pair_wait(bar_bfull + 8u * sb, pb, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns);
