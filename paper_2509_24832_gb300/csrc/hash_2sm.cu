@@ -61,6 +61,7 @@ constexpr int kPM = 256;                    // rows of a pair tile: M of one cta
 constexpr int kCM = 128;                    // rows of each CTA's half, one TMEM lane each
 constexpr int kBK = 64;                     // K elements per stage: one 128-byte row of bf16
 constexpr int kUmmaK = 16;                  // K of one tcgen05.mma kind::f16
+static_assert(kBK / kUmmaK == 4, "the MMA loop issues four instructions per stage");
 constexpr int kRopeWarp0 = 4;
 constexpr int kRopeGroups = 2;              // groups of four warps (one per TMEM lane quadrant)
 constexpr int kEpiWarp0 = kRopeWarp0 + 4 * kRopeGroups;
@@ -363,36 +364,45 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp == 1) {
         // ---------------- MMA issuer (even CTA) ----------------
         if (leader && lane == 0) {
+            // Slot addresses and descriptors advance by constant strides and wrap with the ring.
             const uint32_t idesc = umma_idesc_bf16_f32(kPM, a.nbits);
-            uint32_t q = 0, acc = 0;
+            const uint64_t bdesc0 = sw128_kmajor_desc(b_ring);
+            const uint64_t bstride = a.bh_bytes >> 4;  // descriptor start address is in 16-byte units
+            uint64_t bd = bdesc0;
+            uint32_t a_tmem = tmem_base + kAccCols, bar_s = 0, s = 0, ph = 0, acc = 0;
             bool seg_first = true;
             int kb = static_cast<int>(i0 % nkb);
-            uint32_t s = 0, ph = 0;
-            for (int64_t it = i0; it < i1; ++it, ++q) {
+            for (int64_t it = i0; it < i1; ++it) {
                 if (seg_first) {
                     if (!pair_wait(bar_accempty, (acc & 1u) ^ 1u, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns))
                         break;
                     tc_fence_after_sync();
                 }
-                if (!pair_wait(bar_ready + 8u * s, ph, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns)) break;
+                if (!pair_wait(bar_ready + bar_s, ph, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns)) break;
                 tc_fence_after_sync();
-                const uint32_t bst = b_ring + s * a.bh_bytes;
-                const uint32_t a_tmem = tmem_base + kAccCols + s * kAStageCols;
-#pragma unroll
-                for (int k = 0; k < kBK / kUmmaK; ++k)
-                    umma_bf16_ts_pair(tmem_base, a_tmem + k * (kUmmaK / 2), sw128_kmajor_desc(bst + k * kUmmaK * 2),
-                                      idesc, (seg_first && k == 0) ? 0u : 1u);
-                umma_commit_pair_multicast(bar_done + 8u * s, 0x3);
-                const bool seg_last = (kb == nkb - 1) || (it == i1 - 1);
+                // K = 16 per instruction: 8 TMEM columns of A, 32 bytes (2 descriptor units) of B
+                umma_bf16_ts_pair(tmem_base, a_tmem, bd, idesc, seg_first ? 0u : 1u);
+                umma_bf16_ts_pair(tmem_base, a_tmem + 8, bd + 2, idesc, 1u);
+                umma_bf16_ts_pair(tmem_base, a_tmem + 16, bd + 4, idesc, 1u);
+                umma_bf16_ts_pair(tmem_base, a_tmem + 24, bd + 6, idesc, 1u);
+                umma_commit_pair_multicast(bar_done + bar_s, 0x3);
+                const bool seg_last = (++kb == nkb) || (it == i1 - 1);
+                if (kb == nkb) kb = 0;
                 if (seg_last) {
                     umma_commit_pair_multicast(bar_accfull, 0x3);
                     ++acc;
                 }
                 seg_first = seg_last;
-                if (++kb == nkb) kb = 0;
                 if (++s == SB) {
                     s = 0;
                     ph ^= 1u;
+                    bd = bdesc0;
+                    a_tmem = tmem_base + kAccCols;
+                    bar_s = 0;
+                } else {
+                    bd += bstride;
+                    a_tmem += kAStageCols;
+                    bar_s += 8u;
                 }
             }
             // every MMA issued above has finished once this arrives: TMEM may then be freed
