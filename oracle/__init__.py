@@ -58,6 +58,8 @@ def _load():
         P = ctypes.c_void_p
         i32, i64, f64 = ctypes.c_int32, ctypes.c_int64, ctypes.c_double
         lib.oracle_num_threads.restype = ctypes.c_int
+        lib.oracle_set_threads.argtypes = [ctypes.c_int]
+        lib.oracle_set_threads.restype = ctypes.c_int
         lib.oracle_bf16_value.argtypes = [ctypes.c_uint16]
         lib.oracle_bf16_value.restype = f64
         lib.oracle_bf16_round.argtypes = [f64]
@@ -91,6 +93,12 @@ def _ptr(a: np.ndarray | None):
 def num_threads() -> int:
     """OpenMP threads the oracle uses (OMP_NUM_THREADS, else all cores)."""
     return int(_load().oracle_num_threads())
+
+
+def set_threads(n: int) -> int:
+    """Sets the OpenMP threads of the oracle's later calls; returns the previous count (timing only:
+    the results do not depend on it)."""
+    return int(_load().oracle_set_threads(int(n)))
 
 
 def bf16_round(v: float) -> int:

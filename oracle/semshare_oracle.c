@@ -57,6 +57,19 @@ int oracle_num_threads(void) {
 #endif
 }
 
+/* Threads of the following calls' parallel loops (n >= 1); returns the previous setting.  Only
+ * the timing of the CPU baseline uses it: results do not depend on the thread count. */
+int oracle_set_threads(int n) {
+#ifdef _OPENMP
+    const int prev = omp_get_max_threads();
+    if (n >= 1) omp_set_num_threads(n);
+    return prev;
+#else
+    (void)n;
+    return 1;
+#endif
+}
+
 /* ---- bf16 <-> fp64 --------------------------------------------------------------------- */
 
 /* Value of a bf16 bit pattern (exact). */

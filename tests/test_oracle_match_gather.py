@@ -182,3 +182,18 @@ def test_gather_out_of_range_rows_untouched(oracle_mod):
     assert bad == 2
     assert (ok[0, 0, 0, 0] == 1).all() and (ok[0, 0, 0, 1:] == 7).all()
     assert (ov[0, 0, 0, 0] == 2).all() and (ov[0, 0, 0, 1:] == 9).all()
+
+
+def test_thread_count_does_not_change_results(oracle_mod):
+    """The CPU baseline times the oracle on one thread and on all cores: same results either way."""
+    g = np.random.default_rng(8)
+    t = g.integers(0, 2**32, size=(300, 4), dtype=np.uint64).astype(np.uint32)
+    r = g.integers(0, 2**32, size=(257, 4), dtype=np.uint64).astype(np.uint32)
+    prev = oracle_mod.set_threads(1)
+    try:
+        a = oracle_mod.match(t, r)
+    finally:
+        oracle_mod.set_threads(prev)
+    b = oracle_mod.match(t, r)
+    np.testing.assert_array_equal(a[0], b[0])
+    np.testing.assert_array_equal(a[1], b[1])
