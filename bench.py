@@ -54,7 +54,7 @@ L2_FLUSH_BYTES = 512 << 20
 NCU_TRAFFIC = {
     ("gather", "llama8b-5k"): {"file": "gather.cu", "sha": "8b2db284dbc5f706", "bytes_per_launch": 1079.6e6},
     ("gather_retained", "llama8b-5k"): {"file": "gather.cu", "sha": "8b2db284dbc5f706", "bytes_per_launch": 661.7e6},
-    ("hash", "llama8b-5k"): {"file": "hash.cu", "sha": "62eac1232305cc7e", "bytes_per_launch": 89.46e6},
+    ("hash", "llama8b-5k"): {"file": "hash_2sm.cu", "sha": "a9e3f433112cf4b6", "bytes_per_launch": 86.84e6},
     ("match_tc", "llama8b-5k"): {"file": "match_tc.cu", "sha": "06cdd7c30d30cf11", "bytes_per_launch": 2.717e6},
     ("retrieve", "retrieve-16x4096"): {"file": "match_tc.cu", "sha": "06cdd7c30d30cf11", "bytes_per_launch": 18.41e6},
 }
