@@ -227,6 +227,32 @@ def test_match_tc_ties_and_all_equal(ss):
     assert int(idx2.max()) == 0
 
 
+def test_match_tc_workspace_reused_across_shapes(ss, orc):
+    """One workspace, sized for the largest call and left dirty by each, serves calls of different
+    shapes in turn: many target blocks and few reference blocks, one target block against many
+    reference blocks, ragged last blocks, codes narrower than one 128-bit chunk.  Each result
+    equals the xor/popc search (and the oracle where that is quick)."""
+    shapes = [(40000, 600, 256), (50, 70000, 256), (3001, 2999, 128), (129, 257, 64), (40000, 600, 256)]
+    need = max(ss.semshare_match_tc_workspace_size(t, r, b) for t, r, b in shapes)
+    ws = torch.full((need,), 0x5A, dtype=torch.uint8, device="cuda")
+    for i, (n_tgt, n_ref, nbits) in enumerate(shapes):
+        ref = workloads.random_codes(n_ref, nbits, seed=90 + i, stream=3)
+        tgt = workloads.random_codes(n_tgt, nbits, seed=90 + i, stream=4)
+        tgt[: n_tgt // 4] = ref[np.arange(n_tgt // 4) % n_ref]
+        ti = torch.from_numpy(tgt.view(np.int32)).cuda()
+        ri = torch.from_numpy(ref.view(np.int32)).cuda()
+        flag = ss.new_err_flag()
+        idx, dist = ss.semshare_match_tc(ti, ri, workspace=ws, err_flag=flag)
+        pi, pd = ss.semshare_match(ti, ri)
+        torch.cuda.synchronize()
+        ss.check_flag(flag, "match_tc")
+        assert torch.equal(idx, pi) and torch.equal(dist, pd), (n_tgt, n_ref, nbits)
+        if n_tgt * n_ref <= 10 ** 7:
+            oi, od = orc.match(tgt, ref)
+            np.testing.assert_array_equal(idx.cpu().numpy(), oi)
+            np.testing.assert_array_equal(dist.cpu().numpy(), od)
+
+
 def test_match_identity_ties_and_determinism(ss):
     c = torch.randint(-2 ** 31, 2 ** 31 - 1, (4000, 8), dtype=torch.int32, device="cuda")
     c[3999] = c[5]
