@@ -55,7 +55,8 @@ typedef enum {
     SEMSHARE_ECUDA = 3,         /* a CUDA runtime or driver call failed */
     SEMSHARE_EINDEX = 4,        /* a kernel met an index outside its table (from err_flag) */
     SEMSHARE_ETIMEOUT = 5,      /* a kernel pipeline wait hit its time limit (from err_flag) */
-    SEMSHARE_ETOOLARGE = 6      /* a size exceeds semshare_match_static's fixed scratch capacity */
+    SEMSHARE_ETOOLARGE = 6,     /* a size exceeds semshare_match_static's fixed scratch capacity */
+    SEMSHARE_ECHECK = 7         /* checked build: a pipeline bookkeeping check failed (from err_flag) */
 } semshare_status;
 
 typedef enum { SEMSHARE_BF16 = 0, SEMSHARE_F32 = 1 } semshare_dtype;
@@ -63,12 +64,43 @@ typedef enum { SEMSHARE_BF16 = 0, SEMSHARE_F32 = 1 } semshare_dtype;
 /* Bits a kernel ORs into `err_flag`. */
 #define SEMSHARE_FLAG_INDEX 1u
 #define SEMSHARE_FLAG_TIMEOUT 2u
+/* Checked build only (see semshare_checked_build): a bookkeeping check failed.  The first failed
+ * check also stores its kernel id in bits 8..15 of err_flag and its source line in bits 16..31. */
+#define SEMSHARE_FLAG_CHECK 4u
+#define SEMSHARE_CHECK_KERNEL(flags) (((flags) >> 8) & 0xFFu)
+#define SEMSHARE_CHECK_LINE(flags) ((flags) >> 16)
+/* Kernel ids of SEMSHARE_CHECK_KERNEL. */
+#define SEMSHARE_KERNEL_HASH_2SM 1u      /* bf16 rows on SM pairs (hash_2sm.cu) */
+#define SEMSHARE_KERNEL_HASH 2u          /* fp32 rows, rotate-half (hash.cu) */
+#define SEMSHARE_KERNEL_HAMMING_TC 3u    /* tensor-core search (match_tc.cu) */
+#define SEMSHARE_KERNEL_SELFTEST 15u     /* semshare_check_selftest */
 
 /* Human-readable name of a status. */
 const char* semshare_status_string(semshare_status s);
 
-/* Maps the err_flag bits read back by the caller to a status (TIMEOUT wins over INDEX). */
+/* Maps the err_flag bits read back by the caller to a status (TIMEOUT wins over CHECK, CHECK over
+ * INDEX). */
 semshare_status semshare_flag_status(uint32_t flags);
+
+/*
+ * The checked build: the same library compiled with -DSEMSHARE_CHECKED (libsemshare_checked.so,
+ * built beside libsemshare.so; a stand-in for a race/synchronisation sanitizer, which this
+ * project does not rely on).  Its pipelined kernels also verify their barrier bookkeeping while
+ * they run: every ring slot a consumer acquires was filled exactly once since its last use and
+ * every slot a producer refills was released by all of its consumers; at the end every role has
+ * handled as many stages and segments as its range implies; the tensor-memory allocation starts
+ * at column 0; every stream-K tile is closed after exactly its expected number of arrivals.  A
+ * failed check ORs SEMSHARE_FLAG_CHECK into err_flag (when err_flag is non-NULL) and the kernel
+ * carries on; results are the same as the plain build's.  This is not part of the paper; it
+ * exists to test the library.
+ *
+ * semshare_checked_build: 1 in the checked build, 0 in the plain one.
+ * semshare_check_selftest: checked build only (SEMSHARE_EUNSUPPORTED otherwise): enqueues a
+ * one-thread kernel whose check fails on purpose, so that a caller can confirm how failures
+ * reach err_flag (kernel id SEMSHARE_KERNEL_SELFTEST).  err_flag: device, 4-byte aligned.
+ */
+int32_t semshare_checked_build(void);
+semshare_status semshare_check_selftest(uint32_t* err_flag, void* stream);
 
 /* SEMSHARE_ABI_VERSION of the loaded library. */
 int32_t semshare_abi_version(void);

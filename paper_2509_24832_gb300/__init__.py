@@ -11,9 +11,15 @@ Insight 1).
 The compute lives in libsemshare.so (C ABI: include/semshare.h); this package is its thin
 ctypes binding with the same names.  Build the library with `paper_2509_24832_gb300.build`."""
 from ._native import (  # noqa: F401
+    CHECKED,
+    FLAG_CHECK,
     FLAG_INDEX,
     HD_PERCENT,
     FLAG_TIMEOUT,
+    KERNEL_HAMMING_TC,
+    KERNEL_HASH,
+    KERNEL_HASH_2SM,
+    KERNEL_SELFTEST,
     KVLayout,
     LIB_PATH,
     Prepared,
@@ -33,6 +39,9 @@ from ._native import (  # noqa: F401
     new_err_flag,
     retain_counts,
     semshare_abi_version,
+    semshare_check_selftest,
+    semshare_checked_build,
+    check_record,
     semshare_fetch_rows,
     semshare_fetch_workspace_size,
     semshare_gather_kv,

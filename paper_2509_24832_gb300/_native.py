@@ -13,11 +13,15 @@ from typing import NamedTuple
 import torch
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_PKG, "_lib", "libsemshare.so")
+# SEMSHARE_CHECKED=1 in the environment (read once, at import) selects the checked build, whose
+# kernels also verify their pipeline bookkeeping (semshare_checked_build in include/semshare.h)
+CHECKED = os.environ.get("SEMSHARE_CHECKED", "") not in ("", "0")
+LIB_PATH = os.path.join(_PKG, "_lib", "libsemshare_checked.so" if CHECKED else "libsemshare.so")
 
-OK, EINVAL, EUNSUPPORTED, ECUDA, EINDEX, ETIMEOUT, ETOOLARGE = range(7)
+OK, EINVAL, EUNSUPPORTED, ECUDA, EINDEX, ETIMEOUT, ETOOLARGE, ECHECK = range(8)
 MATCH_STATIC_MAX_TARGETS = 262144
-FLAG_INDEX, FLAG_TIMEOUT = 1, 2
+FLAG_INDEX, FLAG_TIMEOUT, FLAG_CHECK = 1, 2, 4
+KERNEL_HASH_2SM, KERNEL_HASH, KERNEL_HAMMING_TC, KERNEL_SELFTEST = 1, 2, 3, 15
 BF16, F32 = 0, 1
 ROPE_LAYOUTS = {"interleaved": 0, "half": 1, "none": 2}
 
@@ -57,6 +61,9 @@ def load():
         lib.semshare_flag_status.argtypes = [u32]
         lib.semshare_flag_status.restype = ctypes.c_int
         lib.semshare_abi_version.restype = i32
+        lib.semshare_checked_build.restype = i32
+        lib.semshare_check_selftest.argtypes = [P, P]
+        lib.semshare_check_selftest.restype = ctypes.c_int
         lib.semshare_rope_table.argtypes = [i32, ctypes.c_double, P, P]
         lib.semshare_rope_table.restype = ctypes.c_int
         lib.semshare_hash_pair_workspace_size.argtypes = [i64, i32, i32]
@@ -182,6 +189,23 @@ def check_flag(err_flag: torch.Tensor, where: str = "kernel"):
 
 def semshare_abi_version() -> int:
     return int(load().semshare_abi_version())
+
+
+def semshare_checked_build() -> bool:
+    """True when the loaded library is the checked build."""
+    return bool(load().semshare_checked_build())
+
+
+def semshare_check_selftest(err_flag: torch.Tensor, stream=None) -> None:
+    """Checked build: enqueue a kernel whose check fails on purpose (see include/semshare.h)."""
+    _need_cuda(err_flag, "err_flag")
+    _check(load().semshare_check_selftest(_ptr(err_flag), _stream(stream)), "semshare_check_selftest")
+
+
+def check_record(err_flag_value: int) -> tuple[int, int]:
+    """(kernel id, source line) of the first failed check packed into an err_flag word."""
+    v = int(err_flag_value) & 0xFFFFFFFF
+    return (v >> 8) & 0xFF, v >> 16
 
 
 def semshare_rope_table(d: int, rope_base: float = 10000.0, out: torch.Tensor | None = None, device=None,

@@ -21,6 +21,8 @@ SOURCES = ["api.cu", "hash.cu", "hash_2sm.cu", "match.cu", "match_tc.cu", "gathe
 # entry points of include/semshare.h
 PROBE_SOURCES = ["probe.cu"]
 PROBE_LIB = os.path.join(LIBDIR, "libsemshare_probe.so")
+# the same sources with -DSEMSHARE_CHECKED: kernels that also verify their pipeline bookkeeping
+CHECKED_LIB = os.path.join(LIBDIR, "libsemshare_checked.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 # -warn-spills: a register spill in a file with tensor-memory loads is a build error (below).  Those
 # kernels hand tcgen05.ld destination registers to later code before the load's wait; a spill placed
@@ -43,26 +45,30 @@ def _inputs():
 
 
 def up_to_date() -> bool:
-    if not os.path.exists(LIB) or not os.path.exists(PROBE_LIB):
+    if not all(os.path.exists(p) for p in (LIB, PROBE_LIB, CHECKED_LIB)):
         return False
-    t = min(os.path.getmtime(LIB), os.path.getmtime(PROBE_LIB))
+    t = min(os.path.getmtime(p) for p in (LIB, PROBE_LIB, CHECKED_LIB))
     return all(os.path.getmtime(p) <= t for p in _inputs())
 
 
 def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | None = None) -> str:
-    """Compile and link libsemshare.so (and the measurement probe library libsemshare_probe.so);
-    returns the path of libsemshare.so.  No-op when up to date."""
+    """Compile and link libsemshare.so, the measurement probe library libsemshare_probe.so and the
+    checked build libsemshare_checked.so; returns the path of libsemshare.so.  No-op when up to
+    date."""
     if not force and not extra_flags and up_to_date():
         return LIB
     os.makedirs(os.path.join(LIBDIR, "obj"), exist_ok=True)
+    os.makedirs(os.path.join(LIBDIR, "obj_checked"), exist_ok=True)
     cc = nvcc()
     flags = NVCC_FLAGS + list(extra_flags or [])
     procs = []
     objs = []
-    for src in SOURCES + PROBE_SOURCES:
-        obj = os.path.join(LIBDIR, "obj", src.replace(".cu", ".o"))
+    jobs = [(src, "obj", []) for src in SOURCES + PROBE_SOURCES] + \
+        [(src, "obj_checked", ["-DSEMSHARE_CHECKED"]) for src in SOURCES]
+    for src, sub, defs in jobs:
+        obj = os.path.join(LIBDIR, sub, src.replace(".cu", ".o"))
         objs.append(obj)
-        cmd = [cc, *flags, "-c", os.path.join(CSRC, src), "-o", obj]
+        cmd = [cc, *flags, *defs, "-c", os.path.join(CSRC, src), "-o", obj]
         if verbose:
             print(" ".join(cmd), file=sys.stderr)
         procs.append((src, subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.STDOUT, text=True)))
@@ -76,8 +82,8 @@ def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | N
             failed.append(src)
     if failed:
         raise RuntimeError(f"nvcc failed (or spilled registers) on {failed}")
-    n = len(SOURCES)
-    for lib, parts in ((LIB, objs[:n]), (PROBE_LIB, objs[n:])):
+    n, m = len(SOURCES), len(SOURCES) + len(PROBE_SOURCES)
+    for lib, parts in ((LIB, objs[:n]), (PROBE_LIB, objs[n:m]), (CHECKED_LIB, objs[m:])):
         tmp = lib + f".tmp{os.getpid()}"
         subprocess.run([cc, *ARCH, "-shared", "-Xcompiler", "-fPIC", *parts, "-o", tmp], check=True)
         os.replace(tmp, lib)

@@ -24,6 +24,12 @@ __global__ void rope_table_kernel(int32_t d, double base, uint64_t* __restrict__
     table[d / 2 + k] = static_cast<uint64_t>(__float_as_uint(c)) | (static_cast<uint64_t>(__float_as_uint(s)) << 32);
 }
 
+// A check that fails on purpose (checked build): confirms how failures reach err_flag.
+__global__ void check_selftest_kernel(uint32_t* err) {
+    pdl_prologue();
+    if (threadIdx.x == 0) SEMSHARE_CHECK(false, err, SEMSHARE_KERNEL_SELFTEST);
+}
+
 }  // namespace
 }  // namespace semshare
 
@@ -36,14 +42,27 @@ extern "C" const char* semshare_status_string(semshare_status s) {
         case SEMSHARE_EINDEX: return "index out of range";
         case SEMSHARE_ETIMEOUT: return "kernel wait timed out";
         case SEMSHARE_ETOOLARGE: return "size exceeds the fixed scratch capacity";
+        case SEMSHARE_ECHECK: return "checked build: a pipeline bookkeeping check failed";
     }
     return "unknown status";
 }
 
 extern "C" semshare_status semshare_flag_status(uint32_t flags) {
     if (flags & SEMSHARE_FLAG_TIMEOUT) return SEMSHARE_ETIMEOUT;
+    if (flags & SEMSHARE_FLAG_CHECK) return SEMSHARE_ECHECK;
     if (flags & SEMSHARE_FLAG_INDEX) return SEMSHARE_EINDEX;
     return SEMSHARE_OK;
+}
+
+extern "C" int32_t semshare_checked_build(void) { return semshare::kChecked ? 1 : 0; }
+
+extern "C" semshare_status semshare_check_selftest(uint32_t* err_flag, void* stream) {
+    using namespace semshare;
+    if (!kChecked) return SEMSHARE_EUNSUPPORTED;
+    if (err_flag == nullptr || !aligned(err_flag, 4)) return SEMSHARE_EINVAL;
+    if (launch_pdl(check_selftest_kernel, dim3(1), dim3(32), 0, as_stream(stream), err_flag) != cudaSuccess)
+        return SEMSHARE_ECUDA;
+    return launch_status();
 }
 
 extern "C" int32_t semshare_abi_version(void) { return SEMSHARE_ABI_VERSION; }

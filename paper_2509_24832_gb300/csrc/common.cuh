@@ -63,6 +63,32 @@ inline semshare_status launch_status() {
     return cudaGetLastError() == cudaSuccess ? SEMSHARE_OK : SEMSHARE_ECUDA;
 }
 
+// ---- the checked build (-DSEMSHARE_CHECKED) ----
+// SEMSHARE_CHECK(cond, err, kernel): in the checked build, a false cond ORs SEMSHARE_FLAG_CHECK into
+// *err and, if no check has failed before, stores the kernel id (bits 8..15) and the source line
+// (bits 16..31); the kernel carries on.  In the plain build it compiles to nothing (cond is not
+// evaluated).
+#ifdef SEMSHARE_CHECKED
+constexpr bool kChecked = true;
+__device__ __forceinline__ void check_fail(uint32_t* err, uint32_t kernel, uint32_t line) {
+    if (err == nullptr) return;
+    const uint32_t old = atomicOr(err, SEMSHARE_FLAG_CHECK);
+    if ((old >> 8) == 0u) {
+        const uint32_t base = old | SEMSHARE_FLAG_CHECK;
+        atomicCAS(err, base, base | (kernel << 8) | (line << 16));
+    }
+}
+#define SEMSHARE_CHECK(cond, err, kernel)                                   \
+    do {                                                                    \
+        if (!(cond)) ::semshare::check_fail((err), (kernel), __LINE__);     \
+    } while (0)
+#else
+constexpr bool kChecked = false;
+#define SEMSHARE_CHECK(cond, err, kernel) \
+    do {                                  \
+    } while (0)
+#endif
+
 // Limit of every bounded pipeline wait inside a kernel (the host never sees a longer stall).
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 

@@ -79,7 +79,8 @@ static_assert(kEpiWarp0 % 4 == 0, "epilogue warps must start on a warpgroup");
 constexpr uint32_t kABytes = kBM * kBK * 2;    // bf16 operand tile, 16 KB
 constexpr uint32_t kF32Bytes = kBM * kBK * 4;  // fp32 staging: two 128-byte-wide boxes, 32 KB
 constexpr int kEpiBarrier = 1;                 // named barrier of the epilogue warps
-constexpr size_t kFixedSmem = 1024 + 512;      // alignment slack + barriers + TMEM slot + flags
+// alignment slack + barriers + TMEM slot + flags (+ the checked build's counters)
+constexpr size_t kFixedSmem = 1024 + 512 + (kChecked ? 256 : 0);
 
 struct HashArgs {
     int64_t n;
@@ -215,6 +216,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     // hand-off bookkeeping shared with the end phase: [0] final partial staged (0/1), [1] its tile,
     // [2] its slot, [3] b_lo, [4] b_hi, [5] fix-ups pending, [6 + 3f ..] tile, b_lo, b_hi of fix-up f
     volatile int64_t* const ctl = reinterpret_cast<volatile int64_t*>(gbase + (tmem_slot + 16u - sbase));
+    // checked build: fills [0, 8) and rotations [8, 16) per ring slot, producer stages [16], MMA
+    // stages [17], epilogue segments [18]
+    volatile uint32_t* const chk = reinterpret_cast<volatile uint32_t*>(gbase + (bars + 512u - sbase));
+    constexpr uint32_t kRopeArrivals = kHalf ? kRopeWarps : kRopeWarps / kRopeGroups;  // per stage
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -237,6 +242,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         *abort_flag = 0;
         ctl[0] = 0;
         ctl[5] = 0;
+        if (kChecked)
+            for (int i = 0; i < 32; ++i) chk[i] = 0u;
         fence_barrier_init();
     }
     if (warp == 0 && lane == 0) {
@@ -251,6 +258,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after_sync();
     const uint32_t tmem_base = *tmem_slot_ptr;
+    if (threadIdx.x == 0) SEMSHARE_CHECK(tmem_base == 0u, a.err_flag, SEMSHARE_KERNEL_HASH);  // lane 0, column 0
 
     if (warp == 0) {
         // ---------------- TMA producer ----------------
@@ -280,6 +288,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ok = false;
                     break;
                 }
+                if (kChecked) {
+                    // every earlier fill of the slot was rotated by all its warps
+                    SEMSHARE_CHECK(chk[8 + s] == kRopeArrivals * (q / S), a.err_flag, SEMSHARE_KERNEL_HASH);
+                    chk[s] = chk[s] + 1u;
+                }
                 const uint32_t st = sbase + s * a.stage_bytes;
                 const uint32_t full = bar_full + 8u * s;
                 mbar_arrive_expect_tx(full, a.tx_bytes);
@@ -299,6 +312,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ++tile;
                 }
             }
+            if (kChecked && ok) chk[16] = q;
             if (!ok) {
                 // the last issue of every stage may still be landing: wait for it before exit
                 for (uint32_t i = (q > S ? q - S : 0); i < q; ++i)
@@ -326,6 +340,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!mbar_wait_bounded(bar_ready + 8u * s, ph, abort_flag, a.err_flag, SEMSHARE_FLAG_TIMEOUT,
                                        a.wait_limit_ns))
                     break;
+                // the operand tile is this stage's: all its warps have rotated this fill of the slot
+                SEMSHARE_CHECK(chk[8 + s] == kRopeArrivals * (q / S + 1u) && chk[s] == q / S + 1u, a.err_flag, SEMSHARE_KERNEL_HASH);
                 tc_fence_after_sync();
                 const uint32_t st = sbase + s * a.stage_bytes;
 #pragma unroll
@@ -343,6 +359,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 seg_first = seg_last;
                 if (++kb == nkb) kb = 0;
             }
+            if (kChecked) chk[17] = q;
             // every MMA issued above has finished once this arrives: TMEM may then be freed
             umma_commit(bar_mma_done);
             drain_wait(bar_mma_done, 0, kWaitLimitNs);
@@ -388,6 +405,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const bool got = mbar_wait_bounded(bar_full + 8u * s, ph, abort_flag, a.err_flag, SEMSHARE_FLAG_TIMEOUT,
                                                a.wait_limit_ns);
             if (!__all_sync(0xFFFFFFFFu, got)) break;
+            if (kChecked && lane == 0) SEMSHARE_CHECK(chk[s] == q / S + 1u, a.err_flag, SEMSHARE_KERNEL_HASH);  // this stage's fill
             uint8_t* const st = gbase + s * a.stage_bytes;
             const uint8_t* const pt = st + kABytes + a.b_bytes;  // partner block
             float cs[8], sn[8];
@@ -429,7 +447,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) mbar_arrive(bar_ready + 8u * s);
+            if (lane == 0) {
+                    if (kChecked) atomicAdd(const_cast<uint32_t*>(chk + 8 + s), 1u);
+                    mbar_arrive(bar_ready + 8u * s);
+                }
             kb = kb_next;
             if (kb == 0) ++tile;
         }
@@ -483,6 +504,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const bool got = mbar_wait_bounded(bar_full + 8u * s, ph, abort_flag, a.err_flag, SEMSHARE_FLAG_TIMEOUT,
                                                a.wait_limit_ns);
             if (!__all_sync(0xFFFFFFFFu, got)) break;
+            if (kChecked && lane == 0) SEMSHARE_CHECK(chk[s] == q / S + 1u, a.err_flag, SEMSHARE_KERNEL_HASH);  // this stage's fill
             uint8_t* const st = gbase + s * a.stage_bytes;
             if (kRot != kRotAll && !rot) {
                 // rows hashed as they are: bf16 rows already are the MMA operand; fp32 rows are only
@@ -513,7 +535,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     fence_proxy_async_smem();
                 }
                 __syncwarp();
-                if (lane == 0) mbar_arrive(bar_ready + 8u * s);
+                if (lane == 0) {
+                    if (kChecked) atomicAdd(const_cast<uint32_t*>(chk + 8 + s), 1u);
+                    mbar_arrive(bar_ready + 8u * s);
+                }
                 // a pair call's range may go on into rotated tiles: this group's next stage needs its
                 // table entries whichever kind of tile this one was
                 if (kRot == kRotPair && it + kRopeGroups < i1) {
@@ -589,7 +614,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) mbar_arrive(bar_ready + 8u * s);
+            if (lane == 0) {
+                    if (kChecked) atomicAdd(const_cast<uint32_t*>(chk + 8 + s), 1u);
+                    mbar_arrive(bar_ready + 8u * s);
+                }
             // this group's next stage: its table entries load while the other groups work
             if (it + kRopeGroups < i1 && kRot != kRotNone) {
                 const int kb = static_cast<int>((it + kRopeGroups) % nkb);
@@ -620,6 +648,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const bool got = mbar_wait_bounded(bar_accfull + 8u * buf, aph, abort_flag, a.err_flag,
                                                SEMSHARE_FLAG_TIMEOUT, a.wait_limit_ns);
             if (!epilogue_all(got)) break;
+            if (kChecked && threadIdx.x == kEpiWarp0 * 32) chk[18] = chk[18] + 1u;
             tc_fence_after_sync();
             const int64_t row = tile_src_row<kRot>(a, tile) + r;
             uint32_t* const out_codes = tile_codes<kRot>(a, tile);
@@ -688,6 +717,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     tc_fence_before_sync();
     __syncthreads();
+    if (kChecked && threadIdx.x == 0 && *abort_flag == 0) {
+        // every role handled the whole range: i1 - i0 stages, one accumulator per K-block segment
+        const uint32_t stages = static_cast<uint32_t>(i1 - i0);
+        const uint32_t segs = i1 > i0 ? static_cast<uint32_t>((i1 - 1) / nkb - i0 / nkb + 1) : 0u;
+        uint32_t rotated = 0;
+        for (uint32_t q = 0; q < S; ++q) rotated += chk[8 + q];
+        SEMSHARE_CHECK(chk[16] == stages && chk[17] == stages, a.err_flag, SEMSHARE_KERNEL_HASH);
+        SEMSHARE_CHECK(rotated == kRopeArrivals * stages, a.err_flag, SEMSHARE_KERNEL_HASH);
+        SEMSHARE_CHECK(chk[18] == segs, a.err_flag, SEMSHARE_KERNEL_HASH);
+    }
 
     // ---------------- end phase: publish the final partial, finish the tiles this CTA closes ----
     if (*abort_flag == 0) {

@@ -244,6 +244,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     // main loop: [0] 0 none, 1 publish this half's partial, 2 close the half; [1] pair tile,
     // [2] b_lo, [3] b_hi
     volatile int64_t* const defer = reinterpret_cast<volatile int64_t*>(gbase + (tmem_slot + 8u - sbase));
+    // checked build: the bookkeeping counters (fills and releases per ring slot, stages and
+    // segments per role), in the fixed region after the barriers
+    volatile uint32_t* const chk = reinterpret_cast<volatile uint32_t*>(gbase + (tmem_slot + 64u - sbase));
+    constexpr int kChkAFill = 0, kChkARel = 10, kChkBFill = 20, kChkProdA = 24, kChkProdB = 25, kChkMma = 26,
+                  kChkRope = 27, kChkMmaSeg = 28, kChkEpiSeg = 29;
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -273,6 +278,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(bar_mma_done, 1);
         *abort_flag = 0;
         defer[0] = 0;
+        if (kChecked)
+            for (int i = 0; i < 32; ++i) chk[i] = 0u;
         fence_barrier_init();
     }
     if (warp == 0 && lane == 0) {
@@ -287,6 +294,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     cluster_sync_all();  // both CTAs' barriers exist before any remote arrive or multicast commit
     tc_fence_after_sync();
     const uint32_t tmem_base = *tmem_slot_ptr;
+    if (threadIdx.x == 0) SEMSHARE_CHECK(tmem_base == 0u, a.err_flag, SEMSHARE_KERNEL_HASH_2SM);  // lane 0, column 0
 
     if (warp == 0) {
         // ---------------- TMA producer of the embedding blocks (both CTAs) ----------------
@@ -310,6 +318,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t s = 0, ph = 0;  // slot and phase parity of stage q (kept incrementally: no divisions)
             for (int64_t it = i0; it < i1; ++it, ++q) {
                 if (!pair_wait(bar_aempty + 8u * s, ph ^ 1u, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns)) break;
+                if (kChecked) {
+                    // the slot's four RoPE warps released every earlier fill of it
+                    SEMSHARE_CHECK(chk[kChkARel + s] == 4u * (q / SA), a.err_flag, SEMSHARE_KERNEL_HASH_2SM);
+                    chk[kChkAFill + s] = chk[kChkAFill + s] + 1u;
+                }
                 const uint32_t full = bar_afull + 8u * s;
                 mbar_arrive_expect_tx(full, kABytes);
                 tma_load_2d(a_ring + s * kABytes, &tmap_emb, full, kb * kBK,
@@ -324,6 +337,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ph ^= 1u;
                 }
             }
+            if (kChecked) chk[kChkProdA] = q;
             // the copies issued last may still be landing
             for (uint32_t i = (q > SA ? q - SA : 0); i < q; ++i) settle_wait(bar_afull + 8u * (i % SA), (i / SA) & 1u);
         }
@@ -341,6 +355,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ok = false;
                     break;
                 }
+                if (kChecked) chk[kChkBFill + s] = chk[kChkBFill + s] + 1u;
                 const uint32_t full = bar_bfull + 8u * s;
                 mbar_arrive_expect_tx(full, a.bh_bytes);
                 tma_load_2d(b_ring + s * a.bh_bytes, &tmap_hyp, full, kb * kBK, hyp_row);
@@ -350,6 +365,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ph ^= 1u;
                 }
             }
+            if (kChecked) chk[kChkProdB] = q;
             for (uint32_t i = (q > SB ? q - SB : 0); i < q; ++i) settle_wait(bar_bfull + 8u * (i % SB), (i / SB) & 1u);
             if (ok) {
                 // the pair's MMAs on the last stages may still be running: their commits arrive on
@@ -372,6 +388,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t a_tmem = tmem_base + kAccCols, bar_s = 0, s = 0, ph = 0, acc = 0;
             bool seg_first = true;
             int kb = static_cast<int>(i0 % nkb);
+            uint32_t n_st = 0, n_seg = 0;  // checked build: stages and segments issued
             for (int64_t it = i0; it < i1; ++it) {
                 if (seg_first) {
                     if (!pair_wait(bar_accempty, (acc & 1u) ^ 1u, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns))
@@ -391,7 +408,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (seg_last) {
                     umma_commit_pair_multicast(bar_accfull, 0x3);
                     ++acc;
+                    ++n_seg;
                 }
+                ++n_st;
                 seg_first = seg_last;
                 if (++s == SB) {
                     s = 0;
@@ -404,6 +423,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     a_tmem += kAStageCols;
                     bar_s += 8u;
                 }
+            }
+            if (kChecked) {
+                chk[kChkMma] = n_st;
+                chk[kChkMmaSeg] = n_seg;
             }
             // every MMA issued above has finished once this arrives: TMEM may then be freed
             umma_commit_pair(bar_mma_done);
@@ -482,6 +505,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             const bool got = pair_wait(bar_afull + 8u * sa, pa, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns);
             if (!__all_sync(0xFFFFFFFFu, got)) break;
+            // the raw block in the slot is this stage's: the slot's fill count is the stage's turn
+            if (kChecked && lane == 0)
+                SEMSHARE_CHECK(chk[kChkAFill + sa] == static_cast<uint32_t>((it - i0) / SA) + 1u, a.err_flag, SEMSHARE_KERNEL_HASH_2SM);
             // the thread's 16 words of the stage into registers, then the raw block is free again
             const uint8_t* const st = gbase + sa * kABytes + row_off;
             uint32_t y[4][4][2];  // [row j][column group c][pair e]: raw pairs, rotated in place
@@ -496,6 +522,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             __syncwarp();
+            if (kChecked && lane == 0) atomicAdd(const_cast<uint32_t*>(chk + kChkARel + sa), 1u);
             if (lane == 0) mbar_arrive(bar_aempty + 8u * sa);
             // the TMEM operand slot is free once the MMAs of the stage SB before have finished
             const bool slot_free =
@@ -572,6 +599,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             // this CTA's hyperplane half of the stage must have landed before the MMA reads it
             const bool b_in = pair_wait(bar_bfull + 8u * sb, pb, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns);
             if (!__all_sync(0xFFFFFFFFu, b_in)) break;
+            if (kChecked && lane == 0) {
+                SEMSHARE_CHECK(chk[kChkBFill + sb] == static_cast<uint32_t>((it - i0) / SB) + 1u, a.err_flag, SEMSHARE_KERNEL_HASH_2SM);
+                if (qd == 0u) atomicAdd(const_cast<uint32_t*>(chk + kChkRope), 1u);
+            }
             tc_fence_before_sync();
             __syncwarp();
             if (lane == 0) arrive_lead(bar_ready + 8u * sb, ready_lead + 8u * sb, leader);
@@ -615,6 +646,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             const bool got = pair_wait(bar_accfull, acc & 1u, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns);
             if (!epilogue_all(got)) break;
+            if (kChecked && threadIdx.x == kEpiWarp0 * 32) chk[kChkEpiSeg] = chk[kChkEpiSeg] + 1u;
             tc_fence_after_sync();
             const int64_t row = ptile_src_row<kRot>(a, tile) + static_cast<int64_t>(rank) * kCM + trow;
             uint32_t* const out_codes = ptile_codes<kRot>(a, tile);
@@ -674,6 +706,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     tc_fence_before_sync();
     __syncthreads();
+    if (kChecked && threadIdx.x == 0 && *abort_flag == 0) {
+        // every role handled the whole range: i1 - i0 stages, one accumulator per K-block segment
+        const uint32_t stages = static_cast<uint32_t>(i1 - i0);
+        const uint32_t segs = i1 > i0 ? static_cast<uint32_t>((i1 - 1) / nkb - i0 / nkb + 1) : 0u;
+        SEMSHARE_CHECK(chk[kChkProdA] == stages, a.err_flag, SEMSHARE_KERNEL_HASH_2SM);
+        SEMSHARE_CHECK(chk[kChkProdB] == stages, a.err_flag, SEMSHARE_KERNEL_HASH_2SM);
+        SEMSHARE_CHECK(chk[kChkRope] == stages, a.err_flag, SEMSHARE_KERNEL_HASH_2SM);
+        SEMSHARE_CHECK(chk[kChkEpiSeg] == segs, a.err_flag, SEMSHARE_KERNEL_HASH_2SM);
+        if (leader) {
+            SEMSHARE_CHECK(chk[kChkMma] == stages, a.err_flag, SEMSHARE_KERNEL_HASH_2SM);
+            SEMSHARE_CHECK(chk[kChkMmaSeg] == segs, a.err_flag, SEMSHARE_KERNEL_HASH_2SM);
+        }
+    }
 
     // ---------------- end phase: the deferred shared segment, by all 16 warps ----------------
     // Warp w reads TMEM lanes 32*(w%4).. (its quadrant) and code words 2*(w/4), 2*(w/4)+1.  The
@@ -714,6 +759,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 close_ok = count_wait(a.tile_count + 2 * tile + rank, static_cast<uint32_t>(b_hi - b_lo), abort_flag,
                                       peer_abort, a.err_flag, a.wait_limit_ns);
             __syncthreads();
+            if (kChecked && close_ok && threadIdx.x == 0)  // every later contributor counted once
+                SEMSHARE_CHECK(ld_acquire_gpu(a.tile_count + 2 * tile + rank) == static_cast<uint32_t>(b_hi - b_lo),
+                               a.err_flag, SEMSHARE_KERNEL_HASH_2SM);
             if (close_ok) {
                 const int64_t row = ptile_src_row<kRot>(a, tile) + static_cast<int64_t>(rank) * kCM + lane_row(r);
                 uint32_t* const out_codes = ptile_codes<kRot>(a, tile);

@@ -51,7 +51,7 @@ constexpr int kEpiWarps = 8;   // two per lane quadrant, one per 128-column half
 constexpr int kHalfCols = kTN / 2;
 constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
 constexpr unsigned long long kNoKey = ~0ull;
-constexpr size_t kFixedSmem = 1024 + 256;
+constexpr size_t kFixedSmem = 1024 + 256 + (kChecked ? 128 : 0);
 
 // Candidate (segment) boundaries of the reference rows, passed by value: off[0] = 0 <
 // off[1] < ... < off[n_seg] = n_ref.  kMax = 1 for the plain search.
@@ -181,6 +181,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem_slot = bars + 104;
     volatile uint32_t* const tmem_slot_ptr = reinterpret_cast<volatile uint32_t*>(gbase + (tmem_slot - sbase));
     volatile int* const abort_flag = reinterpret_cast<volatile int*>(gbase + (tmem_slot + 4u - sbase));
+    // checked build: fills of the two A [0, 2) and two B [2, 4) buffers, releases of the two
+    // accumulators by the epilogue warps [4, 6), tiles issued by the producer [6], the MMA [7] and
+    // drained by the epilogue [8]
+    volatile uint32_t* const chk = reinterpret_cast<volatile uint32_t*>(gbase + (bars + 256u - sbase));
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t G = gridDim.x, b = blockIdx.x;
@@ -197,6 +201,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         mbar_init(bar_done, 1);
         *abort_flag = 0;
+        if (kChecked)
+            for (int i = 0; i < 16; ++i) chk[i] = 0u;
         fence_barrier_init();
     }
     if (warp == 0 && lane == 0) {
@@ -213,6 +219,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem_base = *tmem_slot_ptr;
     const uint64_t lim = a.wait_limit_ns;
     uint32_t* const err = a.err_flag;
+    if (threadIdx.x == 0) SEMSHARE_CHECK(tmem_base == 0u, err, SEMSHARE_KERNEL_HAMMING_TC);  // lane 0, column 0
 
     if (warp == 0) {
         // ---------------- TMA producer ----------------
@@ -228,6 +235,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         ok = false;
                         break;
                     }
+                    if (kChecked) chk[s] = chk[s] + 1u;
                     mbar_arrive_expect_tx(bar_afull + 8 * s, a.a_bytes);
                     for (int c = 0; c < a.kchunks; ++c)
                         tma_load_2d(a_buf0 + s * a.a_bytes + c * (kTM * kChunk), &tm_t, bar_afull + 8 * s, c * kChunk,
@@ -240,12 +248,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ok = false;
                     break;
                 }
+                if (kChecked) chk[2 + s] = chk[2 + s] + 1u;
                 mbar_arrive_expect_tx(bar_bfull + 8 * s, a.b_bytes);
                 for (int c = 0; c < a.kchunks; ++c)
                     tma_load_2d(b_buf0 + s * a.b_bytes + c * (kTN * kChunk), &tm_r, bar_bfull + 8 * s, c * kChunk,
                                 static_cast<int32_t>(rb * kTN));
                 ++nb;
             }
+            if (kChecked && ok) chk[6] = nb;
             if (!ok) {
                 // loads already issued may still be landing: wait for them before exit
                 if (na > 0) drain_wait(bar_afull + 8 * ((na - 1) & 1u), ((na - 1) >> 1) & 1u, kWaitLimitNs);
@@ -269,6 +279,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (!mbar_wait_bounded(bar_afull + 8 * a_slot, (na >> 1) & 1u, abort_flag, err,
                                            SEMSHARE_FLAG_TIMEOUT, lim))
                         break;
+                    SEMSHARE_CHECK(chk[a_slot] == (na >> 1) + 1u, err, SEMSHARE_KERNEL_HAMMING_TC);  // this target block's fill
                     ++na;
                     cur_tb = tb;
                 }
@@ -276,9 +287,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!mbar_wait_bounded(bar_accempty + 8 * buf, ((acc >> 1) & 1u) ^ 1u, abort_flag, err,
                                        SEMSHARE_FLAG_TIMEOUT, lim))
                     break;
+                // every epilogue warp released each earlier use of the accumulator
+                SEMSHARE_CHECK(chk[4 + buf] == static_cast<uint32_t>(kEpiWarps) * (acc >> 1), err, SEMSHARE_KERNEL_HAMMING_TC);
                 const uint32_t s = nb & 1u;
                 if (!mbar_wait_bounded(bar_bfull + 8 * s, (nb >> 1) & 1u, abort_flag, err, SEMSHARE_FLAG_TIMEOUT, lim))
                     break;
+                SEMSHARE_CHECK(chk[2 + s] == (nb >> 1) + 1u, err, SEMSHARE_KERNEL_HAMMING_TC);  // this tile's reference block
                 tc_fence_after_sync();
                 const uint32_t d_tmem = tmem_base + buf * kTN;
                 const uint32_t abase = a_buf0 + a_slot * a.a_bytes, bbase = b_buf0 + s * a.b_bytes;
@@ -293,6 +307,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ++nb;
                 ++acc;
             }
+            if (kChecked) chk[7] = acc;
             umma_commit(bar_done);
             drain_wait(bar_done, 0, kWaitLimitNs);
         }
@@ -418,14 +433,24 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tc_fence_before_sync();
             __syncwarp();
-            if (lane == 0) mbar_arrive(bar_accempty + 8 * buf);
+            if (lane == 0) {
+                if (kChecked) atomicAdd(const_cast<uint32_t*>(chk + 4 + buf), 1u);
+                mbar_arrive(bar_accempty + 8 * buf);
+            }
             fold(bk);
+            if (kChecked && ew == 0 && lane == 0) chk[8] = chk[8] + 1u;
         }
         if (cur_tb >= 0) flush();
     }
 
     tc_fence_before_sync();
     __syncthreads();
+    if (kChecked && threadIdx.x == 0 && *abort_flag == 0) {
+        // every role handled every tile of the range
+        const uint32_t tiles = static_cast<uint32_t>(u1 - u0);
+        SEMSHARE_CHECK(chk[6] == tiles && chk[7] == tiles && chk[8] == tiles, err, SEMSHARE_KERNEL_HAMMING_TC);
+        SEMSHARE_CHECK(chk[4] + chk[5] == static_cast<uint32_t>(kEpiWarps) * tiles, err, SEMSHARE_KERNEL_HAMMING_TC);
+    }
     if (warp == 1) {
         tc_fence_after_sync();
         tmem_dealloc(tmem_base, 512);

@@ -28,6 +28,24 @@ def probe_lib(lib):
     return p
 
 
+@pytest.fixture(scope="module")
+def checked_lib(lib):
+    from paper_2509_24832_gb300 import build
+
+    c = ctypes.CDLL(build.CHECKED_LIB)
+    c.semshare_check_selftest.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+    return c
+
+
+def test_checked_build_exports_the_same_entry_points(lib, checked_lib):
+    """libsemshare_checked.so: the same library with the bookkeeping checks compiled in."""
+    for n in _declared("semshare.h"):
+        assert hasattr(checked_lib, n), n
+    assert lib.semshare_checked_build() == 0 and checked_lib.semshare_checked_build() == 1
+    assert lib.semshare_check_selftest(None, None) == 2              # EUNSUPPORTED: plain build
+    assert checked_lib.semshare_check_selftest(None, None) == 1      # EINVAL: no error word
+
+
 def _declared(header):
     text = open(os.path.join(ROOT, "include", header)).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
@@ -54,6 +72,10 @@ def test_status_helpers(lib):
     assert lib.semshare_flag_status(0) == 0
     assert lib.semshare_flag_status(1) == 4
     assert lib.semshare_flag_status(3) == 5
+    assert lib.semshare_flag_status(4) == 7                        # a failed check (checked build)
+    assert lib.semshare_flag_status(5 | (3 << 8) | (123 << 16)) == 7
+    assert lib.semshare_flag_status(6) == 5                        # a timeout wins
+    assert lib.semshare_status_string(7).startswith(b"checked build")
     assert lib.semshare_match_workspace_size(1000) == 8000
 
 
