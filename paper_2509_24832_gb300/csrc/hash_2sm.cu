@@ -33,8 +33,10 @@
 // The epilogue reads the accumulator lane by lane with the same map.
 //
 // Roles of each CTA (512 threads):
-//   warp 0       TMA producer: its 128 rows x 64 of the embedding block, its half of the
-//                hyperplane block; L2 prefetch of the embedding blocks 2 pipeline depths ahead
+//   warp 0       TMA producer of its 128 rows x 64 of the embedding block; the first two
+//                blocks are requested before the pair's set-up barrier, and the ring fills
+//                behind them at most two blocks ahead of the last one that has landed
+//   warp 2       TMA producer of its half of the hyperplane block
 //   warp 1       TMEM allocation (both CTAs); MMA issue (even CTA): 4 x tcgen05.mma per stage,
 //                commits multicast to both CTAs' barriers
 //   warps 4-11   RoPE, two groups of four warps on alternate stages
@@ -74,8 +76,13 @@ constexpr uint32_t kAStageCols = kBK / 2;    // TMEM columns of one stage's A op
 constexpr uint32_t kTmemCols = 512;
 constexpr int kBSlots = 4;                   // hyperplane halves and TMEM operand slots in flight
 constexpr int kMaxASlots = 10;               // raw embedding blocks in flight
-constexpr uint32_t kMaxTableSmem = 32768;    // rotation tables up to d = 4096 are staged in shared memory
+// Embedding blocks requested while the ring first fills: at most this many beyond the last block
+// that has landed.  Every SM starts at once on a cold L2 full of dirty lines (the previous work's
+// writes); requesting the whole ring at once makes the first block wait for the others, and the
+// first stage is on the critical path.
+constexpr uint32_t kRampLoads = 2;
 constexpr int kRopeBarrier = 2;              // named barrier of the RoPE warps
+constexpr uint32_t kMaxTableSmem = 32768;    // rotation tables up to d = 4096 are staged in shared memory
 static_assert(kAccCols + kBSlots * kAStageCols <= kTmemCols, "TMEM budget");
 static_assert(kBSlots % 2 == 0, "each TMEM operand slot belongs to one RoPE group");
 constexpr int kEpiBarrier = 1;
@@ -282,9 +289,22 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < 32; ++i) chk[i] = 0u;
         fence_barrier_init();
     }
+    // the first embedding blocks are requested now: this CTA's own ring and barriers, so they
+    // need nothing from the peer (the producer loop below continues after them)
+    const uint32_t n_early = static_cast<uint32_t>((i1 - i0) < static_cast<int64_t>(kRampLoads) ? (i1 - i0) : kRampLoads);
+    auto issue_a = [&](int64_t tile, int kb, uint32_t slot) {
+        const uint32_t full = bar_afull + 8u * slot;
+        mbar_arrive_expect_tx(full, kABytes);
+        tma_load_2d(a_ring + slot * kABytes, &tmap_emb, full, kb * kBK,
+                    static_cast<int32_t>(ptile_src_row<kRot>(a, tile)) + static_cast<int32_t>(rank) * kCM);
+    };
     if (warp == 0 && lane == 0) {
         tma_prefetch_desc(&tmap_emb);
         tma_prefetch_desc(&tmap_hyp);
+        for (uint32_t q = 0; q < n_early; ++q) {
+            if (kChecked) chk[kChkAFill + q] = chk[kChkAFill + q] + 1u;
+            issue_a((i0 + q) / nkb, static_cast<int>((i0 + q) % nkb), q);
+        }
     }
     if (warp == 1) {
         tmem_alloc_pair(tmem_slot, kTmemCols);
@@ -299,35 +319,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 0) {
         // ---------------- TMA producer of the embedding blocks (both CTAs) ----------------
         if (lane == 0) {
-            uint32_t q = 0;
-            int64_t tile = i0 / nkb;
-            int kb = static_cast<int>(i0 % nkb);
-            const int32_t half_row = static_cast<int32_t>(rank) * kCM;
-            int64_t pf_tile = tile, pf_it = i0;
-            int pf_kb = kb;
-            auto prefetch_next = [&]() {
-                if (pf_it >= i1) return;
-                tma_prefetch_l2_2d(&tmap_emb, pf_kb * kBK, static_cast<int32_t>(ptile_src_row<kRot>(a, pf_tile)) + half_row);
-                ++pf_it;
-                if (++pf_kb == nkb) {
-                    pf_kb = 0;
-                    ++pf_tile;
+            // stage q = n_early on (the first blocks went out before the set-up barrier); its slot
+            // and phase parity are kept incrementally (no divisions)
+            uint32_t q = n_early;
+            uint32_t s = n_early, ph = 0;  // n_early < SA
+            int64_t tile = (i0 + n_early) / nkb;
+            int kb = static_cast<int>((i0 + n_early) % nkb);
+            for (int64_t it = i0 + n_early; it < i1; ++it, ++q) {
+                if (q < SA) {
+                    // the ring's first fill: ramp behind the blocks that have landed
+                    if (q >= kRampLoads &&
+                        !pair_wait(bar_afull + 8u * (q - kRampLoads), 0u, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns))
+                        break;
+                } else if (!pair_wait(bar_aempty + 8u * s, ph ^ 1u, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns)) {
+                    break;
                 }
-            };
-            for (uint32_t i = 0; i < SA; ++i) prefetch_next();
-            uint32_t s = 0, ph = 0;  // slot and phase parity of stage q (kept incrementally: no divisions)
-            for (int64_t it = i0; it < i1; ++it, ++q) {
-                if (!pair_wait(bar_aempty + 8u * s, ph ^ 1u, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns)) break;
                 if (kChecked) {
                     // the slot's four RoPE warps released every earlier fill of it
                     SEMSHARE_CHECK(chk[kChkARel + s] == 4u * (q / SA), a.err_flag, SEMSHARE_KERNEL_HASH_2SM);
                     chk[kChkAFill + s] = chk[kChkAFill + s] + 1u;
                 }
-                const uint32_t full = bar_afull + 8u * s;
-                mbar_arrive_expect_tx(full, kABytes);
-                tma_load_2d(a_ring + s * kABytes, &tmap_emb, full, kb * kBK,
-                            static_cast<int32_t>(ptile_src_row<kRot>(a, tile)) + half_row);
-                prefetch_next();
+                issue_a(tile, kb, s);
                 if (++kb == nkb) {
                     kb = 0;
                     ++tile;
@@ -524,11 +536,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             __syncwarp();
             if (kChecked && lane == 0) atomicAdd(const_cast<uint32_t*>(chk + kChkARel + sa), 1u);
             if (lane == 0) mbar_arrive(bar_aempty + 8u * sa);
-            // the TMEM operand slot is free once the MMAs of the stage SB before have finished
-            const bool slot_free =
-                pair_wait(bar_done + 8u * sb, pb ^ 1u, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns);
-            if (!__all_sync(0xFFFFFFFFu, slot_free)) break;
-            tc_fence_after_sync();
+            // The TMEM operand slot is free once the MMAs of the stage SB before have finished.  The
+            // rows are rotated first and the wait comes just before the first store, so that the
+            // rotation overlaps those MMAs.
+            bool slot_ok = true, slot_waited = false;
+            auto wait_slot = [&]() -> bool {
+                if (!slot_waited) {
+                    slot_waited = true;
+                    slot_ok = __all_sync(0xFFFFFFFFu, pair_wait(bar_done + 8u * sb, pb ^ 1u, abort_flag, peer_abort,
+                                                                a.err_flag, a.wait_limit_ns));
+                    tc_fence_after_sync();
+                }
+                return slot_ok;
+            };
             const uint32_t tcol = tmem_base + kAccCols + sb * kAStageCols + lane_field;
             if ((kRot == kRotAll || rot) && steps32) {
                 // the usual case, one branch for the whole stage so that the four column groups'
@@ -566,6 +586,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                             }
                         }
                     }
+                    if (!wait_slot()) break;
                     // these two column groups go to tensor memory while the next two are rotated
 #pragma unroll
                     for (int h = 0; h < 2; ++h)
@@ -588,6 +609,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         y[j][c][1] = rotate_to_bf16(bf16_lo(y[j][c][1]), bf16_hi(y[j][c][1]), cs1, sn1);
                     }
                 }  // rows hashed as they are: the bf16 pairs already are the MMA operand
+                if (wait_slot())
 #pragma unroll
                 for (int h = 0; h < 2; ++h)
 #pragma unroll
@@ -596,6 +618,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                         y[2 * h + 1][c][0], y[2 * h + 1][c][1]);
             }
             tmem_st_wait();
+            if (!slot_ok) break;
             // this CTA's hyperplane half of the stage must have landed before the MMA reads it
             const bool b_in = pair_wait(bar_bfull + 8u * sb, pb, abort_flag, peer_abort, a.err_flag, a.wait_limit_ns);
             if (!__all_sync(0xFFFFFFFFu, b_in)) break;
@@ -770,20 +793,29 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int qq = q0 + qi;
                     if (qq >= W) break;
                     // this CTA's K blocks (the tile's first) in the accumulator, then the later
-                    // contributors' partials in K order
+                    // contributors' partials in K order; the first four values of the first
+                    // contributor are requested before the accumulator is read, so that their L2
+                    // latency overlaps the tensor-memory load (more in flight spills registers)
+                    const float4* pp = a.partials + qq * 8 * kCM + r;
+                    float4 f0[4];
+                    if (b_hi > b_lo) {
+                        const float4* p0 = pp + partial_slot(b_lo + 1, rank, tile_it0, a.total_iters, P) * items;
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) f0[j] = __ldcg(p0 + j * kCM);
+                    }
                     uint32_t v[32];
                     tmem_load_32cols_sync(taddr + qq * 32, v);
                     float sum[32];
 #pragma unroll
                     for (int j = 0; j < 32; ++j) sum[j] = __uint_as_float(v[j]);
                     for (int64_t bb = b_lo + 1; bb <= b_hi; ++bb) {
-                        const float4* p0 = a.partials + partial_slot(bb, rank, tile_it0, a.total_iters, P) * items +
-                                           qq * 8 * kCM + r;
+                        const float4* p0 = pp + partial_slot(bb, rank, tile_it0, a.total_iters, P) * items;
 #pragma unroll
                         for (int h = 0; h < 8; h += 4) {
-                            float4 f0[4];
+                            if (h > 0 || bb > b_lo + 1) {
 #pragma unroll
-                            for (int j = 0; j < 4; ++j) f0[j] = __ldcg(p0 + (h + j) * kCM);
+                                for (int j = 0; j < 4; ++j) f0[j] = __ldcg(p0 + (h + j) * kCM);
+                            }
 #pragma unroll
                             for (int j = 0; j < 4; ++j) {
                                 sum[4 * (h + j)] += f0[j].x;
