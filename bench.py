@@ -67,8 +67,10 @@ def parse_args(argv=None):
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(ALL_WORKLOADS))
     p.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
-    p.add_argument("--matcher", default="tc", choices=["tc", "popc"],
-                   help="Hamming search: tensor-core GEMM (semshare_match_tc) or xor/popc (semshare_match)")
+    p.add_argument("--matcher", default="tc", choices=["tc", "signs", "popc"],
+                   help="Hamming search: tensor-core GEMM from the packed codes (semshare_match_tc: expansion, "
+                        "search, key split), the same search on the sign rows the hash writes beside the codes "
+                        "(semshare_hash_signs + semshare_match_tc_signs, one launch) or xor/popc (semshare_match)")
     p.add_argument("--e2e-steps", type=int, default=20)
     p.add_argument("--rope", default="interleaved", choices=["interleaved", "half"],
                    help="rotary pairing: (2k, 2k+1) as Eq. 1 prints it, or (k, k + d/2)")
@@ -293,8 +295,6 @@ class Problem:
     """Device buffers of one matching problem and the three library calls of a step."""
 
     STAGES = ("hash", "match", "gather")
-    # hash 1, match 3 (tc: expand + key reset, search, split; popc: key init, search, split), gather 1
-    LAUNCHES_PER_STEP = 5
 
     def __init__(self, wl: workloads.Workload, device, seed: int, matcher: str = "tc", with_hd: bool = False,
                  with_retain: bool = False):
@@ -323,6 +323,15 @@ class Problem:
         self.ws = torch.empty(ss.semshare_match_workspace_size(n_t), dtype=torch.uint8, device=device)
         self.tc_ws = torch.empty(max(256, ss.semshare_match_tc_workspace_size(n_t, wl.n_ref, wl.nbits)),
                                  dtype=torch.uint8, device=device)
+        # matcher "signs": the hash also writes the sign rows, which the one-launch search reads; its
+        # workspace starts 0xFF-filled and every call leaves it so
+        self.signs = torch.empty((rows, ss.semshare_signs_pitch(wl.nbits)), dtype=torch.uint8, device=device) \
+            if matcher == "signs" else None
+        self.signs_ws = torch.full((max(512, ss.semshare_match_tc_signs_workspace_size(n_t)),), 0xFF,
+                                   dtype=torch.uint8, device=device) if matcher == "signs" else None
+        # library launches per step: hash 1; match: signs 1 (2 above the fused split's target count),
+        # tc 3 (expansion + key reset, search, key split), popc 3 (key init, search, split); gather 1
+        self.LAUNCHES_PER_STEP = 2 + ({"signs": 1 if n_t <= ss.MATCH_SIGNS_FUSED_MAX_TARGETS else 2}.get(matcher, 3))
         self.hash_ws = torch.zeros(max(256, ss.semshare_hash_workspace_size(rows, wl.d, wl.nbits)), dtype=torch.uint8,
                                    device=device)
         segs = [workloads.kv_cache_device(wl, device, seed=seed, segment=s) for s in range(wl.n_seg)]
@@ -361,7 +370,7 @@ class Problem:
             self.hd_k = ss.hd_count(wl.n_tgt)
             self.hd_idx = torch.empty((wl.n_batch, self.hd_k), dtype=torch.int32, device=device)
             self.STAGES = Problem.STAGES + ("deviation", "select")
-            self.LAUNCHES_PER_STEP = Problem.LAUNCHES_PER_STEP + 2
+            self.LAUNCHES_PER_STEP += 2
 
     def deviation(self):
         self.ss.semshare_kv_deviation(self.out_k[:, 0], self.out_v[:, 0], self.rc_k, self.rc_v, sigma_kv=self.sigma)
@@ -370,12 +379,24 @@ class Problem:
         self.ss.semshare_select_hd(self.sigma, self.hd_k, hd_idx=self.hd_idx)
 
     def hash(self):
-        self.ss.semshare_hash(self.emb, self.table, self.hyp, self.pos, codes=self.codes, err_flag=self.flag,
-                              workspace=self.hash_ws, rope_layout=self.rope_layout)
+        self.hash_rows(self.emb, self.pos, self.codes, self.signs, self.hash_ws)
+
+    def hash_rows(self, emb, pos, codes, signs, ws):
+        """The hash of some rows (all of them, or only the target's), with the sign rows when the
+        matcher reads them."""
+        if signs is not None:
+            self.ss.semshare_hash_signs(emb, self.table, self.hyp, pos, codes=codes, signs=signs, err_flag=self.flag,
+                                        workspace=ws, rope_layout=self.rope_layout)
+        else:
+            self.ss.semshare_hash(emb, self.table, self.hyp, pos, codes=codes, err_flag=self.flag, workspace=ws,
+                                  rope_layout=self.rope_layout)
 
     def match(self):
         n_ref = self.wl.n_ref
-        if self.matcher == "tc":
+        if self.matcher == "signs":
+            self.ss.semshare_match_tc_signs(self.signs[n_ref:], self.signs[:n_ref], self.wl.nbits, idx=self.idx,
+                                            dist=self.dist, workspace=self.signs_ws, err_flag=self.flag)
+        elif self.matcher == "tc":
             self.ss.semshare_match_tc(self.codes[n_ref:], self.codes[:n_ref], idx=self.idx, dist=self.dist,
                                       workspace=self.tc_ws, err_flag=self.flag)
         else:
@@ -440,9 +461,10 @@ class Problem:
                                  dtype=torch.uint8, device=self.dev)
             self.hash()  # the reference codes, once (store time)
 
+            tgt_signs = None if self.signs is None else self.signs[n_ref:]
+
             def hash_step():
-                self.ss.semshare_hash(emb_d, self.table, self.hyp, pos_d, codes=tgt_codes, err_flag=self.flag,
-                                      workspace=tgt_ws, rope_layout=self.rope_layout)
+                self.hash_rows(emb_d, pos_d, tgt_codes, tgt_signs, tgt_ws)
         else:
             hash_step = self.hash
         h_k = [t.cpu().pin_memory() for t in self.ref_k]
@@ -531,7 +553,7 @@ class RetrieveProblem:
 
         import paper_2509_24832_gb300 as ss
 
-        if matcher != "tc":
+        if matcher not in ("signs", "tc"):
             raise ValueError("the retrieval step uses the tensor-core matcher")
         self.ss, self.wl, self.dev, self.matcher = ss, wl, device, matcher
         emb, pos, _ = workloads.prompt_rows(wl, seed=seed)
@@ -995,8 +1017,10 @@ def run_ref_codes_cached(args, prob, device, flush):
                      dtype=torch.uint8, device=device)
     prob.hash()  # the reference codes, once
 
+    tgt_signs = None if prob.signs is None else prob.signs[wl.n_ref:]
+
     def step():
-        ss.semshare_hash(tgt_emb, prob.table, prob.hyp, tgt_pos, codes=tgt_codes, err_flag=prob.flag, workspace=ws)
+        prob.hash_rows(tgt_emb, tgt_pos, tgt_codes, tgt_signs, ws)
         prob.match()
         prob.gather()
         if prob.hd:

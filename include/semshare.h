@@ -215,6 +215,28 @@ semshare_status semshare_hash(const void* emb, semshare_dtype dtype, int64_t n, 
                               size_t workspace_bytes, uint32_t* err_flag, void* stream);
 
 /*
+ * semshare_hash_signs -- semshare_hash_ex that also writes the codes as the +-1 operand rows of
+ * the tensor-core match (semshare_match_tc_signs).
+ *
+ * The tensor-core search of Sec. 3.3's nearest token computes popcount(a XOR b) as
+ * (nbits - <s_a, s_b>) / 2 with s = 2*bit - 1; its operands are the codes as rows of e4m3 bytes.
+ * The hash epilogue holds the sign bits already, so it writes those rows beside the packed codes
+ * and the match needs no expansion pass.
+ *
+ *   every argument as for semshare_hash_ex, plus
+ *   signs   device, [n][semshare_signs_pitch(nbits)] bytes, 16-byte aligned; written: byte j of
+ *           row i is 0x38 (e4m3 +1) if bit j of codes[i] is set, else 0xB8 (e4m3 -1); bytes
+ *           nbits .. pitch-1 of every row are 0
+ * Returns as semshare_hash_ex (EINVAL for a NULL or misaligned signs when n > 0).
+ */
+int32_t semshare_signs_pitch(int32_t nbits); /* 128 * ceil(nbits / 128); 0 for an unsupported nbits */
+semshare_status semshare_hash_signs(const void* emb, semshare_dtype dtype, int64_t n, int32_t d, int64_t row_stride,
+                                    const int32_t* positions, const uint64_t* rope_table, const uint16_t* hyperplanes,
+                                    int32_t nbits, uint32_t rope_layout, uint32_t* codes, uint8_t* signs,
+                                    float* proj_out, void* workspace, size_t workspace_bytes, uint32_t* err_flag,
+                                    void* stream);
+
+/*
  * semshare_match -- step 3: Hamming nearest reference token of every target token.
  *
  * Sec. 3.3: "for each token in the target prompt, the most similar token in the reference
@@ -259,6 +281,32 @@ size_t semshare_match_tc_workspace_size(int64_t n_tgt, int64_t n_ref, int32_t nb
 semshare_status semshare_match_tc(const uint32_t* tgt_codes, int64_t n_tgt, const uint32_t* ref_codes, int64_t n_ref,
                                   int32_t nbits, int32_t* idx, int32_t* dist, void* workspace, size_t workspace_bytes,
                                   uint32_t* err_flag, void* stream);
+
+/*
+ * semshare_match_tc_signs -- semshare_match_tc on sign rows written by semshare_hash_signs, in
+ * one launch.
+ *
+ * Same problem, tie rule and result as semshare_match (Sec. 3.3: the most similar reference token
+ * of each target token, ties to the lowest index).  The operands are already +-1 rows, so there is
+ * no expansion pass, and the search's last CTA to finish turns the per-target keys into idx and
+ * dist (for up to 16384 targets; larger calls add one small launch that does it).
+ *
+ *   tgt_signs  device, [n_tgt][semshare_signs_pitch(nbits)] bytes as semshare_hash_signs writes
+ *              them, 16-byte aligned
+ *   ref_signs  device, [n_ref][semshare_signs_pitch(nbits)] bytes, 16-byte aligned
+ *   n_tgt, n_ref, nbits, idx, dist, err_flag, stream   as for semshare_match_tc
+ *   workspace  device scratch of at least semshare_match_tc_signs_workspace_size(n_tgt) bytes,
+ *              256-byte aligned.  Every byte must be 0xFF before its first use (e.g.
+ *              cudaMemsetAsync(workspace, 0xFF, bytes)); every call leaves it that way again, also
+ *              when a pipeline wait gives up, so one workspace (sized for the largest call) serves
+ *              any number of calls made one after another on the same device.  Calls that may
+ *              run concurrently need separate workspaces.
+ * Returns EINVAL / EUNSUPPORTED for bad arguments, ECUDA if a launch fails.
+ */
+size_t semshare_match_tc_signs_workspace_size(int64_t n_tgt);
+semshare_status semshare_match_tc_signs(const uint8_t* tgt_signs, int64_t n_tgt, const uint8_t* ref_signs,
+                                        int64_t n_ref, int32_t nbits, int32_t* idx, int32_t* dist, void* workspace,
+                                        size_t workspace_bytes, uint32_t* err_flag, void* stream);
 
 /*
  * semshare_retrieve -- reference retrieval: which stored prompt the target should reuse.

@@ -77,6 +77,15 @@ def load():
         lib.semshare_hash_ex.argtypes = [P, ctypes.c_int, i64, i32, i64, P, P, P, i32, u32, P, P, P, ctypes.c_size_t,
                                          P, P]
         lib.semshare_hash_ex.restype = ctypes.c_int
+        lib.semshare_signs_pitch.argtypes = [i32]
+        lib.semshare_signs_pitch.restype = i32
+        lib.semshare_hash_signs.argtypes = [P, ctypes.c_int, i64, i32, i64, P, P, P, i32, u32, P, P, P, P,
+                                            ctypes.c_size_t, P, P]
+        lib.semshare_hash_signs.restype = ctypes.c_int
+        lib.semshare_match_tc_signs_workspace_size.argtypes = [i64]
+        lib.semshare_match_tc_signs_workspace_size.restype = ctypes.c_size_t
+        lib.semshare_match_tc_signs.argtypes = [P, i64, P, i64, i32, P, P, P, ctypes.c_size_t, P, P]
+        lib.semshare_match_tc_signs.restype = ctypes.c_int
         lib.semshare_match_workspace_size.argtypes = [i64]
         lib.semshare_match_workspace_size.restype = ctypes.c_size_t
         lib.semshare_match.argtypes = [P, i64, P, i64, i32, P, P, P, ctypes.c_size_t, P]
@@ -287,6 +296,56 @@ def semshare_hash(emb: torch.Tensor, rope_table: torch.Tensor, hyperplanes: torc
     return call if prepare else call(stream)
 
 
+def semshare_signs_pitch(nbits: int) -> int:
+    """Bytes per sign row of semshare_hash_signs (128 * ceil(nbits / 128))."""
+    return int(load().semshare_signs_pitch(int(nbits)))
+
+
+def semshare_hash_signs(emb: torch.Tensor, rope_table: torch.Tensor, hyperplanes: torch.Tensor,
+                        positions: torch.Tensor | None = None, codes: torch.Tensor | None = None,
+                        signs: torch.Tensor | None = None, proj_out: torch.Tensor | None = None,
+                        err_flag: torch.Tensor | None = None, workspace: torch.Tensor | None = None, stream=None,
+                        rope_layout: str = "interleaved", *, prepare: bool = False):
+    """semshare_hash that also writes the codes as e4m3 +-1 rows, the operands of
+    semshare_match_tc_signs.  Arguments as for semshare_hash, plus signs: uint8
+    [n][semshare_signs_pitch(nbits)] (allocated when None).  Returns (codes, signs)."""
+    _need_cuda(emb, "emb")
+    _need_cuda(hyperplanes, "hyperplanes")
+    if emb.dim() != 2 or emb.stride(1) != 1:
+        raise ValueError("emb must be [n][d] with unit stride along d")
+    dt = {torch.bfloat16: BF16, torch.float32: F32}.get(emb.dtype)
+    if dt is None:
+        raise ValueError("emb must be bfloat16 or float32")
+    if hyperplanes.dtype != torch.bfloat16 or not hyperplanes.is_contiguous():
+        raise ValueError("hyperplanes must be contiguous bfloat16 [nbits][d]")
+    n, d = emb.shape
+    nbits = hyperplanes.shape[0]
+    if hyperplanes.shape[1] != d:
+        raise ValueError("hyperplanes width differs from emb")
+    if positions is not None and (positions.dtype != torch.int32 or positions.numel() != n
+                                  or not positions.is_contiguous()):
+        raise ValueError("positions must be contiguous int32 [n]")
+    pitch = semshare_signs_pitch(nbits)
+    if codes is None:
+        codes = torch.empty((n, nbits // 32), dtype=torch.int32, device=emb.device)
+    if signs is None:
+        signs = torch.empty((n, pitch), dtype=torch.uint8, device=emb.device)
+    elif signs.dtype != torch.uint8 or signs.shape != (n, pitch) or not signs.is_contiguous():
+        raise ValueError(f"signs must be contiguous uint8 [{n}][{pitch}]")
+    if workspace is None:
+        workspace = hash_workspace(n, d, nbits, emb.device)
+    if rope_layout not in ROPE_LAYOUTS:
+        raise ValueError(f"rope_layout must be one of {sorted(ROPE_LAYOUTS)}")
+    if rope_layout != "none":
+        _need_cuda(rope_table, "rope_table")
+    args = (_ptr(emb), dt, n, d, emb.stride(0), _ptr(positions), _ptr(rope_table), _ptr(hyperplanes), nbits,
+            ROPE_LAYOUTS[rope_layout], _ptr(codes), _ptr(signs), _ptr(proj_out), _ptr(workspace),
+            workspace.numel() * workspace.element_size(), _ptr(err_flag))
+    call = Prepared(load().semshare_hash_signs, args, "semshare_hash_signs",
+                    (emb, positions, rope_table, hyperplanes, proj_out, workspace, err_flag), (codes, signs))
+    return call if prepare else call(stream)
+
+
 def semshare_hash_pair_workspace_size(n: int, d: int, nbits: int) -> int:
     return int(load().semshare_hash_pair_workspace_size(int(n), int(d), int(nbits)))
 
@@ -389,6 +448,59 @@ def semshare_match_tc(tgt_codes: torch.Tensor, ref_codes: torch.Tensor, idx: tor
             workspace.numel() * workspace.element_size(), _ptr(err_flag))
     call = Prepared(load().semshare_match_tc, args, "semshare_match_tc", (tgt_codes, ref_codes, workspace, err_flag),
                     (idx, dist))
+    return call if prepare else call(stream)
+
+
+_match_signs_ws = {}
+# Targets up to which semshare_match_tc_signs is one launch (include/semshare.h); above it a small
+# split launch follows the search.
+MATCH_SIGNS_FUSED_MAX_TARGETS = 16384
+
+
+def semshare_match_tc_signs_workspace_size(n_tgt: int) -> int:
+    return int(load().semshare_match_tc_signs_workspace_size(int(n_tgt)))
+
+
+def match_signs_workspace(n_tgt: int, device=None) -> torch.Tensor:
+    """A 0xFF-filled semshare_match_tc_signs workspace large enough for n_tgt targets, kept per
+    device and grown on demand.  Every call leaves it 0xFF-filled, so calls issued one after
+    another (on one stream) can share it; concurrent calls need their own."""
+    dev = torch.device(device or "cuda")
+    if dev.index is None:
+        dev = torch.device("cuda", torch.cuda.current_device())
+    need = max(512, semshare_match_tc_signs_workspace_size(n_tgt))
+    ws = _match_signs_ws.get(dev)
+    if ws is None or ws.numel() < need:
+        ws = torch.full((need,), 0xFF, dtype=torch.uint8, device=dev)
+        _match_signs_ws[dev] = ws
+    return ws
+
+
+def semshare_match_tc_signs(tgt_signs: torch.Tensor, ref_signs: torch.Tensor, nbits: int,
+                            idx: torch.Tensor | None = None, dist: torch.Tensor | None = None,
+                            workspace: torch.Tensor | None = None, err_flag: torch.Tensor | None = None,
+                            stream=None, *, prepare: bool = False):
+    """semshare_match_tc on the sign rows of semshare_hash_signs (uint8 [n][pitch], rows may be a
+    slice of one hash call's output), in one launch.  workspace: 0xFF-filled (default: the
+    per-device one of match_signs_workspace()).  Returns (idx, dist)."""
+    _need_cuda(tgt_signs, "tgt_signs")
+    _need_cuda(ref_signs, "ref_signs")
+    pitch = semshare_signs_pitch(nbits)
+    for name, t in (("tgt_signs", tgt_signs), ("ref_signs", ref_signs)):
+        if t.dtype != torch.uint8 or t.dim() != 2 or t.shape[1] != pitch or not t.is_contiguous():
+            raise ValueError(f"{name} must be contiguous uint8 [n][{pitch}]")
+    n_tgt, n_ref = tgt_signs.shape[0], ref_signs.shape[0]
+    dev = tgt_signs.device
+    if idx is None:
+        idx = torch.empty(n_tgt, dtype=torch.int32, device=dev)
+    if dist is None:
+        dist = torch.empty(n_tgt, dtype=torch.int32, device=dev)
+    if workspace is None:
+        workspace = match_signs_workspace(n_tgt, dev)
+    args = (_ptr(tgt_signs), n_tgt, _ptr(ref_signs), n_ref, int(nbits), _ptr(idx), _ptr(dist), _ptr(workspace),
+            workspace.numel() * workspace.element_size(), _ptr(err_flag))
+    call = Prepared(load().semshare_match_tc_signs, args, "semshare_match_tc_signs",
+                    (tgt_signs, ref_signs, workspace, err_flag), (idx, dist))
     return call if prepare else call(stream)
 
 

@@ -101,6 +101,8 @@ struct HashArgs {
     const uint64_t* rope_table;
     uint32_t* codes;
     float* proj;
+    uint8_t* signs;  // nullable: [n][signs_pitch] e4m3 +-1 bytes of the code bits, zero-padded
+    int32_t signs_pitch;
     uint32_t* err_flag;
     uint32_t* tile_count;  // workspace: [n_tiles] arrivals of shared tiles, zero between calls
     float4* partials;      // workspace: [2 * gridDim.x][nbits/32][8][128] partial accumulators
@@ -668,7 +670,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_before_sync();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar_accempty + 8u * buf);
-                if (row < a.n) store_codes(out_codes, row, W, words);
+                if (row < a.n) {
+                    store_codes(out_codes, row, W, words);
+                    if (a.signs != nullptr) store_sign_row(a.signs, row, a.signs_pitch, W, words);
+                }
             } else {
                 // shared tile: this CTA's partial sum goes to its workspace slot.  The last segment's
                 // is staged in the idle pipeline buffers and published by the whole CTA at the end.
@@ -806,8 +811,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int j = 0; j < 32; ++j) v[j] = __float_as_uint(sum[j]);
                 const int64_t row = tile_src_row<kRot>(a, tile) + rr;
                 if (row < a.n) {
-                    tile_codes<kRot>(a, tile)[row * W + qq] = sign_word(v);
+                    const uint32_t bits = sign_word(v);
+                    tile_codes<kRot>(a, tile)[row * W + qq] = bits;
                     if (a.proj != nullptr) store_proj(a.proj, row, a.nbits, qq, v);
+                    if (a.signs != nullptr) store_sign_bytes(a.signs + row * a.signs_pitch + 32 * qq, bits);
+                }
+            }
+            if (a.signs != nullptr) {
+                // the pad of the sign rows past the code bits
+                const int pads = a.signs_pitch / 32 - W;
+                for (int e = threadIdx.x; e < pads * kBM; e += kThreads) {
+                    const int64_t row = tile_src_row<kRot>(a, tile) + e % kBM;
+                    if (row < a.n) store_sign_pad(a.signs + row * a.signs_pitch + 32 * (W + e / kBM));
                 }
             }
             if (threadIdx.x == 0) a.tile_count[tile] = 0u;  // leave the workspace zeroed
@@ -869,7 +884,7 @@ namespace {
 semshare_status hash_impl(const void* emb, semshare_dtype dtype, int64_t n, int32_t d, int64_t row_stride,
                           const int32_t* positions, const uint64_t* rope_table, const uint16_t* hyperplanes,
                           int32_t nbits, uint32_t rope_layout, uint32_t* codes, uint32_t* codes2, float* proj_out,
-                          void* workspace, size_t workspace_bytes, uint32_t* err_flag, void* stream) {
+                          uint8_t* signs, void* workspace, size_t workspace_bytes, uint32_t* err_flag, void* stream) {
     const bool pair = codes2 != nullptr;
     if (dtype != SEMSHARE_BF16 && dtype != SEMSHARE_F32) return SEMSHARE_EINVAL;
     if (rope_layout != SEMSHARE_ROPE_INTERLEAVED && rope_layout != SEMSHARE_ROPE_HALF &&
@@ -892,7 +907,10 @@ semshare_status hash_impl(const void* emb, semshare_dtype dtype, int64_t n, int3
     if ((proj_out && !aligned(proj_out, 16)) || (positions && !aligned(positions, 4)) ||
         (err_flag && !aligned(err_flag, 4)))
         return SEMSHARE_EINVAL;
-    if (pair && (rope_layout != SEMSHARE_ROPE_INTERLEAVED || proj_out || !aligned(codes2, 16))) return SEMSHARE_EINVAL;
+    if (pair && (rope_layout != SEMSHARE_ROPE_INTERLEAVED || proj_out || signs || !aligned(codes2, 16)))
+        return SEMSHARE_EINVAL;
+    if (signs && !aligned(signs, 16)) return SEMSHARE_EINVAL;
+    const int32_t signs_pitch = semshare_signs_pitch(nbits);
     const int64_t n_pad = ((n + kBM - 1) / kBM) * kBM;
 
     HashPlan plan;
@@ -915,6 +933,8 @@ semshare_status hash_impl(const void* emb, semshare_dtype dtype, int64_t n, int3
         c.codes = codes;
         c.codes2 = codes2;
         c.proj = proj_out;
+        c.signs = signs;
+        c.signs_pitch = signs_pitch;
         c.err_flag = err_flag;
         c.partials = workspace;
         c.partial_bytes = plan.partial_bytes;
@@ -960,6 +980,8 @@ semshare_status hash_impl(const void* emb, semshare_dtype dtype, int64_t n, int3
     a.codes2 = codes2;
     a.codes = codes;
     a.proj = proj_out;
+    a.signs = signs;
+    a.signs_pitch = signs_pitch;
     a.err_flag = err_flag;
     a.partials = static_cast<float4*>(workspace);
     a.tile_count = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(workspace) + plan.partial_bytes);
@@ -995,7 +1017,23 @@ extern "C" semshare_status semshare_hash_ex(const void* emb, semshare_dtype dtyp
                                             uint32_t* codes, float* proj_out, void* workspace,
                                             size_t workspace_bytes, uint32_t* err_flag, void* stream) {
     return semshare::hash_impl(emb, dtype, n, d, row_stride, positions, rope_table, hyperplanes, nbits, rope_layout,
-                               codes, nullptr, proj_out, workspace, workspace_bytes, err_flag, stream);
+                               codes, nullptr, proj_out, nullptr, workspace, workspace_bytes, err_flag, stream);
+}
+
+extern "C" int32_t semshare_signs_pitch(int32_t nbits) {
+    if (nbits < 32 || nbits > 256 || nbits % 32 != 0) return 0;
+    return ((nbits + 127) / 128) * 128;
+}
+
+extern "C" semshare_status semshare_hash_signs(const void* emb, semshare_dtype dtype, int64_t n, int32_t d,
+                                               int64_t row_stride, const int32_t* positions,
+                                               const uint64_t* rope_table, const uint16_t* hyperplanes, int32_t nbits,
+                                               uint32_t rope_layout, uint32_t* codes, uint8_t* signs,
+                                               float* proj_out, void* workspace, size_t workspace_bytes,
+                                               uint32_t* err_flag, void* stream) {
+    if (n > 0 && !signs) return SEMSHARE_EINVAL;
+    return semshare::hash_impl(emb, dtype, n, d, row_stride, positions, rope_table, hyperplanes, nbits, rope_layout,
+                               codes, nullptr, proj_out, signs, workspace, workspace_bytes, err_flag, stream);
 }
 
 extern "C" size_t semshare_hash_pair_workspace_size(int64_t n, int32_t d, int32_t nbits) {
@@ -1013,7 +1051,7 @@ extern "C" semshare_status semshare_hash_pair(const void* emb, semshare_dtype dt
     if (n >= (int64_t(1) << 30)) return SEMSHARE_EUNSUPPORTED;  // twice the rows stay below 2^31
     return semshare::hash_impl(emb, dtype, n, d, row_stride, positions, rope_table, hyperplanes, nbits,
                                SEMSHARE_ROPE_INTERLEAVED, codes_plain, n > 0 ? codes_rotary : nullptr, nullptr,
-                               workspace, workspace_bytes, err_flag, stream);
+                               nullptr, workspace, workspace_bytes, err_flag, stream);
 }
 
 extern "C" semshare_status semshare_hash(const void* emb, semshare_dtype dtype, int64_t n, int32_t d,

@@ -105,6 +105,8 @@ struct Hash2smArgs {
     uint32_t* codes;
     uint32_t* codes2;
     float* proj;
+    uint8_t* signs;       // nullable: [n][signs_pitch] e4m3 +-1 bytes of the code bits, zero-padded
+    int32_t signs_pitch;
     uint32_t* err_flag;
     uint32_t* tile_count;  // workspace: [2 * n_ptiles] arrivals at each CTA half of a shared pair tile
     float4* partials;      // workspace: [2 per CTA][nbits/32 * 8][128] partial accumulators
@@ -689,7 +691,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_before_sync();
                 __syncwarp();
                 if (lane == 0) arrive_lead(bar_accempty, accempty_lead, leader);
-                if (row < a.n) store_codes(out_codes, row, W, words);
+                if (row < a.n) {
+                    store_codes(out_codes, row, W, words);
+                    if (a.signs != nullptr) store_sign_row(a.signs, row, a.signs_pitch, W, words);
+                }
             } else if (it + seg_len == i1) {
                 // the CTA's last segment, part of a shared tile: closed (this cluster owns the tile's
                 // first K blocks) or published (it does not) by all warps after the main loop,
@@ -791,7 +796,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll 1
                 for (int qi = 0; qi < 2; ++qi) {
                     const int qq = q0 + qi;
-                    if (qq >= W) break;
+                    if (qq >= W) {
+                        // the pad of the sign rows past the code bits
+                        if (a.signs != nullptr && 32 * qq < a.signs_pitch && row < a.n)
+                            store_sign_pad(a.signs + row * a.signs_pitch + 32 * qq);
+                        continue;
+                    }
                     // this CTA's K blocks (the tile's first) in the accumulator, then the later
                     // contributors' partials in K order; the first four values of the first
                     // contributor are requested before the accumulator is read, so that their L2
@@ -828,8 +838,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int j = 0; j < 32; ++j) v[j] = __float_as_uint(sum[j]);
                     if (row < a.n) {
-                        out_codes[row * W + qq] = sign_word(v);
+                        const uint32_t bits = sign_word(v);
+                        out_codes[row * W + qq] = bits;
                         if (a.proj != nullptr) store_proj(a.proj, row, a.nbits, qq, v);
+                        if (a.signs != nullptr) store_sign_bytes(a.signs + row * a.signs_pitch + 32 * qq, bits);
                     }
                 }
                 if (threadIdx.x == 0) a.tile_count[2 * tile + rank] = 0u;  // leave the workspace zeroed
@@ -905,6 +917,8 @@ semshare_status launch_hash_2sm(const Hash2smCall& c) {
     a.codes = c.codes;
     a.codes2 = c.codes2;
     a.proj = c.proj;
+    a.signs = c.signs;
+    a.signs_pitch = c.signs_pitch;
     a.err_flag = c.err_flag;
     a.partials = static_cast<float4*>(c.partials);
     a.tile_count = c.tile_count;

@@ -24,6 +24,8 @@ struct Hash2smCall {
     uint32_t* codes;
     uint32_t* codes2;
     float* proj;
+    uint8_t* signs;           // nullable: the codes as e4m3 +-1 rows of signs_pitch bytes
+    int32_t signs_pitch;
     uint32_t* err_flag;
     void* partials;           // workspace partial-slot region
     size_t partial_bytes;

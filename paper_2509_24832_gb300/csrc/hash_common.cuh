@@ -65,6 +65,38 @@ __device__ __forceinline__ void store_proj(float* proj, int64_t row, int nbits, 
                             __uint_as_float(v[4 * j + 3]));
 }
 
+// 32 code bits as the operand bytes of the tensor-core match: e4m3 +1 (0x38) for a set bit, -1
+// (0xB8) for a clear one (byte = 0xB8 ^ bit << 7), bit j at byte j of dst (16-byte aligned).  Four
+// bits m spread to bit 7 of four bytes by one multiply: m * 0x10204080 puts bit i of m at bit
+// 8i+7 (the shifted copies of m do not overlap).
+__device__ __forceinline__ void store_sign_bytes(uint8_t* dst, uint32_t bits) {
+    uint32_t w[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) w[q] = 0xB8B8B8B8u ^ ((((bits >> (4 * q)) & 0xFu) * 0x10204080u) & 0x80808080u);
+    uint4* d = reinterpret_cast<uint4*>(dst);
+    d[0] = make_uint4(w[0], w[1], w[2], w[3]);
+    d[1] = make_uint4(w[4], w[5], w[6], w[7]);
+}
+
+// The zero bytes that pad a sign row to its pitch.
+__device__ __forceinline__ void store_sign_pad(uint8_t* dst) {
+    uint4* d = reinterpret_cast<uint4*>(dst);
+    d[0] = make_uint4(0u, 0u, 0u, 0u);
+    d[1] = make_uint4(0u, 0u, 0u, 0u);
+}
+
+// A whole sign row: the W code words as bytes, then zeros up to pitch (a multiple of 32, <= 256).
+__device__ __forceinline__ void store_sign_row(uint8_t* signs, int64_t row, int pitch, int W, const uint32_t (&words)[8]) {
+    uint8_t* d = signs + row * pitch;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+        if (q < W)
+            store_sign_bytes(d + 32 * q, words[q]);
+        else if (32 * q < pitch)
+            store_sign_pad(d + 32 * q);
+    }
+}
+
 __device__ __forceinline__ void store_codes(uint32_t* codes, int64_t row, int W, const uint32_t (&words)[8]) {
     uint32_t* cp = codes + row * W;
     if ((W & 3) == 0) {

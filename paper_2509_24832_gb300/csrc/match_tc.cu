@@ -51,6 +51,10 @@ constexpr int kEpiWarps = 8;   // two per lane quadrant, one per 128-column half
 constexpr int kHalfCols = kTN / 2;
 constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
 constexpr unsigned long long kNoKey = ~0ull;
+constexpr unsigned int kNoArrivals = ~0u;  // the fused search's arrival counter between calls
+// Targets up to which the last CTA of the search splits the keys itself (a few per thread);
+// larger searches hand them to tc_keys_split_kernel, which spreads them over the GPU.
+constexpr int64_t kFusedSplitMaxTargets = 16384;
 constexpr size_t kFixedSmem = 1024 + 256 + (kChecked ? 128 : 0);
 
 // Candidate (segment) boundaries of the reference rows, passed by value: off[0] = 0 <
@@ -74,6 +78,10 @@ struct TcArgs {
     unsigned long long* keys;  // [n_seg][n_tgt]
     uint32_t* err_flag;
     uint64_t wait_limit_ns;
+    // fused split (kFused): the last CTA to finish writes idx/dist from the keys and resets them
+    int32_t* idx;
+    int32_t* dist;
+    unsigned int* counter;     // arrivals, kNoArrivals between calls
 };
 
 // Offsets of the candidates of a pool, passed by value (semshare_match_tc_selected; kMax = 1
@@ -143,13 +151,15 @@ __global__ void expand_codes_kernel(const uint32_t* __restrict__ tgt, int64_t n_
 
 // sel non-null: idx are pool rows, local + sel[1]; a target with no key (an invalid candidate)
 // gets idx = dist = -1.
-__global__ void tc_keys_split_kernel(const unsigned long long* __restrict__ keys, int64_t n, int32_t* __restrict__ idx,
-                                     int32_t* __restrict__ dist, const int64_t* __restrict__ sel) {
+// reset: leave every key at kNoKey again (the searches over caller sign rows expect it on entry).
+__global__ void tc_keys_split_kernel(unsigned long long* __restrict__ keys, int64_t n, int32_t* __restrict__ idx,
+                                     int32_t* __restrict__ dist, const int64_t* __restrict__ sel, bool reset) {
     pdl_prologue();
     const int64_t base = sel ? sel[1] : 0;
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const unsigned long long k = keys[i];
+        if (reset) keys[i] = kNoKey;
         const bool none = k == kNoKey;
         idx[i] = none ? -1 : static_cast<int32_t>(static_cast<uint32_t>(k) + base);
         if (dist) dist[i] = none ? -1 : static_cast<int32_t>(static_cast<uint32_t>(k >> 32));
@@ -164,11 +174,17 @@ __device__ __forceinline__ bool drain_wait(uint32_t bar, uint32_t parity, uint64
     return true;
 }
 
-template <int kMaxSeg>
+// kFused (plain search only): the keys are kNoKey on entry; the last CTA to finish writes idx and
+// dist from them and resets them (and the arrival counter) for the next call.
+template <int kMaxSeg, bool kFused = false>
 __global__ void __launch_bounds__(kThreads, 1)
     hamming_tc_kernel(const __grid_constant__ CUtensorMap tm_t, const __grid_constant__ CUtensorMap tm_r,
                       const TcArgs a, const __grid_constant__ SegTable<kMaxSeg> seg) {
-    pdl_prologue();
+    static_assert(!kFused || kMaxSeg == 1, "the fused split is for the plain search");
+    // The fused search releases the next kernel only after its split (below).  Released at the
+    // start, the next kernel's CTAs (the gather's) take the SMs' spare room for the whole search
+    // and wait there: the 5k-token step measured 253 us that way against 218 us.
+    if (kFused) grid_dependency_wait(); else pdl_prologue();
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_addr(smem_raw);
     const uint32_t sbase = (raw + 1023u) & ~1023u;
@@ -441,6 +457,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (kChecked && ew == 0 && lane == 0) chk[8] = chk[8] + 1u;
         }
         if (cur_tb >= 0) flush();
+        if (kFused) __threadfence();  // this thread's keys are in place before the CTA counts itself
     }
 
     tc_fence_before_sync();
@@ -454,6 +471,40 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 1) {
         tc_fence_after_sync();
         tmem_dealloc(tmem_base, 512);
+    }
+    if (kFused) {
+        // The last CTA to arrive has every key: it splits them into idx/dist and resets them.
+        // (No CTA waits for another: the others have finished when the last one counts itself.)
+        __shared__ bool last;
+        if (threadIdx.x == 0)
+            last = atomicAdd(a.counter, 1u) == static_cast<unsigned int>(gridDim.x) + kNoArrivals - 1u;
+        __syncthreads();
+        if (last) {
+            __threadfence();
+            // kSplitBatch keys per thread are loaded before any is written, so the split waits for
+            // L2 once per batch (a load per iteration would wait once per key)
+            constexpr int kSplitBatch = 16;
+            for (int64_t t0 = threadIdx.x; t0 < a.n_tgt; t0 += kSplitBatch * kThreads) {
+                unsigned long long k[kSplitBatch];
+#pragma unroll
+                for (int i = 0; i < kSplitBatch; ++i) {
+                    const int64_t t = t0 + static_cast<int64_t>(i) * kThreads;
+                    k[i] = t < a.n_tgt ? __ldcg(a.keys + t) : kNoKey;
+                }
+#pragma unroll
+                for (int i = 0; i < kSplitBatch; ++i) {
+                    const int64_t t = t0 + static_cast<int64_t>(i) * kThreads;
+                    if (t < a.n_tgt) {
+                        a.keys[t] = kNoKey;
+                        const bool none = k[i] == kNoKey;
+                        a.idx[t] = none ? -1 : static_cast<int32_t>(static_cast<uint32_t>(k[i]));
+                        if (a.dist) a.dist[t] = none ? -1 : static_cast<int32_t>(static_cast<uint32_t>(k[i] >> 32));
+                    }
+                }
+            }
+            if (threadIdx.x == 0) *a.counter = kNoArrivals;
+        }
+        grid_dependents_launch();  // every CTA, the last after its split
     }
 }
 
@@ -557,11 +608,16 @@ __global__ void retrieve_select_kernel(const unsigned long long* __restrict__ ke
 // Expand the codes and run the search; leaves keys[n_seg][n_tgt] in the workspace.  kSelect:
 // the reference rows are candidate *best of the pool (cand), n_ref its longest candidate, and
 // sel (two int64 in device memory) receives the candidate's length and first pool row.
+// Sign rows given (tsig/rsig, [n][kpad] bytes from semshare_hash_signs): no expansion; the keys
+// (and, with fused_idx, the arrival counter) must then hold kNoKey (kNoArrivals) on entry, and
+// with fused_idx the search's last CTA writes idx/dist and resets them.
 template <int kMaxSeg, bool kSelect = false>
 semshare_status launch_search(const uint32_t* tgt_codes, int64_t n_tgt, const uint32_t* ref_codes, int64_t n_ref,
                               int32_t nbits, const SegTable<kMaxSeg>& seg, const TcPlan& plan, void* workspace,
                               uint32_t* err_flag, cudaStream_t s, int sms, int dev, const int32_t* best = nullptr,
-                              const CandTableFor<kSelect>* cand = nullptr, int64_t* sel = nullptr) {
+                              const CandTableFor<kSelect>* cand = nullptr, int64_t* sel = nullptr,
+                              const uint8_t* tsig = nullptr, const uint8_t* rsig = nullptr, int32_t* fused_idx = nullptr,
+                              int32_t* fused_dist = nullptr, unsigned int* fused_counter = nullptr) {
     int smem_optin = 0;
     if (cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
         return SEMSHARE_ECUDA;
@@ -585,6 +641,15 @@ semshare_status launch_search(const uint32_t* tgt_codes, int64_t n_tgt, const ui
     a.n_ref_dev = kSelect ? sel : nullptr;
     a.err_flag = err_flag;
     a.wait_limit_ns = wait_limit_ns();
+    a.idx = fused_idx;
+    a.dist = fused_dist;
+    a.counter = fused_counter;
+    const bool signs = tsig != nullptr;
+    const bool fused = fused_idx != nullptr;
+    if (signs) {
+        tpm = const_cast<uint8_t*>(tsig);
+        rpm = const_cast<uint8_t*>(rsig);
+    }
     const size_t smem = kFixedSmem + 2 * static_cast<size_t>(a.a_bytes) + 2 * static_cast<size_t>(a.b_bytes);
     if (smem > static_cast<size_t>(smem_optin)) return SEMSHARE_EUNSUPPORTED;
 
@@ -594,9 +659,16 @@ semshare_status launch_search(const uint32_t* tgt_codes, int64_t n_tgt, const ui
         !encode_tma_2d(&tm_r, CU_TENSOR_MAP_DATA_TYPE_UINT8, rpm, static_cast<uint64_t>(plan.kpad),
                        static_cast<uint64_t>(n_ref), static_cast<uint64_t>(plan.kpad), kChunk, kTN))
         return SEMSHARE_ECUDA;
-    if (cudaFuncSetAttribute(hamming_tc_kernel<kMaxSeg>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(smem)) != cudaSuccess)
+    auto kernel = fused ? hamming_tc_kernel<kMaxSeg, kMaxSeg == 1> : hamming_tc_kernel<kMaxSeg, false>;
+    if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) != cudaSuccess)
         return SEMSHARE_ECUDA;
+    const int64_t grid = a.total < sms ? a.total : sms;
+    if (signs) {
+        if (launch_pdl(kernel, dim3(static_cast<unsigned>(grid)), dim3(kThreads), smem, s, tm_t, tm_r, a, seg) !=
+            cudaSuccess)
+            return SEMSHARE_ECUDA;
+        return launch_status();
+    }
 
     const int64_t pieces = (n_tgt + n_ref) * (plan.kpad / 16);
     const int64_t eg = (pieces + 255) / 256;
@@ -605,9 +677,8 @@ semshare_status launch_search(const uint32_t* tgt_codes, int64_t n_tgt, const ui
                    s, tgt_codes, n_tgt, ref_codes, n_ref, nbits, plan.kpad, tpm, rpm, keys, n_tgt * seg.n_seg, counter,
                    best, cand ? *cand : none, sel, err_flag) != cudaSuccess)
         return SEMSHARE_ECUDA;
-    const int64_t grid = a.total < sms ? a.total : sms;
-    if (launch_pdl(hamming_tc_kernel<kMaxSeg>, dim3(static_cast<unsigned>(grid)), dim3(kThreads), smem, s, tm_t, tm_r, a,
-                   seg) != cudaSuccess)
+    if (launch_pdl(kernel, dim3(static_cast<unsigned>(grid)), dim3(kThreads), smem, s, tm_t, tm_r, a, seg) !=
+        cudaSuccess)
         return SEMSHARE_ECUDA;
     return launch_status();
 }
@@ -651,8 +722,53 @@ extern "C" semshare_status semshare_match_tc(const uint32_t* tgt_codes, int64_t 
                                              err_flag, s, sms, dev);
     if (st != SEMSHARE_OK) return st;
     const int small = static_cast<int>((n_tgt + 255) / 256 < sms * 4 ? (n_tgt + 255) / 256 : sms * 4);
-    if (launch_pdl(tc_keys_split_kernel, dim3(small), dim3(256), 0, s, static_cast<const unsigned long long*>(workspace),
-                   n_tgt, idx, dist, static_cast<const int64_t*>(nullptr)) != cudaSuccess)
+    if (launch_pdl(tc_keys_split_kernel, dim3(small), dim3(256), 0, s, static_cast<unsigned long long*>(workspace),
+                   n_tgt, idx, dist, static_cast<const int64_t*>(nullptr), false) != cudaSuccess)
+        return SEMSHARE_ECUDA;
+    return launch_status();
+}
+
+extern "C" size_t semshare_match_tc_signs_workspace_size(int64_t n_tgt) {
+    using namespace semshare;
+    if (n_tgt <= 0) return 0;
+    return round256(static_cast<size_t>(n_tgt) * 8) + 256;  // keys, then the arrival counter
+}
+
+extern "C" semshare_status semshare_match_tc_signs(const uint8_t* tgt_signs, int64_t n_tgt, const uint8_t* ref_signs,
+                                                   int64_t n_ref, int32_t nbits, int32_t* idx, int32_t* dist,
+                                                   void* workspace, size_t workspace_bytes, uint32_t* err_flag,
+                                                   void* stream) {
+    using namespace semshare;
+    if (n_tgt < 0 || n_ref < 1) return SEMSHARE_EINVAL;
+    if (nbits < 32 || nbits > 256 || nbits % 32 != 0) return SEMSHARE_EUNSUPPORTED;
+    if (n_tgt >= (int64_t(1) << 31) || n_ref >= (int64_t(1) << 31)) return SEMSHARE_EUNSUPPORTED;
+    if (n_tgt == 0) return SEMSHARE_OK;
+    if (!tgt_signs || !ref_signs || !idx || !workspace) return SEMSHARE_EINVAL;
+    if (!aligned(tgt_signs, 16) || !aligned(ref_signs, 16) || !aligned(idx, 4) || !aligned(workspace, 256) ||
+        (dist && !aligned(dist, 4)) || (err_flag && !aligned(err_flag, 4)))
+        return SEMSHARE_EINVAL;
+    if (workspace_bytes < semshare_match_tc_signs_workspace_size(n_tgt)) return SEMSHARE_EINVAL;
+    TcPlan plan;
+    plan_tc(n_tgt, n_ref, nbits, 0, &plan);
+
+    int sms = 0, dev = 0;
+    if (current_sm_count(&sms, &dev) != SEMSHARE_OK) return SEMSHARE_ECUDA;
+    cudaStream_t s = as_stream(stream);
+    SegTable<1> seg{};
+    seg.n_seg = 1;
+    seg.off[0] = 0;
+    seg.off[1] = n_ref;
+    auto* keys = static_cast<unsigned long long*>(workspace);
+    auto* counter = reinterpret_cast<unsigned int*>(static_cast<uint8_t*>(workspace) + round256(static_cast<size_t>(n_tgt) * 8));
+    const bool fused = n_tgt <= kFusedSplitMaxTargets;
+    const semshare_status st = launch_search(static_cast<const uint32_t*>(nullptr), n_tgt,
+                                             static_cast<const uint32_t*>(nullptr), n_ref, nbits, seg, plan, workspace,
+                                             err_flag, s, sms, dev, nullptr, nullptr, nullptr, tgt_signs, ref_signs,
+                                             fused ? idx : nullptr, fused ? dist : nullptr, fused ? counter : nullptr);
+    if (st != SEMSHARE_OK || fused) return st;
+    const int small = static_cast<int>((n_tgt + 255) / 256 < sms * 4 ? (n_tgt + 255) / 256 : sms * 4);
+    if (launch_pdl(tc_keys_split_kernel, dim3(small), dim3(256), 0, s, keys, n_tgt, idx, dist,
+                   static_cast<const int64_t*>(nullptr), true) != cudaSuccess)
         return SEMSHARE_ECUDA;
     return launch_status();
 }
@@ -719,8 +835,8 @@ extern "C" semshare_status semshare_match_tc_selected(const uint32_t* tgt_codes,
                                                       err_flag, s, sms, dev, best, &cand, sel);
     if (st != SEMSHARE_OK) return st;
     const int small = static_cast<int>((n_tgt + 255) / 256 < sms * 4 ? (n_tgt + 255) / 256 : sms * 4);
-    if (launch_pdl(tc_keys_split_kernel, dim3(small), dim3(256), 0, s, static_cast<const unsigned long long*>(workspace),
-                   n_tgt, idx, dist, static_cast<const int64_t*>(sel)) != cudaSuccess)
+    if (launch_pdl(tc_keys_split_kernel, dim3(small), dim3(256), 0, s, static_cast<unsigned long long*>(workspace),
+                   n_tgt, idx, dist, static_cast<const int64_t*>(sel), false) != cudaSuccess)
         return SEMSHARE_ECUDA;
     return launch_status();
 }

@@ -137,6 +137,35 @@ def test_hash_pair_argument_errors(lib):
     assert lib.semshare_hash_pair_workspace_size(0, 128, 64) == 0
 
 
+def test_hash_signs_argument_errors(lib):
+    hs = lib.semshare_hash_signs
+    odd = ctypes.c_void_p((1 << 20) + 8)
+
+    def call(signs=FAKE, n=10, layout=0, codes2_like=None):
+        return hs(FAKE, 0, n, 128, 128, None, FAKE, FAKE, 64, layout, FAKE, signs, None, FAKE, 1 << 30, None, None)
+
+    assert call(signs=None) == 1                       # the sign rows are the point of the call
+    assert call(signs=odd) == 1                        # not 16-byte aligned
+    assert call(layout=3) == 1
+    assert call(n=0, signs=None) == 0                  # empty
+    assert [lib.semshare_signs_pitch(b) for b in (32, 64, 96, 128, 160, 256)] == [128, 128, 128, 128, 256, 256]
+    assert lib.semshare_signs_pitch(48) == 0 and lib.semshare_signs_pitch(288) == 0
+
+
+def test_match_tc_signs_argument_errors(lib):
+    m = lib.semshare_match_tc_signs
+    odd = ctypes.c_void_p((1 << 20) + 8)
+    ws = lib.semshare_match_tc_signs_workspace_size(10)
+    assert ws == 256 + 256                              # 10 keys rounded to 256 bytes, then the counter
+    assert lib.semshare_match_tc_signs_workspace_size(0) == 0
+    assert m(FAKE, 10, FAKE, 0, 64, FAKE, None, FAKE, ws, None, None) == 1      # n_ref = 0
+    assert m(FAKE, 10, FAKE, 5, 40, FAKE, None, FAKE, ws, None, None) == 2      # nbits
+    assert m(FAKE, 10, FAKE, 5, 64, FAKE, None, FAKE, ws - 1, None, None) == 1  # workspace too small
+    assert m(odd, 10, FAKE, 5, 64, FAKE, None, FAKE, ws, None, None) == 1       # TMA rows: 16-byte aligned
+    assert m(FAKE, 10, FAKE, 5, 64, None, None, FAKE, ws, None, None) == 1
+    assert m(None, 0, FAKE, 5, 64, None, None, None, 0, None, None) == 0        # empty target
+
+
 def test_match_argument_errors(lib):
     m = lib.semshare_match
     assert m(FAKE, 10, FAKE, 0, 64, FAKE, None, FAKE, 80, None) == 1   # n_ref = 0
