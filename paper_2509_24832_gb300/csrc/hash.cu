@@ -41,6 +41,8 @@
 // value and its partner's: y = x*c - x_partner*s in the first half, x*c + x_partner*s in the
 // second, at angle index (column mod d/2).  The hyperplane tiles and the MMA are unchanged.
 #include <cuda.h>
+
+#include <cstring>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
 
@@ -879,6 +881,21 @@ extern "C" size_t semshare_hash_workspace_size(int64_t n, int32_t d, int32_t nbi
 namespace semshare {
 namespace {
 
+// bf16 rows with the interleaved pairing (or none) run on SM pairs unless the call is small: below
+// 8 stages (256-row pair tile x 64-wide K block) per SM pair the pair kernel's pipeline fill and end
+// phase outweigh its faster stages (on GB300, 2048 rows x 4096: 27.3 us on pairs against 25.2 us on
+// single SMs; 4096 rows: equal; 10240 rows: 41.6 against 47.7 us).  SEMSHARE_HASH_KERNEL=pair|one
+// (read per call, a test knob) forces one of the two.
+bool use_pair_kernel(int64_t rows, int32_t d) {
+    const char* e = getenv("SEMSHARE_HASH_KERNEL");
+    if (e != nullptr && strcmp(e, "pair") == 0) return true;
+    if (e != nullptr && strcmp(e, "one") == 0) return false;
+    int sms = 0;
+    if (current_sm_count(&sms, nullptr) != SEMSHARE_OK) return true;
+    const int64_t stages = ((rows + 255) / 256) * (d / kBK);
+    return stages >= 4 * static_cast<int64_t>(sms);
+}
+
 // semshare_hash_ex, and with codes2 non-null semshare_hash_pair (the rows as they are into codes,
 // rotated into codes2, in one launch over twice the tiles).
 semshare_status hash_impl(const void* emb, semshare_dtype dtype, int64_t n, int32_t d, int64_t row_stride,
@@ -916,7 +933,7 @@ semshare_status hash_impl(const void* emb, semshare_dtype dtype, int64_t n, int3
     HashPlan plan;
     if (plan_hash(pair ? 2 * n_pad : n, d, &plan) != SEMSHARE_OK) return SEMSHARE_ECUDA;
     if (workspace_bytes < plan.partial_bytes + plan.count_bytes) return SEMSHARE_EINVAL;
-    if (dtype == SEMSHARE_BF16 && !half) {
+    if (dtype == SEMSHARE_BF16 && !half && use_pair_kernel(pair ? 2 * n : n, d)) {
         // bf16 rows, interleaved pairing or none: the CTA-pair kernel (hash_2sm.cu)
         Hash2smCall c{};
         c.emb = emb;

@@ -40,6 +40,7 @@ def run(dev) -> dict:
     hyp = bf16(g.standard_normal((nbits, d)), dev)
     pos = torch.from_numpy((np.arange(n) % 1500).astype(np.int32)).to(dev)
     table = ss.semshare_rope_table(d, device=dev)
+    os.environ["SEMSHARE_HASH_KERNEL"] = "pair"  # a call this small would otherwise go to the one-SM kernel
     for cl in ("", "3", "37"):
         if cl:
             os.environ["SEMSHARE_HASH_CLUSTERS"] = cl
@@ -51,6 +52,7 @@ def run(dev) -> dict:
     # the pair call (plain and rotary codes in one launch)
     cp, cr = ss.semshare_hash_pair(emb[:513].contiguous(), table, hyp, pos[:513].contiguous(), err_flag=flag())
     out["pair_plain"], out["pair_rotary"] = cp, cr
+    os.environ.pop("SEMSHARE_HASH_KERNEL", None)
     # the one-SM kernel: fp32 rows, and the rotate-half pairing
     e32 = torch.from_numpy(g.standard_normal((700, 512)).astype(np.float32)).to(dev)
     h128 = bf16(g.standard_normal((128, 512)), dev)

@@ -1,9 +1,9 @@
-"""The bf16 hash on CTA pairs (hash_2sm.cu): the stream-K split over clusters must not change
-what is computed.  With the cluster count lowered through SEMSHARE_HASH_CLUSTERS (1, odd counts
-that leave one cluster straddling tiles, and counts above the tile count), the codes and
-projections must satisfy the oracle's rules, and the pair call (plain + rotated codes in one
-launch) must equal the two separate calls even when a cluster's range crosses from the plain
-into the rotated half."""
+"""The bf16 hash on CTA pairs (hash_2sm.cu, forced with SEMSHARE_HASH_KERNEL=pair at these
+sizes): the stream-K split over clusters must not change what is computed.  With the cluster
+count lowered through SEMSHARE_HASH_CLUSTERS (1, odd counts that leave one cluster straddling
+tiles, and counts above the tile count), the codes and projections must satisfy the oracle's
+rules, and the pair call (plain + rotated codes in one launch) must equal the two separate calls
+even when a cluster's range crosses from the plain into the rotated half."""
 import numpy as np
 import pytest
 
@@ -22,6 +22,12 @@ def ss():
 
     ss.load()
     return ss
+
+
+@pytest.fixture(autouse=True)
+def _pair_kernel(monkeypatch):
+    # these sizes are below the pair kernel's dispatch threshold: force it
+    monkeypatch.setenv("SEMSHARE_HASH_KERNEL", "pair")
 
 
 def _inputs(n, d, nbits, seed):

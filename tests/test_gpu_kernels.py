@@ -386,10 +386,14 @@ def test_wait_timeout_reports_status_and_context_survives(ss, orc, monkeypatch):
                      device="cuda")
     codes = torch.empty((len(emb), wl.nbits // 32), dtype=torch.int32, device="cuda")
     monkeypatch.setenv("SEMSHARE_WAIT_LIMIT_NS", "1")
-    flag = ss.new_err_flag()
-    ss.semshare_hash(e, table, R, p, codes=codes, workspace=ws, err_flag=flag)
-    torch.cuda.synchronize()
-    assert ss.flag_status(flag) == 5  # SEMSHARE_ETIMEOUT
+    for kernel in ("pair", "one"):  # the bf16 hash on SM pairs and on single SMs
+        monkeypatch.setenv("SEMSHARE_HASH_KERNEL", kernel)
+        ws.zero_()
+        flag = ss.new_err_flag()
+        ss.semshare_hash(e, table, R, p, codes=codes, workspace=ws, err_flag=flag)
+        torch.cuda.synchronize()
+        assert ss.flag_status(flag) == 5, kernel  # SEMSHARE_ETIMEOUT
+    monkeypatch.delenv("SEMSHARE_HASH_KERNEL")
     tgt, ref = codes[wl.n_ref:], codes[: wl.n_ref]
     flag2 = ss.new_err_flag()
     ss.semshare_match_tc(tgt, ref, err_flag=flag2)

@@ -62,6 +62,7 @@ def _hash_inputs(n, d, nbits, dtype, seed):
 def test_hash_signs_are_the_expanded_codes(ss, monkeypatch, n, d, nbits, dtype, layout, clusters):
     if clusters:
         monkeypatch.setenv("SEMSHARE_HASH_CLUSTERS", clusters)
+        monkeypatch.setenv("SEMSHARE_HASH_KERNEL", "pair")  # below the pair kernel's dispatch threshold
     emb, hyp, pos = _hash_inputs(n, d, nbits, dtype, seed=n + nbits)
     table = ss.semshare_rope_table(d)
     flag = ss.new_err_flag()
