@@ -34,7 +34,10 @@ inline semshare_status current_sm_count(int* sms, int* device) {
 __device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void grid_dependents_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
-// Every kernel of the library starts with this pair: nothing before it touches global memory.
+// Every kernel of the library starts with grid_dependency_wait: nothing before it touches global
+// memory.  The short kernels release their dependents right away (pdl_prologue); the persistent
+// ones that fill every SM (the hash kernels, the tensor-core search) release them only at their
+// end, since dependents released early queue behind them for their whole run (measured slower).
 __device__ __forceinline__ void pdl_prologue() {
     grid_dependency_wait();
     grid_dependents_launch();

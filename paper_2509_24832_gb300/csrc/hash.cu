@@ -201,7 +201,8 @@ template <bool kHalf, int kRot>
 __global__ void __launch_bounds__(kThreads, 1)
     lsh_hash_kernel(const __grid_constant__ CUtensorMap tmap_emb, const __grid_constant__ CUtensorMap tmap_hyp,
                     const HashArgs a) {
-    pdl_prologue();
+    // the next kernel is released at the end (below), as in hash_2sm.cu
+    grid_dependency_wait();
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_addr(smem_raw);
     const uint32_t sbase = (raw + 1023u) & ~1023u;  // stage tiles on the swizzle-atom boundary
@@ -832,6 +833,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 
     __syncthreads();
+    grid_dependents_launch();  // every CTA, at its end
     if (warp == 1) {
         tc_fence_after_sync();
         tmem_dealloc(tmem_base, a.tmem_cols);

@@ -224,7 +224,10 @@ template <int kRot>
 __global__ void __launch_bounds__(kThreads, 1)
     lsh_hash_2sm_kernel(const __grid_constant__ CUtensorMap tmap_emb, const __grid_constant__ CUtensorMap tmap_hyp,
                         const Hash2smArgs a) {
-    pdl_prologue();
+    // The next kernel is released at the end (below), not here: released at the start, its CTAs
+    // queued behind this grid for its whole run and the batched step (135 K rows, then the match
+    // and the gather) measured 3.04 ms against 2.91 ms.
+    grid_dependency_wait();
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_addr(smem_raw);
     const uint32_t sbase = (raw + 1023u) & ~1023u;  // stage tiles on the swizzle-atom boundary
@@ -857,6 +860,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after_sync();
         tmem_dealloc_pair(tmem_base, kTmemCols);
     }
+    grid_dependents_launch();  // every CTA, after it has freed its tensor memory
 }
 
 // Clusters of the launch: as many pairs as can be resident at once (one CTA per SM), no more
