@@ -127,12 +127,11 @@ __device__ __forceinline__ uint32_t* ptile_codes(const Hash2smArgs& a, int64_t t
     return (kRot == kRotPair && tile * kPM >= a.pair_rows) ? a.codes2 : a.codes;
 }
 
-// Workspace slot of cluster b's partial of CTA half `rank` of the tile whose first iteration is
-// tile_it0: two slots per CTA, the first for a segment that starts the CTA's range (the only kind
-// this kernel publishes), the second for a later one.
-__device__ __forceinline__ int64_t partial_slot(int64_t b, uint32_t rank, int64_t tile_it0, int64_t total, int64_t P) {
-    return 2 * (2 * b + rank) + (range_begin(b, total, P) >= tile_it0 ? 0 : 1);
-}
+// Workspace slot of cluster b's partial of CTA half `rank`.  The workspace plan has two slots per
+// CTA; this kernel uses the first only: a cluster publishes a partial only for a segment that
+// starts its range inside a tile (the tile's first K block belongs to an earlier cluster, its
+// closer), so every partial of a shared tile comes from a different cluster.
+__device__ __forceinline__ int64_t partial_slot(int64_t b, uint32_t rank) { return 2 * (2 * b + rank); }
 
 // phi: the rows of one half warp's threads fall on swizzle phases 0,2,4,6 and 1,3,5,7.
 __device__ __forceinline__ int row_phase(int i) { return i < 4 ? 2 * i : 2 * i - 7; }
@@ -711,7 +710,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             } else {
                 // the CTA's first segment, the tail of a tile another cluster started: publish this
                 // half's partial and count it
-                float4* dst = a.partials + partial_slot(pid, rank, tile_it0, a.total_iters, P) * items;
+                float4* dst = a.partials + partial_slot(pid, rank) * items;
 #pragma unroll
                 for (int qq = 0; qq < 8; ++qq) {
                     if (qq < W) {
@@ -768,7 +767,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t taddr = tmem_base + (static_cast<uint32_t>((warp & 3) * 32) << 16);
         const int q0 = 2 * (warp >> 2);
         if (dkind == 1) {
-            float4* dst = a.partials + partial_slot(pid, rank, tile_it0, a.total_iters, P) * items;
+            float4* dst = a.partials + partial_slot(pid, rank) * items;
 #pragma unroll
             for (int qi = 0; qi < 2; ++qi) {
                 const int qq = q0 + qi;
@@ -812,7 +811,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const float4* pp = a.partials + qq * 8 * kCM + r;
                     float4 f0[4];
                     if (b_hi > b_lo) {
-                        const float4* p0 = pp + partial_slot(b_lo + 1, rank, tile_it0, a.total_iters, P) * items;
+                        const float4* p0 = pp + partial_slot(b_lo + 1, rank) * items;
 #pragma unroll
                         for (int j = 0; j < 4; ++j) f0[j] = __ldcg(p0 + j * kCM);
                     }
@@ -822,7 +821,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int j = 0; j < 32; ++j) sum[j] = __uint_as_float(v[j]);
                     for (int64_t bb = b_lo + 1; bb <= b_hi; ++bb) {
-                        const float4* p0 = pp + partial_slot(bb, rank, tile_it0, a.total_iters, P) * items;
+                        const float4* p0 = pp + partial_slot(bb, rank) * items;
 #pragma unroll
                         for (int h = 0; h < 8; h += 4) {
                             if (h > 0 || bb > b_lo + 1) {
