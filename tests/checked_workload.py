@@ -71,6 +71,13 @@ def run(dev) -> dict:
     out["ret_mean"], out["ret_best"], out["ret_idx"] = r.mean_dist, r.best, r.idx
     si, sd = ss.semshare_match_tc_selected(tgt[:900].contiguous(), ref, offs, r.best, err_flag=flag())
     out["sel_idx"], out["sel_dist"] = si, sd
+    # the sign rows of the hash and the one-launch search on them (its last CTA splits the keys)
+    os.environ["SEMSHARE_HASH_KERNEL"] = "pair"
+    sc, signs = ss.semshare_hash_signs(emb, table, hyp, pos, err_flag=flag())
+    os.environ.pop("SEMSHARE_HASH_KERNEL", None)
+    out["signs_codes"], out["signs"] = sc, signs
+    si2, sd2 = ss.semshare_match_tc_signs(signs[1200:], signs[:1200], nbits, err_flag=flag())
+    out["signs_idx"], out["signs_dist"] = si2, sd2
     torch.cuda.synchronize()
     for i, f in enumerate(flags):
         v = int(f.item()) & 0xFFFFFFFF

@@ -89,3 +89,26 @@ def test_positions_not_32_apart(ss, oracle_mod):
     ss.check_flag(flag, "hash")
     oc, op = oracle_mod.hash_codes(emb, pos, R)
     check_hash(codes_host(codes), proj.cpu().numpy(), oc, op)
+
+
+@pytest.mark.parametrize("n,d,nbits", [(2048, 4096, 128), (2432, 4096, 256), (600, 512, 64)])
+def test_dispatch_either_kernel_keeps_parity(ss, oracle_mod, monkeypatch, n, d, nbits):
+    # bf16 calls below 8 stages per SM pair go to the one-SM kernel; 2432 rows x 4096 is 10 pair
+    # tiles x 64 K blocks = 640 stages, just above the threshold on 152 SMs.  Whichever kernel the
+    # dispatch picks, and either one forced, the codes and projections follow the oracle's rules.
+    emb, R = _inputs(n, d, nbits, seed=n + d)
+    pos = np.arange(n, dtype=np.int32)
+    oc, op = oracle_mod.hash_codes(emb, pos, R)
+    table = ss.semshare_rope_table(d)
+    for kernel in ("", "pair", "one"):
+        if kernel:
+            monkeypatch.setenv("SEMSHARE_HASH_KERNEL", kernel)
+        else:
+            monkeypatch.delenv("SEMSHARE_HASH_KERNEL", raising=False)
+        proj = torch.empty((n, nbits), dtype=torch.float32, device="cuda")
+        flag = ss.new_err_flag()
+        codes = ss.semshare_hash(emb_dev(emb), table, bf16_dev(R), torch.from_numpy(pos).cuda(), proj_out=proj,
+                                 err_flag=flag)
+        torch.cuda.synchronize()
+        assert int(flag.item()) == 0, kernel
+        check_hash(codes_host(codes), proj.cpu().numpy(), oc, op)
