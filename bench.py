@@ -47,6 +47,21 @@ DEFAULT_WORKLOAD = "llama8b-5k"
 ALL_WORKLOADS = {**workloads.WORKLOADS, **workloads.RETRIEVAL_WORKLOADS}
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 L2_FLUSH_BYTES = 512 << 20
+NVTX = [False]  # --nvtx: stage ranges on the timeline
+
+
+def nvtx_push(name: str):
+    if NVTX[0]:
+        import torch
+
+        torch.cuda.nvtx.range_push(name)
+
+
+def nvtx_pop():
+    if NVTX[0]:
+        import torch
+
+        torch.cuda.nvtx.range_pop()
 
 # DRAM bytes per launch from ncu captures (dram__bytes_read.sum + dram__bytes_write.sum) on a
 # workload, valid only for that workload and while the kernel source has the recorded sha256
@@ -85,6 +100,8 @@ def parse_args(argv=None):
                         "enqueues one graph instead of the library calls)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-clocks", action="store_true")
+    p.add_argument("--nvtx", action="store_true",
+                   help="name each stage of a step with an NVTX range (for a profiler's timeline)")
     return p.parse_args(argv)
 
 
@@ -414,24 +431,15 @@ class Problem:
                                    out_k=self.out_k, out_v=self.out_v, err_flag=self.flag)
 
     def step(self, ev=None):
+        stages = [self.hash, self.match, self.gather] + ([self.deviation, self.select] if self.hd else [])
         if ev:
             ev[0].record()
-        self.hash()
-        if ev:
-            ev[1].record()
-        self.match()
-        if ev:
-            ev[2].record()
-        self.gather()
-        if ev:
-            ev[3].record()
-        if self.hd:
-            self.deviation()
+        for i, (name, fn) in enumerate(zip(self.STAGES, stages)):
+            nvtx_push(name)
+            fn()
+            nvtx_pop()
             if ev:
-                ev[4].record()
-            self.select()
-            if ev:
-                ev[5].record()
+                ev[i + 1].record()
 
     def unique_rows(self) -> int:
         """Distinct reference rows the current match selects (over every target prompt)."""
@@ -615,16 +623,23 @@ class RetrieveProblem:
         ss, wl = self.ss, self.wl
         if ev:
             ev[0].record()
+        nvtx_push("hash")
         ss.semshare_hash_pair(self.emb, self.table, self.hyp, self.pos, codes_plain=self.t_rcodes,
                               codes_rotary=self.codes, err_flag=self.flag, workspace=self.hash_ws)
+        nvtx_pop()
         if ev:
             ev[1].record()
+        nvtx_push("retrieve")
         ss.semshare_retrieve(self.t_rcodes, self.pool_rcodes, self.offsets, workspace=self.ret_ws,
                              err_flag=self.flag, out=self.ret)
+        nvtx_pop()
         if ev:
             ev[2].record()
+        nvtx_push("match")
         ss.semshare_match_tc_selected(self.codes, self.pool_codes, self.offsets, self.ret.best, idx=self.idx,
                                       dist=self.dist, workspace=self.tc_ws, err_flag=self.flag)
+        nvtx_pop()
+        nvtx_push("gather")
         if self.fetch_gather is not None:
             # e2e fetch mode: the rows come in from host memory and are gathered, in layer groups
             self.fetch_gather()
@@ -636,6 +651,7 @@ class RetrieveProblem:
             src_k, src_v = (self.ref_k, self.ref_v) if self.gather_src is None else self.gather_src
             ss.semshare_gather_kv(src_k, src_v, self.idx.view(1, wl.n_tgt), out_k=self.out_k, out_v=self.out_v,
                                   err_flag=self.flag)
+        nvtx_pop()
         if ev:
             ev[4].record()
         self.h_choice.copy_(self.choice, non_blocking=True)  # best, applies
@@ -1382,6 +1398,7 @@ def run_reference_arm(args, rank, world):
 
 def main(argv=None):
     args = parse_args(argv)
+    NVTX[0] = args.nvtx
     rank, world, local_rank = dist_info()
     if world > 1:
         import torch.distributed as dist
