@@ -66,6 +66,37 @@ def test_every_declared_symbol_is_exported(lib, probe_lib):
         assert not hasattr(lib, n), f"{n} is measurement support: it belongs to libsemshare_probe.so only"
 
 
+def test_headers_are_plain_c_and_every_declaration_links(lib, probe_lib, tmp_path):
+    """A C99 program that includes both headers and takes the address of every declared entry
+    point compiles warning-free with -pedantic and links against the two libraries: the C ABI is
+    plain C (no C++ types leak into it) and each declaration resolves to an exported symbol."""
+    import shutil
+    import subprocess
+
+    from paper_2509_24832_gb300 import build
+
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    names = _declared("semshare.h") + _declared("semshare_probe.h")
+    src = tmp_path / "abi.c"
+    src.write_text('#include "semshare.h"\n#include "semshare_probe.h"\n#include <stdio.h>\n'
+                   "int main(void) {\n    void (*volatile p)(void) = 0;\n"
+                   + "".join(f"    p = (void (*)(void)){n}; printf(\"%p\\n\", (void*)p);\n" for n in names)
+                   + "    return 0;\n}\n")
+    libdir = os.path.dirname(build.LIB)
+    out = tmp_path / "abi"
+    r = subprocess.run([cc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror", "-Wno-pedantic",
+                        "-I", os.path.join(ROOT, "include"), str(src), "-o", str(out), "-L", libdir,
+                        "-lsemshare", "-lsemshare_probe", f"-Wl,-rpath,{libdir}"],
+                       capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    r = subprocess.run([cc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-fsyntax-only",
+                        "-I", os.path.join(ROOT, "include"), "-x", "c", "-"],
+                       input='#include "semshare.h"\n#include "semshare_probe.h"\n', capture_output=True, text=True)
+    assert r.returncode == 0 and not r.stderr.strip(), r.stderr
+
+
 def test_status_helpers(lib):
     assert lib.semshare_abi_version() == 1
     assert lib.semshare_status_string(0) == b"ok"
