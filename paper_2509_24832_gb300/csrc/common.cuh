@@ -34,10 +34,11 @@ inline semshare_status current_sm_count(int* sms, int* device) {
 __device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void grid_dependents_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
-// Every kernel of the library starts with grid_dependency_wait: nothing before it touches global
-// memory.  The short kernels release their dependents right away (pdl_prologue); the persistent
-// ones that fill every SM (the hash kernels, the tensor-core search) release them only at their
-// end, since dependents released early queue behind them for their whole run (measured slower).
+// Every kernel of the library calls grid_dependency_wait before it touches global memory: most as
+// their first statement, the tensor-core search after its shared- and tensor-memory set-up.  The
+// short kernels release their dependents right away (pdl_prologue); the persistent ones that fill
+// every SM (the hash kernels, the tensor-core search) release them only at their end, since
+// dependents released early queue behind them for their whole run (measured slower).
 __device__ __forceinline__ void pdl_prologue() {
     grid_dependency_wait();
     grid_dependents_launch();
@@ -45,7 +46,7 @@ __device__ __forceinline__ void pdl_prologue() {
 
 // Launches kernel<<<grid, block, smem, s>>>(args...) as a programmatic dependent of the work
 // before it in the stream: its CTAs may be scheduled while the previous kernel drains, and they
-// wait (griddepcontrol.wait, first thing in every kernel of the library) until it has completed.
+// wait (griddepcontrol.wait, before any global memory access) until it has completed.
 template <typename... KArgs, typename... Args>
 inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
                               Args&&... args) {

@@ -185,7 +185,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     // start, its CTAs queue behind this persistent grid for its whole run (the 5k-token step with
     // the fused search measured 253 us that way against 218 us; the batched step 2.91 against
     // 2.89 ms with the plain search).
-    grid_dependency_wait();
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_addr(smem_raw);
     const uint32_t sbase = (raw + 1023u) & ~1023u;
@@ -233,6 +232,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_before_sync();
     __syncthreads();
     tc_fence_after_sync();
+    // The set-up above touches only this CTA's shared and tensor memory, so it overlaps the
+    // previous kernel's drain; global memory is read and written only from here on.
+    grid_dependency_wait();
     const uint32_t tmem_base = *tmem_slot_ptr;
     const uint64_t lim = a.wait_limit_ns;
     uint32_t* const err = a.err_flag;
