@@ -20,9 +20,11 @@
 //
 // Work split (stream-K over pair tiles).  The n_ptiles x n_kblocks (256-row pair tile, 64-wide
 // K block) iterations are cut into one equal contiguous range per cluster; both CTAs of a
-// cluster walk the same range, each on its 128-row half.  Tiles shared by several clusters are
-// finished as in hash.cu: each contributor publishes its fp32 partial of its half, the last to
-// arrive adds them in K order and packs the signs.
+// cluster walk the same range, each on its 128-row half.  A tile shared by several clusters is
+// closed by the cluster that owns its first K blocks: every later contributor publishes the fp32
+// partial of its half and counts it; the closer waits (bounded) for the count, adds the partials
+// to its own accumulator in K order and packs the signs.  All clusters are resident at once (the
+// grid is the occupancy figure), so that wait depends only on work already running.
 //
 // Rotation layout.  A RoPE thread owns 4 rows 32 apart and 8 bf16 pairs of each (the .16x256b
 // tensor-memory store gives a thread lanes 8 apart and two adjacent columns of every 8-column
