@@ -10,7 +10,8 @@
 // e4m3 +-1 rows (zero-padded to a multiple of 128 bytes), multiplied as a GEMM with fp32
 // accumulation (every partial sum is a small integer, so the products are exact), and each
 // accumulator row is reduced on the fly to its best reference with the exact fp32 key
-// 256*dot - j (largest dot first, then lowest j within the 256-wide tile).  The best
+// 256*dot - j (largest dot first, then the lowest column j of the epilogue warp's 128-column
+// half of the tile).  The best
 // (distance << 32 | index) of a target over the tiles a CTA visits goes to a 64-bit atomicMin,
 // which is "smallest distance, then lowest index" whatever the split.
 //
@@ -34,6 +35,10 @@
 // chosen by a device value (the retrieval's `best`): the expand kernel reads the choice, expands
 // that candidate's rows and publishes its length and first pool row; the search, sized for the
 // longest candidate, masks the columns past that length; the split adds the first pool row.
+//
+// Sign-row mode (semshare_match_tc_signs).  The operands are the caller's e4m3 rows written by
+// semshare_hash_signs (no expand kernel); the search's last CTA to finish (an arrival counter, no
+// CTA waits for another) splits the keys into idx/dist and resets them for the next call.
 #include <cuda.h>
 
 #include "common.cuh"
