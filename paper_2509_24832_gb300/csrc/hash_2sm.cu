@@ -797,6 +797,27 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (close_ok) {
                 const int64_t row = ptile_src_row<kRot>(a, tile) + static_cast<int64_t>(rank) * kCM + lane_row(r);
                 uint32_t* const out_codes = ptile_codes<kRot>(a, tile);
+                // This CTA's K blocks (the tile's first) are in the accumulator; the later
+                // contributors' partials are added in K order.  They come through the raw embedding
+                // ring, idle now (its copies all landed before the barrier above): copy e = 8 qi + j
+                // (float4 j of the thread's word qi) sits at (e * kThreads + threadIdx.x) * 16 bytes.
+                // A contributor's sixteen copies are in flight together (cp.async holds no
+                // registers), the first contributor's while the accumulator is read.
+                const uint32_t stage0 = a_ring + static_cast<uint32_t>(threadIdx.x) * 16u;
+                const float4* const staged = reinterpret_cast<const float4*>(gbase + (a_ring - sbase)) + threadIdx.x;
+                auto request = [&](int64_t bb, int qi_lo, int qi_hi) {
+                    const float4* p0 = a.partials + partial_slot(bb, rank) * items + r;
+                    for (int qi = qi_lo; qi < qi_hi; ++qi) {
+                        const int qq = q0 + qi;
+                        if (qq < W) {
+#pragma unroll
+                            for (int j = 0; j < 8; ++j)
+                                cp_async_16(stage0 + static_cast<uint32_t>((8 * qi + j) * kThreads) * 16u,
+                                            p0 + (qq * 8 + j) * kCM);
+                        }
+                    }
+                };
+                if (b_hi > b_lo) request(b_lo + 1, 0, 2);
 #pragma unroll 1
                 for (int qi = 0; qi < 2; ++qi) {
                     const int qq = q0 + qi;
@@ -806,37 +827,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                             store_sign_pad(a.signs + row * a.signs_pitch + 32 * qq);
                         continue;
                     }
-                    // this CTA's K blocks (the tile's first) in the accumulator, then the later
-                    // contributors' partials in K order; the first four values of the first
-                    // contributor are requested before the accumulator is read, so that their L2
-                    // latency overlaps the tensor-memory load (more in flight spills registers)
-                    const float4* pp = a.partials + qq * 8 * kCM + r;
-                    float4 f0[4];
-                    if (b_hi > b_lo) {
-                        const float4* p0 = pp + partial_slot(b_lo + 1, rank) * items;
-#pragma unroll
-                        for (int j = 0; j < 4; ++j) f0[j] = __ldcg(p0 + j * kCM);
-                    }
                     uint32_t v[32];
                     tmem_load_32cols_sync(taddr + qq * 32, v);
                     float sum[32];
 #pragma unroll
                     for (int j = 0; j < 32; ++j) sum[j] = __uint_as_float(v[j]);
                     for (int64_t bb = b_lo + 1; bb <= b_hi; ++bb) {
-                        const float4* p0 = pp + partial_slot(bb, rank) * items;
+                        // a third contributor on: this word's copies again, into the slots its
+                        // previous values were read from
+                        if (bb > b_lo + 1) request(bb, qi, qi + 1);
+                        cp_async_wait_all();
 #pragma unroll
-                        for (int h = 0; h < 8; h += 4) {
-                            if (h > 0 || bb > b_lo + 1) {
-#pragma unroll
-                                for (int j = 0; j < 4; ++j) f0[j] = __ldcg(p0 + (h + j) * kCM);
-                            }
-#pragma unroll
-                            for (int j = 0; j < 4; ++j) {
-                                sum[4 * (h + j)] += f0[j].x;
-                                sum[4 * (h + j) + 1] += f0[j].y;
-                                sum[4 * (h + j) + 2] += f0[j].z;
-                                sum[4 * (h + j) + 3] += f0[j].w;
-                            }
+                        for (int j = 0; j < 8; ++j) {
+                            const float4 f = staged[(8 * qi + j) * kThreads];
+                            sum[4 * j] += f.x;
+                            sum[4 * j + 1] += f.y;
+                            sum[4 * j + 2] += f.z;
+                            sum[4 * j + 3] += f.w;
                         }
                     }
 #pragma unroll
@@ -915,7 +922,9 @@ semshare_status launch_hash_2sm(const Hash2smCall& c) {
     int a_slots = static_cast<int>(room / kABytes);
     if (a_slots > kMaxASlots) a_slots = kMaxASlots;
     a_slots -= a_slots % kRopeGroups;  // each slot belongs to one RoPE group
-    if (a_slots < 2) return SEMSHARE_EUNSUPPORTED;
+    // the ring must also hold the close's staging area: 16 copies of 16 bytes per thread
+    if (a_slots < 2 || static_cast<size_t>(a_slots) * kABytes < static_cast<size_t>(kThreads) * 16 * 16)
+        return SEMSHARE_EUNSUPPORTED;
     a.a_slots = a_slots;
     a.positions = c.positions;
     a.rope_table = c.rope_table;
