@@ -805,19 +805,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // registers), the first contributor's while the accumulator is read.
                 const uint32_t stage0 = a_ring + static_cast<uint32_t>(threadIdx.x) * 16u;
                 const float4* const staged = reinterpret_cast<const float4*>(gbase + (a_ring - sbase)) + threadIdx.x;
-                auto request = [&](int64_t bb, int qi_lo, int qi_hi) {
-                    const float4* p0 = a.partials + partial_slot(bb, rank) * items + r;
-                    for (int qi = qi_lo; qi < qi_hi; ++qi) {
-                        const int qq = q0 + qi;
-                        if (qq < W) {
+                // word qi's copies of contributor bb into the slots of word `slot_qi`
+                auto request = [&](int64_t bb, int qi, int slot_qi) {
+                    const float4* p0 = a.partials + partial_slot(bb, rank) * items + r + (q0 + qi) * 8 * kCM;
 #pragma unroll
-                            for (int j = 0; j < 8; ++j)
-                                cp_async_16(stage0 + static_cast<uint32_t>((8 * qi + j) * kThreads) * 16u,
-                                            p0 + (qq * 8 + j) * kCM);
-                        }
-                    }
+                    for (int j = 0; j < 8; ++j)
+                        cp_async_16(stage0 + static_cast<uint32_t>((8 * slot_qi + j) * kThreads) * 16u, p0 + j * kCM);
                 };
-                if (b_hi > b_lo) request(b_lo + 1, 0, 2);
+                const bool two_words = q0 + 1 < W;
+                if (b_hi > b_lo && q0 < W) {
+                    request(b_lo + 1, 0, 0);
+                    if (two_words) request(b_lo + 1, 1, 1);
+                }
+                // with a second later contributor, its word-1 copies go into word 0's slots as soon
+                // as word 0 is summed, and land while word 0 is packed and word 1's first partial added
+                bool w1_second_early = false;
 #pragma unroll 1
                 for (int qi = 0; qi < 2; ++qi) {
                     const int qq = q0 + qi;
@@ -833,18 +835,24 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int j = 0; j < 32; ++j) sum[j] = __uint_as_float(v[j]);
                     for (int64_t bb = b_lo + 1; bb <= b_hi; ++bb) {
-                        // a third contributor on: this word's copies again, into the slots its
-                        // previous values were read from
-                        if (bb > b_lo + 1) request(bb, qi, qi + 1);
+                        int slot_qi = qi;
+                        if (bb == b_lo + 2 && qi == 1 && w1_second_early)
+                            slot_qi = 0;  // requested after word 0
+                        else if (bb > b_lo + 1)
+                            request(bb, qi, qi);  // into the slots its previous values were read from
                         cp_async_wait_all();
 #pragma unroll
                         for (int j = 0; j < 8; ++j) {
-                            const float4 f = staged[(8 * qi + j) * kThreads];
+                            const float4 f = staged[(8 * slot_qi + j) * kThreads];
                             sum[4 * j] += f.x;
                             sum[4 * j + 1] += f.y;
                             sum[4 * j + 2] += f.z;
                             sum[4 * j + 3] += f.w;
                         }
+                    }
+                    if (qi == 0 && two_words && b_hi >= b_lo + 2) {
+                        request(b_lo + 2, 1, 0);
+                        w1_second_early = true;
                     }
 #pragma unroll
                     for (int j = 0; j < 32; ++j) v[j] = __float_as_uint(sum[j]);
