@@ -42,6 +42,7 @@
 // second, at angle index (column mod d/2).  The hyperplane tiles and the MMA are unchanged.
 #include <cuda.h>
 
+#include <cstdlib>
 #include <cstring>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -861,7 +862,15 @@ semshare_status plan_hash(int64_t n, int32_t d, HashPlan* p) {
     if (current_sm_count(&sms, nullptr) != SEMSHARE_OK) return SEMSHARE_ECUDA;
     p->n_tiles = (n + kBM - 1) / kBM;
     p->total_iters = p->n_tiles * (d / kBK);
-    p->grid = static_cast<int>(p->total_iters < sms ? p->total_iters : sms);
+    // SEMSHARE_HASH_CTAS (read per call, a test knob) lowers the number of CTAs, so that tests can
+    // make a CTA's range cross from the plain into the rotated tiles of a pair call
+    int ctas = sms;
+    const char* e = getenv("SEMSHARE_HASH_CTAS");
+    if (e != nullptr && *e != 0) {
+        const long v = strtol(e, nullptr, 10);
+        if (v >= 1 && v < sms) ctas = static_cast<int>(v);
+    }
+    p->grid = static_cast<int>(p->total_iters < ctas ? p->total_iters : ctas);
     p->partial_bytes = static_cast<size_t>(2) * sms * kBM * static_cast<size_t>(kMaxBits) * 4;
     // counters of 128-row tiles (this kernel) or of the two halves of 256-row pair tiles
     // (hash_2sm.cu): n_tiles + 4 words covers both, for single and pair calls

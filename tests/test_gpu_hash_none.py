@@ -1,7 +1,8 @@
 """semshare_hash_ex with SEMSHARE_ROPE_NONE (no rotation: the retrieval codes of Sec. 3.2) against
 the oracle's hash at position 0, where RoPE is the identity (Eq. 1 at m = 0): projections within
 1e-3 of the row's largest |p|, codes bit-exact outside that band; and bit-identical to the
-interleaved kernel given every position 0."""
+interleaved kernel given every position 0.  The pair call (plain and rotary codes in one launch)
+equals the two calls, on every SM and, for the one-SM kernel, on odd numbers of CTAs."""
 import numpy as np
 import pytest
 
@@ -86,3 +87,15 @@ def test_pair_equals_the_two_calls(ss, oracle_mod, n, d, nbits, dtype, pos):
                 _, op = oracle_mod.hash_codes(emb[rows], sub_pos, R)
                 band = np.abs(op) < 1e-3 * np.abs(op).max(axis=1, keepdims=True)
                 assert (band | ~diff[rows]).all(), "a bit outside the band differs between the launches"
+
+
+@pytest.mark.parametrize("ctas", ["1", "7", "33", "151"])
+@pytest.mark.parametrize("n,d,nbits,dtype,pos", [(700, 512, 128, "f32", "random"), (3000, 1024, 256, "bf16", "own")])
+def test_pair_call_on_one_sm_with_odd_grids(ss, oracle_mod, monkeypatch, ctas, n, d, nbits, dtype, pos):
+    """The one-SM kernel's pair call on fewer CTAs than SMs (SEMSHARE_HASH_CTAS), odd counts among
+    them: a CTA's range then runs from the last plain tiles into the first rotated ones, and the
+    rotation table entries of its next stage are fetched across that boundary.  The same checks
+    as the call on every SM."""
+    monkeypatch.setenv("SEMSHARE_HASH_CTAS", ctas)
+    monkeypatch.setenv("SEMSHARE_HASH_KERNEL", "one")
+    test_pair_equals_the_two_calls(ss, oracle_mod, n, d, nbits, dtype, pos)
